@@ -1,0 +1,509 @@
+#!/usr/bin/env python3
+"""Benchmark of the dMoE MoE-layer forward (one block-diffusion decoding step's MoE layer).
+
+Workload (one GPU): d=2048, 256 routed experts, top-8, expert SwiGLU intermediate 512, one
+shared expert of intermediate 512, one sequence x one diffusion block of 32 tokens, router
+bias 0.5*ln(1/rank), block routing with the coreset floor (p=0, "block top-k"); token
+routing and p=0.6 are measured beside it. A step is one full layer forward (router,
+Algorithm 1, dispatch, expert GEMMs, combine) through the C ABI.
+
+L2 honesty: the steps rotate over --sets independently seeded copies of the layer (weights,
+router and input), so consecutive steps never find their ~60 MB of expert weights in the
+129 MB L2. Steps are replayed from CUDA graphs (launch-bound otherwise).
+
+Prints one JSON line (rank 0). --impl reference times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+_CORES = len(os.sched_getaffinity(0)) if hasattr(os, "sched_getaffinity") else os.cpu_count()
+for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+    os.environ.setdefault(_v, str(_CORES))
+
+import numpy as np  # noqa: E402
+
+METRIC = "MoE-layer tokens/s (block routing, block size 32)"
+UNIT = "tokens/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def workload_shape(mode: str, top_p: float):
+    from dmoe_synth import LAYER, ROUTE_BLOCK, ROUTE_TOKEN
+    return LAYER.with_(mode=ROUTE_BLOCK if mode == "block" else ROUTE_TOKEN, top_p=top_p)
+
+
+def workload_name(shape) -> str:
+    mode = "block" if shape.mode == 1 else "token"
+    tail = f"_p{shape.top_p:g}" if shape.mode == 1 else ""
+    return (f"moe_layer_d{shape.d_model}_E{shape.n_experts}_k{shape.top_k}_I{shape.d_ff}"
+            f"_shared{shape.d_ff_shared}_B{shape.block_size}x{shape.n_blocks}_{mode}{tail}")
+
+
+def measured_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return json.load(f), "measured"
+    except OSError:
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+# ----------------------------------------------------------------------------- byte model
+def layer_bytes(shape, U: float) -> float:
+    """Algorithmic HBM bytes of one layer forward: the unique experts' and the shared
+    expert's bf16 weights once, the fp32 router weight and bias, x read and y written."""
+    d, E, I, Is, T = shape.d_model, shape.n_experts, shape.d_ff, shape.d_ff_shared, shape.T
+    return (U * 3 * d * I * 2 + 3 * d * Is * 2 + d * E * 4 + E * 4 + T * d * 2 * 2)
+
+
+def gate_up_bytes(shape, U: float) -> float:
+    """Algorithmic bytes of one gate/up launch: gate and up weights of the unique and shared
+    experts, the token rows read once, the bf16 SwiGLU output written."""
+    d, I, Is, T, k = shape.d_model, shape.d_ff, shape.d_ff_shared, shape.T, shape.top_k
+    return U * 2 * d * I * 2 + 2 * d * Is * 2 + T * d * 2 + (T * k * I + T * Is) * 2
+
+
+def layer_flops(shape) -> float:
+    d, E, I, Is, T, k = (shape.d_model, shape.n_experts, shape.d_ff, shape.d_ff_shared, shape.T,
+                         shape.top_k)
+    return 2 * T * (k * 3 * d * I + 3 * d * Is) + 2 * T * d * E
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons while the timed region runs."""
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_uuid: str | None):
+        self.uuid = gpu_uuid
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        cmd = ["nvidia-smi", f"--query-gpu=uuid,{self.FIELDS}", "--format=csv,noheader,nounits",
+               "-lms", "50"]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL,
+                                         text=True)
+        except OSError:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"],
+                    "samples": 0}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.thread.join(timeout=5)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            if self.uuid and parts[0] != self.uuid:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": float(max(smax)) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def gpu_uuid(torch):
+    try:
+        u = str(torch.cuda.get_device_properties(torch.cuda.current_device()).uuid)
+        return u if u.startswith("GPU-") else "GPU-" + u
+    except Exception:
+        return None
+
+
+# ----------------------------------------------------------------------------- our arm
+class Arm:
+    """n_sets resident copies of the layer, CUDA graphs of one rotation each."""
+
+    def __init__(self, shape, n_sets, seed0, torch, dm, MoELayer, layer_inputs, host_io=False):
+        self.shape, self.torch, self.dm = shape, torch, dm
+        self.layers, self.x = [], []
+        for s in range(n_sets):
+            inp = layer_inputs(shape, seed=seed0 + s, device="cuda")
+            if s == 0:
+                self.inputs0 = inp
+            self.layers.append(MoELayer.from_shape(shape, inp))
+            self.x.append(inp["x"])
+        self.set_host_io(host_io)
+
+    def set_host_io(self, on: bool):
+        self.host_io = on
+        if on and not hasattr(self, "x_host"):
+            self.x_host = [x.cpu().pin_memory() for x in self.x]
+            self.y_host = [self.torch.empty_like(x, device="cpu").pin_memory() for x in self.x]
+
+    def step(self, i):
+        L = self.layers[i % len(self.layers)]
+        if self.host_io:
+            x = self.x[i % len(self.x)]
+            x.copy_(self.x_host[i % len(self.x)], non_blocking=True)
+            y = L.forward(x)
+            self.y_host[i % len(self.x)].copy_(y, non_blocking=True)
+        else:
+            L.forward(self.x[i % len(self.x)])
+
+    def check(self):
+        for L in self.layers:
+            st, info = self.dm.dmoe_get_device_error(L.ws)
+            if st != 0:
+                raise RuntimeError(f"device fault {info}")
+
+    def unique_counts(self):
+        return [int(L.n_unique.item()) for L in self.layers]
+
+    def capture(self, n_steps, first, events=None):
+        """A CUDA graph of n_steps consecutive steps starting at index `first`; events[i] =
+        (begin, end) recorded around step i's gate/up kernel."""
+        torch = self.torch
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            for i in range(n_steps):
+                if events is not None:
+                    self.dm.dmoe_set_profile_events("gate_up", *events[i])
+                self.step(first + i)
+            if events is not None:
+                self.dm.dmoe_set_profile_events("gate_up", None, None)
+        return g
+
+
+def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
+    """W warm-up steps, then exactly K steps from graph replays; returns (seconds over the
+    timed region, max over ranks; mean gate/up launch seconds or None)."""
+    n_sets = len(arm.layers)
+    for i in range(W):
+        arm.step(i)
+    torch.cuda.synchronize()
+    arm.check()
+    M = n_sets
+    R, tail = divmod(K, M)
+    NG = 3
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(M)] for _ in range(NG)] if want_kernel else None
+    if want_kernel:           # torch creates the CUDA event on its first record
+        for row in evs:
+            for b, e in row:
+                b.record()
+                e.record()
+    graphs = [arm.capture(M, 0, evs[j] if want_kernel else None) for j in range(NG)]
+    tail_g = arm.capture(tail, 0) if tail else None
+    for g in graphs:       # graph upload
+        g.replay()
+    if tail_g is not None:
+        tail_g.replay()
+    torch.cuda.synchronize()
+    arm.check()
+    kernel_ms = []
+
+    def collect(j):
+        for b, e in evs[j]:
+            e.synchronize()
+            kernel_ms.append(b.elapsed_time(e))
+
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    if sampler is not None:
+        sampler.start()
+        time.sleep(0.2)
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record()
+    for r in range(R):
+        graphs[r % NG].replay()
+        if want_kernel and r >= 2:
+            collect((r - 2) % NG)
+    if tail_g is not None:
+        tail_g.replay()
+    end.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop() if sampler is not None else None
+    if want_kernel:
+        for r in range(max(0, R - 2), R):
+            collect(r % NG)
+    if dist is not None:
+        dist.barrier()
+    secs = start.elapsed_time(end) / 1e3
+    if dist is not None and world > 1:
+        t = torch.tensor([secs], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        secs = float(t.item())
+    arm.check()
+    kern = (float(np.mean(kernel_ms)) / 1e3) if kernel_ms else None
+    return secs, kern, clocks
+
+
+def traffic_from_profile(kernel: str):
+    """dram bytes per launch from the committed ncu summary, if it was taken on the current
+    source of the kernel (matching source hash); else None."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"{kernel}_layer_block.txt")
+    src = os.path.join(ROOT, "paper_2605_30876_gb300", "csrc", "expert_ffn.cu")
+    try:
+        h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+        vals = {}
+        for ln in open(path):
+            if ":" in ln:
+                k, v = ln.split(":", 1)
+                vals[k.strip()] = v.strip()
+        if vals.get("source_sha256_16") != h:
+            return None
+        return float(vals["dram_bytes_per_launch"])
+    except (OSError, KeyError, ValueError):
+        return None
+
+
+def host_inputs(shape, seed: int):
+    """Host copies of the workload's inputs (drawn on the GPU when there is one: the CPU
+    generator needs minutes for the 1.6 GB of weights)."""
+    import torch
+    from dmoe_synth import layer_inputs, to_numpy
+    dev = "cuda" if torch.cuda.is_available() else "cpu"
+    return to_numpy(layer_inputs(shape, seed=seed, device=dev))
+
+
+def cpu_baseline(shape, budget_s: float, host):
+    """The oracle as it stands, timed on the host cores on a bounded sample: full layer
+    forwards of the same workload until `budget_s` is used (at least one)."""
+    import oracle as O
+    n, t0 = 0, time.perf_counter()
+    while True:
+        O.layer_forward(host, shape.top_k, shape.mode, shape.block_size, shape.top_p)
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= budget_s:
+            break
+    return {"value": n * shape.T / el, "unit": UNIT, "cores": _CORES, "kind": "oracle",
+            "sample": f"{n} full layer forward(s) of the benchmark workload ({n * shape.T} tokens)"
+                      f" in {el:.1f} s; float64 NumPy, BLAS threads = {_CORES}"}
+
+
+# ----------------------------------------------------------------------------- reference arm
+def run_reference(args, shape, rank):
+    """The CPU oracle as the reference implementation: K timed steps, each a bounded sample
+    of the layer forward (a slice of its (token, expert) evaluations, plus the routing of
+    the block each time the sample wraps around), sized so the whole run takes minutes."""
+    if rank != 0:
+        return
+    import oracle as O
+    host = host_inputs(shape, args.seed)
+    k, T = shape.top_k, shape.T
+    n_per_token = k + (1 if shape.d_ff_shared else 0)
+    x64 = O.bf16_bits_to_f64(host["x"])
+
+    def route():
+        return O.route(host["x"], host["w_r"], host["bias"], k, shape.mode, shape.block_size,
+                       shape.top_p)
+
+    state = {"r": route(), "pos": 0}
+
+    def pair(p):
+        t, j = divmod(p, n_per_token)
+        if j < k:
+            e = int(state["r"].idx[t, j])
+            wg, wu, wd = host["w_gate"][e], host["w_up"][e], host["w_down"][e]
+            g = state["r"].gate[t, j]
+        else:
+            wg, wu, wd, g = host["ws_gate"], host["ws_up"], host["ws_down"], 1.0
+        return g * O.swiglu_ffn(x64[t:t + 1], O.bf16_bits_to_f64(wg), O.bf16_bits_to_f64(wu),
+                                O.bf16_bits_to_f64(wd))
+
+    # calibration (untimed): per-(token, expert) and per-routing cost
+    t0 = time.perf_counter()
+    for p in range(3):
+        pair(p)
+    c_pair = (time.perf_counter() - t0) / 3
+    t0 = time.perf_counter()
+    route()
+    c_route = time.perf_counter() - t0
+    budget = max(20.0, min(150.0, args.ref_budget)) / max(1, args.steps + args.warmup)
+    m = int(max(1, min(T * n_per_token, budget / max(c_pair, 1e-6))))
+    total_pairs = T * n_per_token
+
+    def step():
+        for _ in range(m):
+            if state["pos"] == total_pairs:
+                state["r"] = route()
+                state["pos"] = 0
+            pair(state["pos"])
+            state["pos"] += 1
+
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    tokens = args.steps * m / n_per_token
+    value = tokens / el
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic",
+        "config": {"workload": workload_name(shape), "tokens_per_forward": T,
+                   "l2": "n/a (CPU)"},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": _CORES, "kind": "oracle",
+                         "sample": f"each step: {m} of the {total_pairs} (token, expert) SwiGLU "
+                                   f"evaluations of one forward, plus the block's routing each "
+                                   f"time the forward wraps (routing {c_route * 1e3:.1f} ms, "
+                                   f"{c_pair * 1e3:.1f} ms per evaluation)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20000)
+    ap.add_argument("--warmup", type=int, default=16)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--sets", type=int, default=8, help="weight sets rotated between steps")
+    ap.add_argument("--seed", type=int, default=1000)
+    ap.add_argument("--side-steps", type=int, default=4000,
+                    help="steps of each side-by-side configuration (token routing, p=0.6)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--ref-budget", type=float, default=90.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    shape = workload_shape("block", 0.0)
+
+    if args.impl == "reference":
+        run_reference(args, shape, rank)
+        return
+
+    import torch
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    import paper_2605_30876_gb300 as dm
+    from dmoe_synth import layer_inputs
+    from paper_2605_30876_gb300.layer import MoELayer
+
+    peaks, peak_src = measured_peaks()
+    hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    sampler = ClockSampler(gpu_uuid(torch)) if rank == 0 else None
+
+    # headline: block routing, p = 0
+    arm = Arm(shape, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
+    secs, kern_s, clocks = timed_region(arm, args.steps, args.warmup, torch, dist, world,
+                                        sampler=sampler)
+    U = arm.unique_counts()
+    U_mean = float(np.mean(U))
+    T = shape.T
+    tokens_total = T * args.steps * world
+    value = tokens_total / secs
+    ms_per_step = secs / args.steps * 1e3
+
+    # end to end: x from pinned host memory in, y back to pinned host memory, every step
+    arm.set_host_io(True)
+    secs_e2e, _, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world,
+                                  want_kernel=False)
+    arm.set_host_io(False)
+
+    # side by side: token routing and the paper's p = 0.6
+    side = {}
+    for name, sh in (("token", workload_shape("token", 0.0)),
+                     ("block_p0.6", workload_shape("block", 0.6))):
+        a2 = Arm(sh, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
+        s2, k2, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world)
+        u2 = float(np.mean(a2.unique_counts()))
+        us = s2 / args.side_steps * 1e6
+        side[name] = {"us_per_forward": us, "tokens_per_s": T * args.side_steps * world / s2,
+                      "unique_experts_mean": u2,
+                      "hbm_roofline_frac": layer_bytes(sh, u2) / (us * 1e-6) / 1e9 / hbm,
+                      "gate_up_us": k2 * 1e6 if k2 else None}
+        del a2
+
+    if rank != 0:
+        if dist is not None:
+            dist.destroy_process_group()
+        return
+
+    lbytes = layer_bytes(shape, U_mean)
+    gbytes = gate_up_bytes(shape, U_mean)
+    achieved = gbytes / kern_s / 1e9 if kern_s else None
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": workload_name(shape), "tokens_per_forward": T,
+                   "weight_sets_rotated": args.sets,
+                   "l2": f"inputs larger than L2: {args.sets} rotated layer copies, "
+                         f"~{lbytes / 1e6:.0f} MB of weights touched per step",
+                   "graph_steps": args.sets, "parallelism": f"replicas{world}"},
+        "us_per_forward": ms_per_step * 1e3,
+        "unique_experts": {"per_set": U, "mean": U_mean},
+        "layer_roofline": {"bytes_per_forward": lbytes,
+                           "achieved_gbs": lbytes / (ms_per_step * 1e-3) / 1e9,
+                           "frac_measured_hbm": lbytes / (ms_per_step * 1e-3) / 1e9 / hbm,
+                           "frac_nominal_8tbs": lbytes / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+                           "peak_source": peak_src},
+        "roofline": {"kernel": "gate_up", "bound": "hbm", "achieved": achieved, "peak": hbm,
+                     "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
+                     "traffic": traffic_from_profile("gate_up"),
+                     "algorithmic_bytes_per_launch": gbytes,
+                     "launch_us": kern_s * 1e6 if kern_s else None,
+                     "peak_source": f"{peak_src} hbm_gbs"},
+        "side_by_side": side,
+        "e2e": {"value": tokens_total / secs_e2e, "unit": UNIT,
+                "h2d_bytes_per_step": T * shape.d_model * 2,
+                "d2h_bytes_per_step": T * shape.d_model * 2},
+        "gpu_launches": args.steps * 8,
+        "flops_per_forward": layer_flops(shape),
+        "clocks": clocks,
+    }
+    if not args.no_cpu_baseline and world == 1:
+        from dmoe_synth import to_numpy
+        line["cpu_baseline"] = cpu_baseline(shape, args.cpu_budget, to_numpy(arm.inputs0))
+    print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,187 @@
+/*
+ * dmoe.h — C ABI of the block-routed MoE-layer forward of dMoE
+ * ("dLLMs with Learnable Block Experts", arXiv 2605.30876) on one GB300 (sm_103a).
+ *
+ * The layer: a router scores every token over the |E| routed experts (§4.2,
+ * s_i = Router(t_i)); Algorithm 1 (§4.2) aggregates the token scores of each diffusion
+ * block, keeps a top-p coreset of experts and routes every token to its k best experts
+ * inside that coreset; the selected experts run as SwiGLU FFNs, an optional shared expert
+ * runs on every token, and the outputs are combined with the gate weights. Token-level
+ * routing (the "Original" baseline of §5.1) is kept as a mode.
+ *
+ * Conventions for every call below
+ *  - All tensor pointers are DEVICE pointers of the current CUDA device unless marked
+ *    "host". The caller owns all memory; the library never allocates, frees or
+ *    synchronises on the forward path (dmoe_get_device_error is the one call that syncs).
+ *  - Layouts are dense row-major, the last index fastest. bf16 tensors are passed as
+ *    `const void*` (IEEE bfloat16 bit patterns); every tensor base must be 16-byte aligned.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = the legacy default stream). All
+ *    work is enqueued asynchronously on it, in order; calls on one workspace must not
+ *    overlap on the GPU.
+ *  - Outputs are fully overwritten (no need to zero them).
+ *  - Argument errors are detected on the host before anything is launched and return
+ *    DMOE_ERR_INVALID_ARG / DMOE_ERR_UNSUPPORTED / DMOE_ERR_WORKSPACE; launch failures
+ *    return DMOE_ERR_CUDA (dmoe_last_error_message() has the CUDA text). Faults detected
+ *    on the device (an expert id out of range, a pipeline wait that timed out) never
+ *    trap: the kernels record a code in the workspace and exit; dmoe_get_device_error()
+ *    reads and clears it.
+ *  - Notation: T = n_blocks * block_size tokens, d = d_model, E = n_experts, k = top_k,
+ *    I = d_ff, I_s = d_ff_shared.
+ */
+#ifndef DMOE_H_
+#define DMOE_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define DMOE_ABI_VERSION 1
+
+typedef enum {
+  DMOE_OK = 0,
+  DMOE_ERR_INVALID_ARG = 1,   /* null pointer, bad size, misaligned pointer           */
+  DMOE_ERR_UNSUPPORTED = 2,   /* valid but outside what this build implements         */
+  DMOE_ERR_WORKSPACE = 3,     /* workspace smaller than dmoe_workspace_size()         */
+  DMOE_ERR_CUDA = 4,          /* a CUDA runtime/driver call or a launch failed        */
+  DMOE_ERR_DEVICE = 5,        /* a kernel recorded a fault (see dmoe_get_device_error) */
+  DMOE_ERR_TIMEOUT = 6        /* a kernel's bounded wait ran out                      */
+} dmoe_status;
+
+typedef enum {
+  DMOE_ROUTE_TOKEN = 0,       /* R_i = TopK(s_i, k): the token-level baseline (§5.1)  */
+  DMOE_ROUTE_BLOCK = 1        /* Algorithm 1 (§4.2) per diffusion block               */
+} dmoe_route_mode;
+
+/* Shape and routing parameters of one MoE-layer forward (plain data, host memory).
+ * Limits of this build: 1 <= k <= 16, k <= E <= 256, E % 8 == 0; d % 128 == 0,
+ * 128 <= d <= 16384; I % 128 == 0 and I_s % 128 == 0 (I_s may be 0), I, I_s <= 8192;
+ * 1 <= T <= 4096; block_size >= 1. */
+typedef struct {
+  int32_t d_model;        /* d                                                       */
+  int32_t n_experts;      /* |E| routed experts                                      */
+  int32_t top_k;          /* k experts per token                                     */
+  int32_t d_ff;           /* I, intermediate size of a routed SwiGLU expert          */
+  int32_t d_ff_shared;    /* I_s of the shared expert, 0 = no shared expert          */
+  int32_t block_size;     /* B, tokens per diffusion block                           */
+  int32_t n_blocks;       /* blocks in this forward (one per sequence), T = n_blocks*B */
+  int32_t mode;           /* dmoe_route_mode                                         */
+  float top_p;            /* block mode: coreset threshold p. The coreset is the
+                             shortest prefix of the experts sorted by normalised block
+                             score whose running sum reaches p, extended to at least k
+                             entries; p <= 0 gives exactly k (block top-k), p >= 1 every
+                             expert with a nonzero block score. Ignored in token mode. */
+} dmoe_layer_desc;
+
+/* Bytes of device workspace needed by every call below for this shape (host only; no
+ * CUDA call). One workspace sized for the desc serves all calls on that desc. */
+dmoe_status dmoe_workspace_size(const dmoe_layer_desc* desc, size_t* bytes /* host */);
+
+/* Router and routing — §4.2 (s_i = Router(t_i); S_block = aggregation of the s_i;
+ * C = Top-P(S~_block, p)) and Algorithm 1 (TopKMask, sum, Normalize, TopP,
+ * MaskOutside, TopK), or token-level TopK in DMOE_ROUTE_TOKEN mode.
+ *   x        bf16 [T, d]     token representations t_i (tokens of block b are rows
+ *                            b*B .. b*B+B-1)
+ *   w_r      fp32 [d, E]     router weight
+ *   bias     fp32 [E]        router bias, or NULL for none
+ *   topk_idx int32 [T, k]    out: R_i, expert ids by descending s_i (ties: lower id)
+ *   topk_gate fp32 [T, k]    out: g_ij = s_i[R_ij] / sum_j s_i[R_ij]
+ *   coreset  int32 [n_blocks, E] out or NULL: coreset ids of each block sorted by
+ *                            normalised block score (ties: lower id), -1 past its size
+ *   coreset_size int32 [n_blocks] out or NULL (in token mode the coreset rows are all -1
+ *                            and the sizes 0)
+ *   probs    fp32 [T, E]     out or NULL: the router scores s_i (softmax of the logits)
+ * The router runs in fp32: logits = x W_r + b, softmax, all decisions on fp32 values. */
+dmoe_status dmoe_router(const dmoe_layer_desc* desc, const void* x, const float* w_r,
+                        const float* bias, int32_t* topk_idx, float* topk_gate,
+                        int32_t* coreset, int32_t* coreset_size, float* probs,
+                        void* workspace, size_t workspace_bytes, void* stream);
+
+/* Dispatch: the unique experts of one forward (the "unique expert count" of §3 and §5)
+ * and the expert -> (token, slot) lists, computed on the device without a host round-trip.
+ *   topk_idx   int32 [T, k]   routed experts (e.g. from dmoe_router); every id must be in
+ *                             [0, E) and distinct within a token, else the device flag is
+ *                             set (DMOE_ERR_DEVICE) and the outputs are unspecified
+ *   n_unique   int32 [1]      out: U
+ *   unique_ids int32 [E]      out: the U ids ascending, then -1
+ *   offsets    int32 [E + 1]  out: offsets[u] .. offsets[u+1] is the slice of `rows` of
+ *                             the u-th unique expert; offsets[u] = T*k for u >= U
+ *   rows       int32 [T * k]  out: t*k + slot, ordered by (expert, token)
+ *   pos        int32 [T * k]  out: pos[t*k + slot] = r such that rows[r] = t*k + slot */
+dmoe_status dmoe_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx,
+                          int32_t* n_unique, int32_t* unique_ids, int32_t* offsets,
+                          int32_t* rows, int32_t* pos,
+                          void* workspace, size_t workspace_bytes, void* stream);
+
+/* Expert execution ("MoE includes routing and expert execution", §3): for every token t,
+ *   y_t = sum_j g_tj * W_down[R_tj] (silu(W_gate[R_tj] x_t) * (W_up[R_tj] x_t))
+ *         + W_sd (silu(W_sg x_t) * (W_su x_t))            (shared expert, if I_s > 0)
+ * as a grouped GEMM over the unique experts only: each unique expert's bf16 weights are
+ * streamed from HBM once per forward (tcgen05 MMA, fp32 accumulation; the SwiGLU
+ * intermediate is rounded to bf16; the combine is fp32, y is rounded to bf16).
+ *   x          bf16 [T, d]
+ *   w_gate     bf16 [E, I, d];  w_up bf16 [E, I, d];  w_down bf16 [E, d, I]
+ *   ws_gate    bf16 [I_s, d];   ws_up bf16 [I_s, d];  ws_down bf16 [d, I_s]  (NULL if I_s == 0)
+ *   topk_gate  fp32 [T, k]      gates g (as from dmoe_router)
+ *   n_unique, unique_ids, offsets, rows, pos: as written by dmoe_dispatch
+ *   y          bf16 [T, d]      out */
+dmoe_status dmoe_moe_forward(const dmoe_layer_desc* desc, const void* x,
+                             const void* w_gate, const void* w_up, const void* w_down,
+                             const void* ws_gate, const void* ws_up, const void* ws_down,
+                             const float* topk_gate, const int32_t* n_unique,
+                             const int32_t* unique_ids, const int32_t* offsets,
+                             const int32_t* rows, const int32_t* pos, void* y,
+                             void* workspace, size_t workspace_bytes, void* stream);
+
+/* The whole layer: dmoe_router + dmoe_dispatch + dmoe_moe_forward on `stream` with every
+ * intermediate in the workspace and no host round-trip. The optional outputs (NULL to
+ * skip) receive the routing: topk_idx [T,k], topk_gate [T,k], n_unique [1],
+ * unique_ids [E]. Arguments otherwise as above. */
+dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x,
+                               const float* w_r, const float* bias,
+                               const void* w_gate, const void* w_up, const void* w_down,
+                               const void* ws_gate, const void* ws_up, const void* ws_down,
+                               void* y, int32_t* topk_idx, float* topk_gate,
+                               int32_t* n_unique, int32_t* unique_ids,
+                               void* workspace, size_t workspace_bytes, void* stream);
+
+/* Kernels of the forward, for dmoe_set_profile_events. */
+typedef enum {
+  DMOE_KERNEL_ROUTER = 0,     /* router logits, softmax/top-k and Algorithm 1 kernels */
+  DMOE_KERNEL_DISPATCH = 1,   /* unique experts and expert -> token lists            */
+  DMOE_KERNEL_GATHER = 2,     /* x rows in dispatch order                            */
+  DMOE_KERNEL_GATE_UP = 3,    /* grouped gate/up GEMM + SwiGLU                       */
+  DMOE_KERNEL_DOWN = 4,       /* grouped down GEMM, gate-weighted                    */
+  DMOE_KERNEL_COMBINE = 5,    /* sum over slots + shared expert -> y                 */
+  DMOE_KERNEL_COUNT = 6
+} dmoe_kernel_id;
+
+/* Profiling aid, not part of the method: while set, every launch of `kernel` made by a
+ * call on this host thread records `ev_begin` just before it and `ev_end` just after it on
+ * the call's stream (cudaEvent_t handles passed as void*, created with timing enabled;
+ * recorded as external events, so they also work inside a CUDA-graph capture). Passing
+ * NULL for both clears the setting. Returns DMOE_ERR_INVALID_ARG for an unknown kernel. */
+dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end);
+
+/* Synchronises `stream`, then reads and clears the fault code the kernels recorded in
+ * `workspace`. Returns DMOE_OK if none, DMOE_ERR_TIMEOUT for a bounded wait that ran out,
+ * DMOE_ERR_DEVICE for any other recorded fault, DMOE_ERR_CUDA if the sync failed.
+ * `info` (host, 4 int32, or NULL) receives {code, where, value, 0}. */
+dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info);
+
+/* Static description of a status code (host). */
+const char* dmoe_status_string(dmoe_status status);
+
+/* Text of the last CUDA error seen by a call on this host thread ("" if none). */
+const char* dmoe_last_error_message(void);
+
+/* DMOE_ABI_VERSION of the loaded library. */
+int32_t dmoe_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DMOE_H_ */

@@ -1,0 +1,377 @@
+// C-ABI entry points of libdmoe: argument checks, workspace carve-up and kernel launches.
+// Nothing here allocates device memory or synchronises, except dmoe_get_device_error.
+#include <stdio.h>
+#include <string.h>
+
+#include "dmoe_internal.cuh"
+
+namespace dmoe {
+
+namespace {
+thread_local char g_last_error[256] = "";
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// Split of the router's d-reduction: enough CTAs to spread the W_r read (about 128 tiles),
+// a divisor of d/32, at most 32 partial sums.
+int router_splits(const dmoe_layer_desc& d) {
+  const int tiles = ((d.n_experts + 63) / 64) * ((d.n_blocks * d.block_size + 31) / 32);
+  int target = 128 / tiles;
+  if (target < 1) target = 1;
+  if (target > 32) target = 32;
+  const int kch = d.d_model / 32;
+  int best = 1;
+  for (int s = 1; s <= target; ++s)
+    if (kch % s == 0) best = s;
+  return best;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+}  // namespace
+
+namespace {
+struct ProfSlot {
+  cudaEvent_t begin = nullptr, end = nullptr;
+};
+thread_local ProfSlot g_prof[DMOE_KERNEL_COUNT];
+}  // namespace
+
+void prof_begin(int kernel, cudaStream_t s) {
+  if (g_prof[kernel].begin != nullptr)
+    cudaEventRecordWithFlags(g_prof[kernel].begin, s, cudaEventRecordExternal);
+}
+void prof_end(int kernel, cudaStream_t s) {
+  if (g_prof[kernel].end != nullptr)
+    cudaEventRecordWithFlags(g_prof[kernel].end, s, cudaEventRecordExternal);
+}
+
+void set_last_error(cudaError_t e) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e),
+           cudaGetErrorString(e));
+}
+
+int device_sm_count() {
+  static int cache[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+  if (dev >= 0 && dev < 64 && cache[dev] > 0) return cache[dev];
+  int n = 1;
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  if (dev >= 0 && dev < 64) cache[dev] = n;
+  return n;
+}
+
+Workspace plan_workspace(const dmoe_layer_desc& d) {
+  Workspace w{};
+  const size_t T = (size_t)d.n_blocks * d.block_size, E = d.n_experts, k = d.top_k;
+  const size_t dm = d.d_model, I = d.d_ff, Is = d.d_ff_shared;
+  w.router_splits = router_splits(d);
+  w.n_max = expert_n_max((int)T);
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t o = off;
+    off = align_up(off + (bytes == 0 ? 1 : bytes), 256);
+    return o;
+  };
+  w.err = take(sizeof(DevErrRecord));
+  w.n_unique = take(sizeof(int32_t));
+  w.logits_part = take(sizeof(float) * w.router_splits * T * E);
+  w.probs = take(sizeof(float) * T * E);
+  w.probs_hat = take(sizeof(float) * T * E);
+  w.tk_idx = take(sizeof(int32_t) * T * k);
+  w.tk_gate = take(sizeof(float) * T * k);
+  w.unique_ids = take(sizeof(int32_t) * E);
+  w.offsets = take(sizeof(int32_t) * (E + 1));
+  w.rows = take(sizeof(int32_t) * T * k);
+  w.pos = take(sizeof(int32_t) * T * k);
+  w.xperm = take(2 * T * k * dm);
+  w.h = take(2 * T * k * I);
+  w.hs = take(2 * T * Is);
+  w.part_floats = (w.n_max <= 64) ? (size_t)kMaxPersistentCtas * 2 * w.n_max * kTileM : 0;
+  w.part = take(sizeof(float) * w.part_floats);
+  w.n_counters = kMaxPersistentCtas;
+  w.counters = take(sizeof(int32_t) * w.n_counters);
+  w.yslot = take(sizeof(float) * T * k * dm);
+  w.yshared = take(sizeof(float) * T * dm);
+  w.total = off;
+  return w;
+}
+
+}  // namespace dmoe
+
+using namespace dmoe;
+
+namespace {
+
+dmoe_status check_desc(const dmoe_layer_desc* d) {
+  if (d == nullptr) return DMOE_ERR_INVALID_ARG;
+  const long T = (long)d->n_blocks * d->block_size;
+  if (d->d_model <= 0 || d->n_experts <= 0 || d->top_k <= 0 || d->d_ff <= 0 ||
+      d->d_ff_shared < 0 || d->block_size <= 0 || d->n_blocks <= 0)
+    return DMOE_ERR_INVALID_ARG;
+  if (d->mode != DMOE_ROUTE_TOKEN && d->mode != DMOE_ROUTE_BLOCK) return DMOE_ERR_INVALID_ARG;
+  if (!(d->top_p == d->top_p) || d->top_p < 0.f) return DMOE_ERR_INVALID_ARG;  // NaN or < 0
+  if (d->top_k > d->n_experts) return DMOE_ERR_INVALID_ARG;
+  if (d->top_k > kMaxTopK || d->n_experts > kMaxExperts || d->n_experts % 8 != 0)
+    return DMOE_ERR_UNSUPPORTED;
+  if (d->d_model % 128 != 0 || d->d_model > kMaxDModel) return DMOE_ERR_UNSUPPORTED;
+  if (d->d_ff % kTileM != 0 || d->d_ff > kMaxFF) return DMOE_ERR_UNSUPPORTED;
+  if (d->d_ff_shared % kTileM != 0 || d->d_ff_shared > kMaxFF) return DMOE_ERR_UNSUPPORTED;
+  if (T > kMaxTokens) return DMOE_ERR_UNSUPPORTED;
+  return DMOE_OK;
+}
+
+dmoe_status check_ws(const dmoe_layer_desc* d, void* ws, size_t ws_bytes, Workspace* plan) {
+  *plan = plan_workspace(*d);
+  if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255u) != 0) return DMOE_ERR_INVALID_ARG;
+  if (ws_bytes < plan->total) return DMOE_ERR_WORKSPACE;
+  return DMOE_OK;
+}
+
+template <class T>
+T* at(void* ws, size_t off) {
+  return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
+}
+
+dmoe_status cuda_status(cudaError_t e) {
+  if (e == cudaSuccess) return DMOE_OK;
+  set_last_error(e);
+  return DMOE_ERR_CUDA;
+}
+
+bool all_aligned(std::initializer_list<const void*> ptrs) {
+  for (const void* p : ptrs)
+    if (p == nullptr || (reinterpret_cast<uintptr_t>(p) & 15u) != 0) return false;
+  return true;
+}
+
+dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* w_r,
+                       const float* bias, int32_t* topk_idx, float* topk_gate, int32_t* coreset,
+                       int32_t* coreset_size, float* probs, void* ws, const Workspace& plan,
+                       cudaStream_t s) {
+  RouterArgs a{};
+  a.x = static_cast<const __nv_bfloat16*>(x);
+  a.w_r = w_r;
+  a.bias = bias;
+  a.logits_part = at<float>(ws, plan.logits_part);
+  a.probs = probs != nullptr ? probs : at<float>(ws, plan.probs);
+  a.probs_hat = at<float>(ws, plan.probs_hat);
+  a.topk_idx = topk_idx;
+  a.topk_gate = topk_gate;
+  a.coreset = coreset;
+  a.coreset_size = coreset_size;
+  a.T = desc->n_blocks * desc->block_size;
+  a.d = desc->d_model;
+  a.E = desc->n_experts;
+  a.k = desc->top_k;
+  a.B = desc->block_size;
+  a.n_blocks = desc->n_blocks;
+  a.mode = desc->mode;
+  a.splits = plan.router_splits;
+  a.top_p = desc->top_p;
+  a.err = at<DevErrRecord>(ws, plan.err);
+  return cuda_status(launch_router(a, s));
+}
+
+dmoe_status run_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx, int32_t* n_unique,
+                         int32_t* unique_ids, int32_t* offsets, int32_t* rows, int32_t* pos,
+                         void* ws, const Workspace& plan, cudaStream_t s) {
+  DispatchArgs a{};
+  a.topk_idx = topk_idx;
+  a.n_unique = n_unique;
+  a.unique_ids = unique_ids;
+  a.offsets = offsets;
+  a.rows = rows;
+  a.pos = pos;
+  a.T = desc->n_blocks * desc->block_size;
+  a.E = desc->n_experts;
+  a.k = desc->top_k;
+  a.err = at<DevErrRecord>(ws, plan.err);
+  return cuda_status(launch_dispatch(a, s));
+}
+
+dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* w_gate,
+                        const void* w_up, const void* w_down, const void* ws_gate,
+                        const void* ws_up, const void* ws_down, const float* topk_gate,
+                        const int32_t* n_unique, const int32_t* unique_ids,
+                        const int32_t* offsets, const int32_t* rows, const int32_t* pos,
+                        void* y, void* ws, const Workspace& plan, cudaStream_t s) {
+  ExpertArgs a{};
+  a.x = static_cast<const __nv_bfloat16*>(x);
+  a.w_gate = w_gate;
+  a.w_up = w_up;
+  a.w_down = w_down;
+  a.ws_gate = ws_gate;
+  a.ws_up = ws_up;
+  a.ws_down = ws_down;
+  a.topk_gate = topk_gate;
+  a.n_unique = n_unique;
+  a.unique_ids = unique_ids;
+  a.offsets = offsets;
+  a.rows = rows;
+  a.pos = pos;
+  a.y = static_cast<__nv_bfloat16*>(y);
+  a.xperm = at<__nv_bfloat16>(ws, plan.xperm);
+  a.h = at<__nv_bfloat16>(ws, plan.h);
+  a.hs = at<__nv_bfloat16>(ws, plan.hs);
+  a.part = at<float>(ws, plan.part);
+  a.counters = at<int32_t>(ws, plan.counters);
+  a.yslot = at<float>(ws, plan.yslot);
+  a.yshared = at<float>(ws, plan.yshared);
+  a.n_counters = plan.n_counters;
+  a.part_floats = plan.part_floats;
+  a.err = at<DevErrRecord>(ws, plan.err);
+  a.T = desc->n_blocks * desc->block_size;
+  a.d = desc->d_model;
+  a.E = desc->n_experts;
+  a.k = desc->top_k;
+  a.I = desc->d_ff;
+  a.Is = desc->d_ff_shared;
+  a.n_max = plan.n_max;
+  return cuda_status(launch_experts(a, s));
+}
+
+}  // namespace
+
+extern "C" {
+
+dmoe_status dmoe_workspace_size(const dmoe_layer_desc* desc, size_t* bytes) {
+  if (bytes == nullptr) return DMOE_ERR_INVALID_ARG;
+  const dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  *bytes = plan_workspace(*desc).total;
+  return DMOE_OK;
+}
+
+dmoe_status dmoe_router(const dmoe_layer_desc* desc, const void* x, const float* w_r,
+                        const float* bias, int32_t* topk_idx, float* topk_gate,
+                        int32_t* coreset, int32_t* coreset_size, float* probs,
+                        void* workspace, size_t workspace_bytes, void* stream) {
+  dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  if (!all_aligned({x, w_r, topk_idx, topk_gate})) return DMOE_ERR_INVALID_ARG;
+  if ((bias != nullptr && !aligned16(bias)) || (probs != nullptr && !aligned16(probs)) ||
+      (coreset != nullptr && !aligned16(coreset)) ||
+      (coreset_size != nullptr && !aligned16(coreset_size)))
+    return DMOE_ERR_INVALID_ARG;
+  Workspace plan;
+  st = check_ws(desc, workspace, workspace_bytes, &plan);
+  if (st != DMOE_OK) return st;
+  return run_router(desc, x, w_r, bias, topk_idx, topk_gate, coreset, coreset_size, probs,
+                    workspace, plan, static_cast<cudaStream_t>(stream));
+}
+
+dmoe_status dmoe_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx,
+                          int32_t* n_unique, int32_t* unique_ids, int32_t* offsets,
+                          int32_t* rows, int32_t* pos, void* workspace, size_t workspace_bytes,
+                          void* stream) {
+  dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  if (!all_aligned({topk_idx, n_unique, unique_ids, offsets, rows, pos}))
+    return DMOE_ERR_INVALID_ARG;
+  Workspace plan;
+  st = check_ws(desc, workspace, workspace_bytes, &plan);
+  if (st != DMOE_OK) return st;
+  return run_dispatch(desc, topk_idx, n_unique, unique_ids, offsets, rows, pos, workspace, plan,
+                      static_cast<cudaStream_t>(stream));
+}
+
+dmoe_status dmoe_moe_forward(const dmoe_layer_desc* desc, const void* x, const void* w_gate,
+                             const void* w_up, const void* w_down, const void* ws_gate,
+                             const void* ws_up, const void* ws_down, const float* topk_gate,
+                             const int32_t* n_unique, const int32_t* unique_ids,
+                             const int32_t* offsets, const int32_t* rows, const int32_t* pos,
+                             void* y, void* workspace, size_t workspace_bytes, void* stream) {
+  dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  if (!all_aligned({x, w_gate, w_up, w_down, topk_gate, n_unique, unique_ids, offsets, rows,
+                    pos, y}))
+    return DMOE_ERR_INVALID_ARG;
+  if (desc->d_ff_shared > 0 && !all_aligned({ws_gate, ws_up, ws_down})) return DMOE_ERR_INVALID_ARG;
+  Workspace plan;
+  st = check_ws(desc, workspace, workspace_bytes, &plan);
+  if (st != DMOE_OK) return st;
+  return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, topk_gate, n_unique,
+                     unique_ids, offsets, rows, pos, y, workspace, plan,
+                     static_cast<cudaStream_t>(stream));
+}
+
+dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const float* w_r,
+                               const float* bias, const void* w_gate, const void* w_up,
+                               const void* w_down, const void* ws_gate, const void* ws_up,
+                               const void* ws_down, void* y, int32_t* topk_idx,
+                               float* topk_gate, int32_t* n_unique, int32_t* unique_ids,
+                               void* workspace, size_t workspace_bytes, void* stream) {
+  dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  if (!all_aligned({x, w_r, w_gate, w_up, w_down, y})) return DMOE_ERR_INVALID_ARG;
+  if (desc->d_ff_shared > 0 && !all_aligned({ws_gate, ws_up, ws_down})) return DMOE_ERR_INVALID_ARG;
+  if ((bias != nullptr && !aligned16(bias)) || (topk_idx != nullptr && !aligned16(topk_idx)) ||
+      (topk_gate != nullptr && !aligned16(topk_gate)) ||
+      (n_unique != nullptr && !aligned16(n_unique)) ||
+      (unique_ids != nullptr && !aligned16(unique_ids)))
+    return DMOE_ERR_INVALID_ARG;
+  Workspace plan;
+  st = check_ws(desc, workspace, workspace_bytes, &plan);
+  if (st != DMOE_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  int32_t* idx = topk_idx != nullptr ? topk_idx : at<int32_t>(workspace, plan.tk_idx);
+  float* gate = topk_gate != nullptr ? topk_gate : at<float>(workspace, plan.tk_gate);
+  int32_t* nu = n_unique != nullptr ? n_unique : at<int32_t>(workspace, plan.n_unique);
+  int32_t* uid = unique_ids != nullptr ? unique_ids : at<int32_t>(workspace, plan.unique_ids);
+  int32_t* offs = at<int32_t>(workspace, plan.offsets);
+  int32_t* rows = at<int32_t>(workspace, plan.rows);
+  int32_t* pos = at<int32_t>(workspace, plan.pos);
+  st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s);
+  if (st != DMOE_OK) return st;
+  st = run_dispatch(desc, idx, nu, uid, offs, rows, pos, workspace, plan, s);
+  if (st != DMOE_OK) return st;
+  return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid, offs,
+                     rows, pos, y, workspace, plan, s);
+}
+
+dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) {
+  if (workspace == nullptr) return DMOE_ERR_INVALID_ARG;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return cuda_status(e);
+  DevErrRecord rec{};
+  e = cudaMemcpy(&rec, workspace, sizeof(rec), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_status(e);
+  if (info != nullptr) {
+    info[0] = rec.code;
+    info[1] = rec.where;
+    info[2] = rec.value;
+    info[3] = 0;
+  }
+  if (rec.code == kErrNone) return DMOE_OK;
+  e = cudaMemset(workspace, 0, sizeof(rec));
+  if (e != cudaSuccess) return cuda_status(e);
+  return rec.code == kErrTimeout ? DMOE_ERR_TIMEOUT : DMOE_ERR_DEVICE;
+}
+
+dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end) {
+  if (kernel < 0 || kernel >= DMOE_KERNEL_COUNT) return DMOE_ERR_INVALID_ARG;
+  g_prof[kernel].begin = static_cast<cudaEvent_t>(ev_begin);
+  g_prof[kernel].end = static_cast<cudaEvent_t>(ev_end);
+  return DMOE_OK;
+}
+
+const char* dmoe_status_string(dmoe_status status) {
+  switch (status) {
+    case DMOE_OK: return "DMOE_OK";
+    case DMOE_ERR_INVALID_ARG: return "DMOE_ERR_INVALID_ARG: invalid argument";
+    case DMOE_ERR_UNSUPPORTED: return "DMOE_ERR_UNSUPPORTED: shape outside this build's limits";
+    case DMOE_ERR_WORKSPACE: return "DMOE_ERR_WORKSPACE: workspace too small";
+    case DMOE_ERR_CUDA: return "DMOE_ERR_CUDA: CUDA call or launch failed";
+    case DMOE_ERR_DEVICE: return "DMOE_ERR_DEVICE: a kernel recorded a fault";
+    case DMOE_ERR_TIMEOUT: return "DMOE_ERR_TIMEOUT: a kernel's bounded wait ran out";
+  }
+  return "unknown dmoe_status";
+}
+
+const char* dmoe_last_error_message(void) { return g_last_error; }
+
+int32_t dmoe_abi_version(void) { return DMOE_ABI_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,150 @@
+// Internal declarations shared by the CUDA translation units of libdmoe (not installed).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/dmoe.h"
+
+namespace dmoe {
+
+// ---------------------------------------------------------------------------------------
+// limits of this build (mirrored in include/dmoe.h)
+// ---------------------------------------------------------------------------------------
+constexpr int kMaxExperts = 256;
+constexpr int kMaxTopK = 16;
+constexpr int kMaxTokens = 4096;
+constexpr int kMaxDModel = 16384;
+constexpr int kMaxFF = 8192;
+constexpr int kTileM = 128;        // MMA M (weight rows per tile)
+constexpr int kTileK = 64;         // K elements per pipeline stage (128 B of bf16)
+constexpr int kMaxPersistentCtas = 320;
+
+// ---------------------------------------------------------------------------------------
+// device fault record, at the head of the workspace
+// ---------------------------------------------------------------------------------------
+enum DevErr : int32_t {
+  kErrNone = 0,
+  kErrTimeout = 1,        // a bounded mbarrier wait ran out
+  kErrExpertId = 2,       // an expert id outside [0, E)
+  kErrDupExpert = 3,      // the same expert twice in one token's list
+  kErrBadDispatch = 4,    // dispatch data inconsistent (counts, offsets)
+};
+enum DevWhere : int32_t {
+  kAtRouter = 1, kAtBlockRoute = 2, kAtDispatch = 3, kAtGateUp = 4, kAtDown = 5,
+  kAtCombine = 6, kAtGather = 7,
+};
+struct DevErrRecord {
+  int32_t code;
+  int32_t where;
+  int32_t value;
+  int32_t pad;
+};
+
+__device__ __forceinline__ void record_error(DevErrRecord* rec, int code, int where, int value) {
+  if (atomicCAS(&rec->code, 0, code) == 0) {
+    rec->where = where;
+    rec->value = value;
+  }
+}
+
+// ---------------------------------------------------------------------------------------
+// workspace layout (byte offsets from the workspace base; every region 256-B aligned)
+// ---------------------------------------------------------------------------------------
+struct Workspace {
+  size_t err;          // DevErrRecord
+  size_t n_unique;     // int32 [1]  (used when the caller does not supply one)
+  size_t logits_part;  // fp32 [router_splits, T, E]
+  size_t probs;        // fp32 [T, E]
+  size_t probs_hat;    // fp32 [T, E]   TopKMask(s_i, k)
+  size_t tk_idx;       // int32 [T, k] routed experts (when the caller does not supply)
+  size_t tk_gate;      // fp32 [T, k]
+  size_t unique_ids;   // int32 [E]
+  size_t offsets;      // int32 [E + 1]
+  size_t rows;         // int32 [T*k]
+  size_t pos;          // int32 [T*k]
+  size_t xperm;        // bf16 [T*k, d]   x gathered in dispatch order
+  size_t h;            // bf16 [T*k, I]   SwiGLU intermediate of the routed experts
+  size_t hs;           // bf16 [T, I_s]   shared-expert intermediate
+  size_t part;         // fp32 split-K partials of the gate/up GEMM
+  size_t counters;     // int32 split-K tickets
+  size_t yslot;        // fp32 [T*k, d]   gate-weighted expert outputs per (token, slot)
+  size_t yshared;      // fp32 [T, d]
+  size_t total;
+  int router_splits;
+  int n_max;           // token tile (MMA N) of the expert GEMMs
+  int n_counters;
+  size_t part_floats;
+};
+
+// Token tile of the expert GEMMs: every group's rows are covered by tiles of n_max.
+inline int expert_n_max(int T) {
+  int n = ((T + 15) / 16) * 16;
+  return n > 256 ? 256 : (n < 16 ? 16 : n);
+}
+
+Workspace plan_workspace(const dmoe_layer_desc& d);
+
+// ---------------------------------------------------------------------------------------
+// launchers (each defined in its own translation unit)
+// ---------------------------------------------------------------------------------------
+struct RouterArgs {
+  const __nv_bfloat16* x;
+  const float* w_r;
+  const float* bias;
+  float* logits_part;
+  float* probs;        // [T, E]
+  float* probs_hat;    // [T, E] (block mode)
+  int32_t* topk_idx;   // [T, k] final routing
+  float* topk_gate;    // [T, k]
+  int32_t* coreset;    // [n_blocks, E] or null
+  int32_t* coreset_size;
+  int T, d, E, k, B, n_blocks, mode, splits;
+  float top_p;
+  DevErrRecord* err;
+};
+cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
+
+struct DispatchArgs {
+  const int32_t* topk_idx;
+  int32_t* n_unique;
+  int32_t* unique_ids;
+  int32_t* offsets;
+  int32_t* rows;
+  int32_t* pos;
+  int T, E, k;
+  DevErrRecord* err;
+};
+cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s);
+
+struct ExpertArgs {
+  // inputs
+  const __nv_bfloat16* x;
+  const void* w_gate; const void* w_up; const void* w_down;
+  const void* ws_gate; const void* ws_up; const void* ws_down;
+  const float* topk_gate;
+  const int32_t* n_unique; const int32_t* unique_ids; const int32_t* offsets;
+  const int32_t* rows; const int32_t* pos;
+  __nv_bfloat16* y;
+  // workspace
+  __nv_bfloat16* xperm; __nv_bfloat16* h; __nv_bfloat16* hs;
+  float* part; int32_t* counters; float* yslot; float* yshared;
+  int n_counters;
+  size_t part_floats;
+  DevErrRecord* err;
+  // shape
+  int T, d, E, k, I, Is, n_max;
+};
+cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
+
+// profiling events (dmoe_set_profile_events), per host thread
+void prof_begin(int kernel, cudaStream_t s);
+void prof_end(int kernel, cudaStream_t s);
+
+// host helpers
+int device_sm_count();
+void set_last_error(cudaError_t e);
+
+}  // namespace dmoe

@@ -24,3 +24,17 @@ def pytest_collection_modifyitems(config, items):
     for it in items:
         if "gpu" in it.keywords:
             it.add_marker(skip)
+
+
+def _ensure_library():
+    """Builds libdmoe.so in-tree when it is missing or older than its sources (the build
+    module is loaded by path: importing the package itself needs the built library)."""
+    import importlib.util
+    path = os.path.join(ROOT, "paper_2605_30876_gb300", "_build.py")
+    spec = importlib.util.spec_from_file_location("_dmoe_build", path)
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    mod.build()
+
+
+_ensure_library()

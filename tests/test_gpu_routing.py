@@ -1,0 +1,122 @@
+"""GPU parity of the router, Algorithm 1 and dispatch against the CPU oracle (through the
+C ABI). Expert selections and dispatch indices are compared bit-exactly except at decisions
+whose oracle margin is below 1e-5 (see tests/parity.py)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+from dmoe_synth import (LAYER, LAYER_B8, ROUTE_BLOCK, ROUTE_TOKEN, STACK20, TINY, MoEShape,
+                        layer_inputs, to_numpy)
+from tests import parity as P
+
+pytestmark = pytest.mark.gpu
+
+ROUTING_CASES = {
+    "tiny_block_p0": TINY,
+    "tiny_block_p06": TINY.with_(top_p=0.6),
+    "tiny_token": TINY.with_(mode=ROUTE_TOKEN),
+    "layer_block_p0": LAYER,
+    "layer_block_p06": LAYER.with_(top_p=0.6),
+    "layer_block_p1": LAYER.with_(top_p=1.0),
+    "layer_token": LAYER.with_(mode=ROUTE_TOKEN),
+    "layer_b8_block_p0": LAYER_B8,
+    "layer_b8_block_p06": LAYER_B8.with_(top_p=0.6),
+    "layer_b8_token": LAYER_B8.with_(mode=ROUTE_TOKEN),
+    "stack_T2048_block_p0": STACK20,
+    "stack_T2048_token": STACK20.with_(mode=ROUTE_TOKEN),
+    "sweep_B4x32_bias0": LAYER.with_(block_size=4, n_blocks=32, bias_scale=0.0),
+    "sweep_B64x16_bias1": LAYER.with_(block_size=64, n_blocks=16, bias_scale=1.0, top_p=0.6),
+    "block_size_1": LAYER.with_(block_size=1, n_blocks=40, top_p=0.6),
+    "ragged_T60_k1": TINY.with_(block_size=12, n_blocks=5, top_k=1, top_p=0.5),
+    "k_equals_E": TINY.with_(top_k=16, top_p=0.3),
+    "E8_k3": TINY.with_(n_experts=8, top_k=3, top_p=0.7, d_model=128),
+    "max_tokens_4096": LAYER.with_(block_size=64, n_blocks=64, top_p=0.6),
+}
+
+
+def _routing_case(name, seed=0):
+    shape = ROUTING_CASES[name]
+    dev = layer_inputs(shape, seed=seed, device="cuda", with_weights=False)
+    host = to_numpy(dev)
+    return shape, dev, host
+
+
+@pytest.mark.parametrize("name", list(ROUTING_CASES))
+def test_routing_matches_oracle(name):
+    shape, dev, host = _routing_case(name)
+    g = P.gpu_router(shape, dev)
+    orc = P.oracle_routing(shape, host)
+    stats = P.check_routing(shape, g, orc)
+    assert stats["exact"] >= 0.9 * stats["tokens"], stats
+    if shape.mode == ROUTE_BLOCK and shape.top_p == 0.0:
+        for b in range(shape.n_blocks):
+            blk = g["idx"][b * shape.block_size:(b + 1) * shape.block_size]
+            assert len(np.unique(blk)) == shape.top_k
+
+
+@pytest.mark.parametrize("name", ["tiny_block_p06", "layer_block_p0", "layer_token",
+                                  "layer_b8_block_p06", "stack_T2048_token", "ragged_T60_k1",
+                                  "max_tokens_4096"])
+def test_dispatch_bit_exact(name):
+    shape, dev, host = _routing_case(name)
+    g = P.gpu_router(shape, dev)
+    idx_t = torch.from_numpy(g["idx"]).cuda()
+    out, ws = P.gpu_dispatch(shape, idx_t)
+    st, info = P.dm().dmoe_get_device_error(ws)
+    assert st == 0, info
+    P.check_dispatch(shape, g["idx"], out)
+    # the oracle's own selection injected
+    orc = P.oracle_routing(shape, host)
+    out2, _ = P.gpu_dispatch(shape, torch.from_numpy(orc.idx).cuda(), ws)
+    P.check_dispatch(shape, orc.idx, out2)
+
+
+def test_hand_case_on_gpu():
+    """The hand-worked Algorithm 1 case (E=4 padded to 8 with near-zero scores, k=2, B=2):
+    x_i one-hot, W_r row i = ln s_i, so the router returns s_i up to fp32 rounding."""
+    s_hand = np.array([[0.5, 0.3, 0.15, 0.05], [0.1, 0.4, 0.2, 0.3]])
+    d, E = 128, 8
+    x = torch.zeros((2, d), dtype=torch.bfloat16)
+    x[0, 0] = 1.0
+    x[1, 3] = 1.0
+    w_r = torch.full((d, E), 0.0)
+    w_r[0, :4] = torch.tensor(np.log(s_hand[0]))
+    w_r[3, :4] = torch.tensor(np.log(s_hand[1]))
+    w_r[0, 4:] = -80.0
+    w_r[3, 4:] = -80.0
+    dev = dict(x=x.cuda(), w_r=w_r.float().cuda(), bias=torch.zeros(E).cuda())
+    expect = {0.6: ([1, 0], [[0, 1], [1, 0]]), 0.9: ([1, 0, 3], [[0, 1], [1, 3]]),
+              0.0: ([1, 0], [[0, 1], [1, 0]])}
+    for p, (core, idx) in expect.items():
+        shape = MoEShape(d_model=d, n_experts=E, top_k=2, d_ff=128, d_ff_shared=0,
+                         block_size=2, n_blocks=1, mode=ROUTE_BLOCK, top_p=p)
+        g = P.gpu_router(shape, dev)
+        assert g["coreset"][0][:len(core)].tolist() == core
+        assert int(g["coreset_size"][0]) == len(core)
+        assert g["idx"].tolist() == idx
+    np.testing.assert_allclose(g["gate"], [[0.625, 0.375], [0.8, 0.2]], rtol=1e-5)
+
+
+def test_routing_is_deterministic():
+    shape, dev, _ = _routing_case("layer_b8_block_p06")
+    a = P.gpu_router(shape, dev)
+    b = P.gpu_router(shape, dev)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_dispatch_rejects_bad_ids():
+    shape = TINY
+    m = P.dm()
+    idx = torch.zeros((shape.T, shape.top_k), dtype=torch.int32, device="cuda")
+    idx[:, 1] = 1
+    idx[3, 0] = shape.n_experts          # out of range
+    _, ws = P.gpu_dispatch(shape, idx)
+    st, info = m.dmoe_get_device_error(ws)
+    assert st == 5 and info[0] == 2
+    idx[3, 0] = 1                        # duplicate expert in one token
+    _, ws = P.gpu_dispatch(shape, idx, ws)
+    st, info = m.dmoe_get_device_error(ws)
+    assert st == 5 and info[0] == 3
+    assert m.dmoe_get_device_error(ws)[0] == 0   # cleared
