@@ -315,61 +315,68 @@ def cpu_baseline(shape, budget_s: float, host):
 # ----------------------------------------------------------------------------- reference arm
 def run_reference(args, shape, rank):
     """The CPU oracle as the reference implementation: K timed steps, each a bounded sample
-    of the layer forward (a slice of its (token, expert) evaluations, plus the routing of
-    the block each time the sample wraps around), sized so the whole run takes minutes."""
+    of the layer forward. The oracle evaluates a forward expert by expert (one SwiGLU over
+    the rows routed to that expert, the shared expert over all tokens); a step runs the next
+    m of those expert groups, and re-routes the block (router + Algorithm 1) each time the
+    forward wraps around. m is sized so that the whole run takes minutes."""
     if rank != 0:
         return
     import oracle as O
     host = host_inputs(shape, args.seed)
     k, T = shape.top_k, shape.T
-    n_per_token = k + (1 if shape.d_ff_shared else 0)
+    rows_per_token = k + (1 if shape.d_ff_shared else 0)
     x64 = O.bf16_bits_to_f64(host["x"])
 
     def route():
-        return O.route(host["x"], host["w_r"], host["bias"], k, shape.mode, shape.block_size,
-                       shape.top_p)
+        r = O.route(host["x"], host["w_r"], host["bias"], k, shape.mode, shape.block_size,
+                    shape.top_p)
+        groups = []
+        for e in sorted(set(int(v) for v in r.idx.ravel())):
+            tt, jj = np.nonzero(r.idx == e)
+            groups.append((e, tt, r.gate[tt, jj]))
+        if shape.d_ff_shared:
+            groups.append((-1, np.arange(T), np.ones(T)))
+        return groups
 
-    state = {"r": route(), "pos": 0}
-
-    def pair(p):
-        t, j = divmod(p, n_per_token)
-        if j < k:
-            e = int(state["r"].idx[t, j])
+    def run_group(grp):
+        e, tt, g = grp
+        if e >= 0:
             wg, wu, wd = host["w_gate"][e], host["w_up"][e], host["w_down"][e]
-            g = state["r"].gate[t, j]
         else:
-            wg, wu, wd, g = host["ws_gate"], host["ws_up"], host["ws_down"], 1.0
-        return g * O.swiglu_ffn(x64[t:t + 1], O.bf16_bits_to_f64(wg), O.bf16_bits_to_f64(wu),
-                                O.bf16_bits_to_f64(wd))
+            wg, wu, wd = host["ws_gate"], host["ws_up"], host["ws_down"]
+        y = O.swiglu_ffn(x64[tt], O.bf16_bits_to_f64(wg), O.bf16_bits_to_f64(wu),
+                         O.bf16_bits_to_f64(wd))
+        return g[:, None] * y, len(tt)
 
-    # calibration (untimed): per-(token, expert) and per-routing cost
+    # calibration (untimed)
     t0 = time.perf_counter()
-    for p in range(3):
-        pair(p)
-    c_pair = (time.perf_counter() - t0) / 3
-    t0 = time.perf_counter()
-    route()
+    groups = route()
     c_route = time.perf_counter() - t0
+    t0 = time.perf_counter()
+    run_group(groups[0])
+    c_group = time.perf_counter() - t0
     budget = max(20.0, min(150.0, args.ref_budget)) / max(1, args.steps + args.warmup)
-    m = int(max(1, min(T * n_per_token, budget / max(c_pair, 1e-6))))
-    total_pairs = T * n_per_token
+    m = int(max(1, min(len(groups), budget / max(c_group, 1e-6))))
+    state = {"groups": groups, "pos": 0}
 
     def step():
+        rows = 0
         for _ in range(m):
-            if state["pos"] == total_pairs:
-                state["r"] = route()
+            if state["pos"] == len(state["groups"]):
+                state["groups"] = route()
                 state["pos"] = 0
-            pair(state["pos"])
+            rows += run_group(state["groups"][state["pos"]])[1]
             state["pos"] += 1
+        return rows
 
     for _ in range(args.warmup):
         step()
+    rows = 0
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        step()
+        rows += step()
     el = time.perf_counter() - t0
-    tokens = args.steps * m / n_per_token
-    value = tokens / el
+    value = rows / rows_per_token / el
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": el / args.steps * 1e3,
@@ -378,10 +385,12 @@ def run_reference(args, shape, rank):
         "config": {"workload": workload_name(shape), "tokens_per_forward": T,
                    "l2": "n/a (CPU)"},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": _CORES, "kind": "oracle",
-                         "sample": f"each step: {m} of the {total_pairs} (token, expert) SwiGLU "
-                                   f"evaluations of one forward, plus the block's routing each "
-                                   f"time the forward wraps (routing {c_route * 1e3:.1f} ms, "
-                                   f"{c_pair * 1e3:.1f} ms per evaluation)"},
+                         "sample": f"each step: {m} of the {len(groups)} expert groups of one "
+                                   f"forward (one fp64 SwiGLU over the rows routed to an "
+                                   f"expert), plus the block's routing each time the forward "
+                                   f"wraps (routing {c_route * 1e3:.1f} ms, "
+                                   f"{c_group * 1e3:.1f} ms per group); tokens counted as "
+                                   f"rows / (k + shared)"},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -401,6 +410,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--ref-budget", type=float, default=90.0)
+    ap.add_argument("--only-headline", action="store_true",
+                    help="skip the e2e and side-by-side arms (small profiling runs)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -440,15 +451,18 @@ def main():
     ms_per_step = secs / args.steps * 1e3
 
     # end to end: x from pinned host memory in, y back to pinned host memory, every step
-    arm.set_host_io(True)
-    secs_e2e, _, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world,
-                                  want_kernel=False)
-    arm.set_host_io(False)
+    secs_e2e = None
+    if not args.only_headline:
+        arm.set_host_io(True)
+        secs_e2e, _, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world,
+                                      want_kernel=False)
+        arm.set_host_io(False)
 
     # side by side: token routing and the paper's p = 0.6
     side = {}
-    for name, sh in (("token", workload_shape("token", 0.0)),
-                     ("block_p0.6", workload_shape("block", 0.6))):
+    side_cfgs = () if args.only_headline else (("token", workload_shape("token", 0.0)),
+                                               ("block_p0.6", workload_shape("block", 0.6)))
+    for name, sh in side_cfgs:
         a2 = Arm(sh, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
         s2, k2, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world)
         u2 = float(np.mean(a2.unique_counts()))
@@ -490,7 +504,7 @@ def main():
                      "launch_us": kern_s * 1e6 if kern_s else None,
                      "peak_source": f"{peak_src} hbm_gbs"},
         "side_by_side": side,
-        "e2e": {"value": tokens_total / secs_e2e, "unit": UNIT,
+        "e2e": None if secs_e2e is None else {"value": tokens_total / secs_e2e, "unit": UNIT,
                 "h2d_bytes_per_step": T * shape.d_model * 2,
                 "d2h_bytes_per_step": T * shape.d_model * 2},
         "gpu_launches": args.steps * 8,

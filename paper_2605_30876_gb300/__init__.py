@@ -74,7 +74,7 @@ def _load() -> ctypes.CDLL:
     lib.dmoe_router.restype = st
     lib.dmoe_dispatch.argtypes = [D, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.dmoe_dispatch.restype = st
-    lib.dmoe_moe_forward.argtypes = [D] + [P] * 15 + [P, ctypes.c_size_t, P]
+    lib.dmoe_moe_forward.argtypes = [D] + [P] * 14 + [P, ctypes.c_size_t, P]
     lib.dmoe_moe_forward.restype = st
     lib.dmoe_layer_forward.argtypes = [D] + [P] * 14 + [P, ctypes.c_size_t, P]
     lib.dmoe_layer_forward.restype = st

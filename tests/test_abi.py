@@ -88,7 +88,7 @@ def test_null_and_misaligned_pointers_are_rejected_before_launch(dm):
     assert st == 1
     # shared expert declared but its weights missing
     st = lib.dmoe_moe_forward(ctypes.byref(desc), *([P(fake)] * 4), None, None, None,
-                              *([P(fake)] * 8), P(fake), n, None)
+                              *([P(fake)] * 7), P(fake), n, None)
     assert st == 1
     st = lib.dmoe_layer_forward(None, *([P(fake)] * 14), P(fake), n, None)
     assert st == 1
