@@ -165,6 +165,31 @@ typedef enum {
  * NULL for both clears the setting. Returns DMOE_ERR_INVALID_ARG for an unknown kernel. */
 dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end);
 
+/* dmoe_router for callers that cannot allocate device memory. The paper has no
+ * counterpart: this is a deployment convenience. Some callers may not call cudaMalloc (or
+ * any allocator) at all: code running inside an allocator or memory-pool callback, a host
+ * framework or plugin that owns every device allocation itself, or a latency-critical loop
+ * that must never enter the allocator. This call takes no workspace: its scratch (partial
+ * logits, scores, the fault record) lives in a fixed 4 MiB array in the library's own
+ * device memory, which every GPU that loads the library holds until the process exits.
+ * The caller still passes every input and output, exactly as for dmoe_router, and the
+ * results are the same.
+ *  - The call allocates nothing and frees nothing (no cudaMalloc/cudaFree, no allocating
+ *    library routine). Shapes whose router scratch exceeds 4 MiB (partial logits + 2 x
+ *    T*E fp32 + 512 bytes; e.g. T = 4096 tokens with 256 experts) return
+ *    DMOE_ERR_UNSUPPORTED, with the sizes in dmoe_last_error_message().
+ *  - The first call on each device looks up the array's device address (with that device
+ *    current) and caches it; make that first call before any CUDA-graph stream capture.
+ *  - All calls share the one array and it keeps the previous call's contents: each call
+ *    clears the fault record it uses, and everything else it reads it has written first.
+ *    Calls whose executions overlap on the GPU (two streams, or two host threads) race on
+ *    the array and give wrong results: serialise them.
+ * Arguments, layouts and errors otherwise as for dmoe_router. */
+dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const void* x, const float* w_r,
+                                 const float* bias, int32_t* topk_idx, float* topk_gate,
+                                 int32_t* coreset, int32_t* coreset_size, float* probs,
+                                 void* stream);
+
 /* Synchronises `stream`, then reads and clears the fault code the kernels recorded in
  * `workspace`. Returns DMOE_OK if none, DMOE_ERR_TIMEOUT for a bounded wait that ran out,
  * DMOE_ERR_DEVICE for any other recorded fault, DMOE_ERR_CUDA if the sync failed.

@@ -50,6 +50,10 @@ void set_last_error(cudaError_t e) {
            cudaGetErrorString(e));
 }
 
+void set_last_error_text(const char* msg) {
+  snprintf(g_last_error, sizeof(g_last_error), "%s", msg);
+}
+
 int device_sm_count() {
   static int cache[64] = {0};
   int dev = 0;

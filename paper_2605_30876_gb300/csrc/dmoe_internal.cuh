@@ -146,5 +146,6 @@ void prof_end(int kernel, cudaStream_t s);
 // host helpers
 int device_sm_count();
 void set_last_error(cudaError_t e);
+void set_last_error_text(const char* msg);
 
 }  // namespace dmoe
