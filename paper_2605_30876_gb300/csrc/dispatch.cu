@@ -29,6 +29,8 @@ dispatch_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
   __shared__ int bad;
   const int tid = threadIdx.x, nthr = blockDim.x;
   const int pairs = T * k;
+  pdl_launch_dependents();
+  pdl_wait();
 
   if (tid == 0) bad = 0;
   for (int i = tid; i < nchunks * E; i += nthr) bits[i] = 0u;
@@ -95,19 +97,22 @@ size_t dispatch_smem_bytes(int T, int E) {
 
 cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s) {
   const size_t smem = dispatch_smem_bytes(a.T, a.E);
-  static bool attr_set = false;  // per process; max smem is a property of the kernel
-  if (!attr_set) {
+  static int attr_dev_mask = 0;  // the dynamic smem limit is a per-device function attribute
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
     cudaError_t e = cudaFuncSetAttribute(dispatch_kernel,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          200 * 1024);
     if (e != cudaSuccess) return e;
-    attr_set = true;
+    if (dev < 31) attr_dev_mask |= 1 << dev;
   }
   prof_begin(DMOE_KERNEL_DISPATCH, s);
-  dispatch_kernel<<<1, kDispatchThreads, smem, s>>>(a.topk_idx, a.T, a.E, a.k, a.n_unique,
-                                                    a.unique_ids, a.offsets, a.rows, a.pos,
-                                                    a.err);
+  cudaError_t e = launch_ex(dispatch_kernel, dim3(1), dim3(kDispatchThreads), smem, s, true,
+                            a.topk_idx, a.T, a.E, a.k, a.n_unique, a.unique_ids, a.offsets,
+                            a.rows, a.pos, a.err);
   prof_end(DMOE_KERNEL_DISPATCH, s);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

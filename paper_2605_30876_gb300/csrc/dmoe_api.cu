@@ -12,9 +12,12 @@ thread_local char g_last_error[256] = "";
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-// Split of the router's d-reduction: enough CTAs to spread the W_r read (about 128 tiles),
-// a divisor of d/32, at most 32 partial sums.
+// Router logits kernel choice: 0 = the full-d small-token kernel (d a multiple of 512 and
+// at most 128 tokens: logits written directly); otherwise the split of the tiled kernel's
+// d-reduction: enough CTAs to spread the W_r read (about 128 tiles), a divisor of d/32, at
+// most 32 partial sums.
 int router_splits(const dmoe_layer_desc& d) {
+  if ((long)d.n_blocks * d.block_size <= 128 && d.d_model % 512 == 0) return 0;
   const int tiles = ((d.n_experts + 63) / 64) * ((d.n_blocks * d.block_size + 31) / 32);
   int target = 128 / tiles;
   if (target < 1) target = 1;
@@ -79,7 +82,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   };
   w.err = take(sizeof(DevErrRecord));
   w.n_unique = take(sizeof(int32_t));
-  w.logits_part = take(sizeof(float) * w.router_splits * T * E);
+  w.logits_part = take(sizeof(float) * (w.router_splits == 0 ? 1 : w.router_splits) * T * E);
   w.probs = take(sizeof(float) * T * E);
   w.probs_hat = take(sizeof(float) * T * E);
   w.tk_idx = take(sizeof(int32_t) * T * k);
@@ -91,10 +94,6 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.xperm = take(2 * T * k * dm);
   w.h = take(2 * T * k * I);
   w.hs = take(2 * T * Is);
-  w.part_floats = (w.n_max <= 64) ? (size_t)kMaxPersistentCtas * 2 * w.n_max * kTileM : 0;
-  w.part = take(sizeof(float) * w.part_floats);
-  w.n_counters = kMaxPersistentCtas;
-  w.counters = take(sizeof(int32_t) * w.n_counters);
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
   w.total = off;
@@ -218,12 +217,8 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
   a.xperm = at<__nv_bfloat16>(ws, plan.xperm);
   a.h = at<__nv_bfloat16>(ws, plan.h);
   a.hs = at<__nv_bfloat16>(ws, plan.hs);
-  a.part = at<float>(ws, plan.part);
-  a.counters = at<int32_t>(ws, plan.counters);
   a.yslot = at<float>(ws, plan.yslot);
   a.yshared = at<float>(ws, plan.yshared);
-  a.n_counters = plan.n_counters;
-  a.part_floats = plan.part_floats;
   a.err = at<DevErrRecord>(ws, plan.err);
   a.T = desc->n_blocks * desc->block_size;
   a.d = desc->d_model;

@@ -68,15 +68,11 @@ struct Workspace {
   size_t xperm;        // bf16 [T*k, d]   x gathered in dispatch order
   size_t h;            // bf16 [T*k, I]   SwiGLU intermediate of the routed experts
   size_t hs;           // bf16 [T, I_s]   shared-expert intermediate
-  size_t part;         // fp32 split-K partials of the gate/up GEMM
-  size_t counters;     // int32 split-K tickets
   size_t yslot;        // fp32 [T*k, d]   gate-weighted expert outputs per (token, slot)
   size_t yshared;      // fp32 [T, d]
   size_t total;
   int router_splits;
   int n_max;           // token tile (MMA N) of the expert GEMMs
-  int n_counters;
-  size_t part_floats;
 };
 
 // Token tile of the expert GEMMs: every group's rows are covered by tiles of n_max.
@@ -130,9 +126,7 @@ struct ExpertArgs {
   __nv_bfloat16* y;
   // workspace
   __nv_bfloat16* xperm; __nv_bfloat16* h; __nv_bfloat16* hs;
-  float* part; int32_t* counters; float* yslot; float* yshared;
-  int n_counters;
-  size_t part_floats;
+  float* yslot; float* yshared;
   DevErrRecord* err;
   // shape
   int T, d, E, k, I, Is, n_max;
@@ -142,6 +136,30 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 // profiling events (dmoe_set_profile_events), per host thread
 void prof_begin(int kernel, cudaStream_t s);
 void prof_end(int kernel, cudaStream_t s);
+
+// Programmatic dependent launch: a kernel launched with `pdl` set may start while the
+// previous kernel on the stream is still running; it must call pdl_wait() before reading
+// anything that kernel writes. pdl_launch_dependents() lets the next kernel start early.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                      cudaStream_t s, bool pdl, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 // host helpers
 int device_sm_count();

@@ -29,6 +29,8 @@ router_logits_kernel(const __nv_bfloat16* __restrict__ x, const float* __restric
   const int e0 = blockIdx.x * kRtExp, t0 = blockIdx.y * kRtTok, split = blockIdx.z;
   const int dbeg = split * dchunk, dend = dbeg + dchunk;
   const int tid = threadIdx.x, ty = tid >> 4, tx = tid & 15;
+  pdl_launch_dependents();
+  pdl_wait();
   float acc[2][4];
 #pragma unroll
   for (int i = 0; i < 2; ++i)
@@ -75,6 +77,111 @@ router_logits_kernel(const __nv_bfloat16* __restrict__ x, const float* __restric
   }
 }
 
+// Logits of 8 tokens x 16 experts over the full d, for small token counts (no partial
+// sums): x and W_r slices are staged in shared memory by cp.async in 512-wide d chunks
+// (double-buffered); warp w reduces d sub-range w of every chunk, lane l owns token l/4 and
+// experts 4*(l%4)..+3; the 8 warp partials are added in warp order at the end.
+constexpr int kSmTok = 8, kSmExp = 16, kSmChunk = 512, kSmXPad = 8;
+
+__device__ __forceinline__ void cp_async16(void* dst, const void* src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(d), "l"(src), "r"(n)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() {
+  asm volatile("cp.async.commit_group;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_le1() {
+  asm volatile("cp.async.wait_group 1;" ::: "memory");
+}
+__device__ __forceinline__ void cp_async_wait_all() {
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(256)
+router_logits_small_kernel(const __nv_bfloat16* __restrict__ x, const float* __restrict__ w_r,
+                           float* __restrict__ logits, int T, int d, int E) {
+  extern __shared__ __align__(16) uint8_t lsm[];
+  // per buffer: W [kSmChunk][kSmExp] fp32, then x [kSmTok][kSmChunk + kSmXPad] bf16
+  constexpr int kWBytes = kSmChunk * kSmExp * 4;
+  constexpr int kXStride = kSmChunk + kSmXPad;
+  constexpr int kBufBytes = kWBytes + kSmTok * kXStride * 2;
+  const int e0 = blockIdx.x * kSmExp, t0 = blockIdx.y * kSmTok;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tl = lane >> 2, el = (lane & 3) * 4;
+  const int nchunks = d / kSmChunk;
+  pdl_launch_dependents();
+  pdl_wait();
+
+  auto stage = [&](int c, int buf) {
+    float* ws = reinterpret_cast<float*>(lsm + buf * kBufBytes);
+    __nv_bfloat16* xs = reinterpret_cast<__nv_bfloat16*>(lsm + buf * kBufBytes + kWBytes);
+    const int dbase = c * kSmChunk;
+    // W: kSmChunk rows x 64 B = 4 x 16 B per row
+    for (int i = tid; i < kSmChunk * 4; i += 256) {
+      const int r = i >> 2, q = i & 3;
+      const int e = e0 + q * 4;
+      const bool ok = e < E;
+      cp_async16(ws + r * kSmExp + q * 4, w_r + (size_t)(dbase + r) * E + (ok ? e : 0), ok);
+    }
+    // x: kSmTok rows x kSmChunk bf16 = 64 x 16 B per row
+    for (int i = tid; i < kSmTok * (kSmChunk / 8); i += 256) {
+      const int r = i / (kSmChunk / 8), q = i % (kSmChunk / 8);
+      const int t = t0 + r;
+      const bool ok = t < T;
+      cp_async16(xs + r * kXStride + q * 8, x + (size_t)(ok ? t : 0) * d + dbase + q * 8, ok);
+    }
+    cp_async_commit();
+  };
+
+  float acc0 = 0.f, acc1 = 0.f, acc2 = 0.f, acc3 = 0.f;
+  stage(0, 0);
+  for (int c = 0; c < nchunks; ++c) {
+    const int buf = c & 1;
+    if (c + 1 < nchunks) {
+      stage(c + 1, buf ^ 1);
+      cp_async_wait_le1();
+    } else {
+      cp_async_wait_all();
+    }
+    __syncthreads();
+    const float* ws = reinterpret_cast<const float*>(lsm + buf * kBufBytes);
+    const __nv_bfloat16* xs =
+        reinterpret_cast<const __nv_bfloat16*>(lsm + buf * kBufBytes + kWBytes);
+    const int dl0 = warp * (kSmChunk / 8);
+#pragma unroll 8
+    for (int j = 0; j < kSmChunk / 8; ++j) {
+      const int dl = dl0 + j;
+      const float xv = __bfloat162float(xs[tl * kXStride + dl]);
+      const float4 w = *reinterpret_cast<const float4*>(ws + dl * kSmExp + el);
+      acc0 = fmaf(xv, w.x, acc0);
+      acc1 = fmaf(xv, w.y, acc1);
+      acc2 = fmaf(xv, w.z, acc2);
+      acc3 = fmaf(xv, w.w, acc3);
+    }
+    __syncthreads();
+  }
+  // cross-warp sum in warp order
+  float* red = reinterpret_cast<float*>(lsm);  // [8 warps][kSmTok][kSmExp]
+  red[(warp * kSmTok + tl) * kSmExp + el + 0] = acc0;
+  red[(warp * kSmTok + tl) * kSmExp + el + 1] = acc1;
+  red[(warp * kSmTok + tl) * kSmExp + el + 2] = acc2;
+  red[(warp * kSmTok + tl) * kSmExp + el + 3] = acc3;
+  __syncthreads();
+  if (tid < kSmTok * kSmExp) {
+    const int t = tid / kSmExp, e = tid % kSmExp;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) v += red[(w * kSmTok + t) * kSmExp + e];
+    if (t0 + t < T && e0 + e < E) logits[(size_t)(t0 + t) * E + e0 + e] = v;
+  }
+}
+
+size_t router_small_smem() {
+  return 2 * ((size_t)kSmChunk * kSmExp * 4 + (size_t)kSmTok * (kSmChunk + kSmXPad) * 2);
+}
+
 // One CTA per token, thread e = expert e (E <= 256).
 __global__ void __launch_bounds__(256)
 router_softmax_kernel(const float* __restrict__ part, int splits, const float* __restrict__ bias,
@@ -85,9 +192,12 @@ router_softmax_kernel(const float* __restrict__ part, int splits, const float* _
   __shared__ float topv[kMaxTopK];
   __shared__ float scratch[32];
   const int t = blockIdx.x, e = threadIdx.x;
+  pdl_launch_dependents();
+  pdl_wait();
   float logit = -INFINITY;
   if (e < E) {
     float acc = 0.f;
+#pragma unroll 4
     for (int s = 0; s < splits; ++s) acc += part[((size_t)s * T + t) * E + e];
     if (bias != nullptr) acc += bias[e];
     logit = acc;
@@ -140,11 +250,15 @@ block_route_kernel(const float* __restrict__ probs, const float* __restrict__ pr
   const int b = blockIdx.x, tid = threadIdx.x;
   const int t0 = b * B;
   const bool live = tid < E;
+  pdl_launch_dependents();
+  pdl_wait();
 
   // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k)
   float S = 0.f;
-  if (live)
+  if (live) {
+#pragma unroll 8
     for (int i = 0; i < B; ++i) S += probs_hat[(size_t)(t0 + i) * E + tid];
+  }
   // Normalize: L1
   const float tot = block_sum(S, fscr);
   const float st = live ? S / tot : 0.f;
@@ -210,17 +324,37 @@ block_route_kernel(const float* __restrict__ probs, const float* __restrict__ pr
 }  // namespace
 
 cudaError_t launch_router(const RouterArgs& a, cudaStream_t s) {
-  const int dchunk = a.d / a.splits;
   prof_begin(DMOE_KERNEL_ROUTER, s);
-  dim3 g1((a.E + kRtExp - 1) / kRtExp, (a.T + kRtTok - 1) / kRtTok, a.splits);
-  router_logits_kernel<<<g1, 256, 0, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E, dchunk);
-  router_softmax_kernel<<<a.T, 256, 0, s>>>(a.logits_part, a.splits, a.bias, a.probs,
-                                            a.probs_hat, a.topk_idx, a.topk_gate, a.T, a.E,
-                                            a.k, a.mode);
+  if (a.splits == 0) {
+    // small token count: full-d tiles of 8 tokens x 16 experts, logits written directly
+    static int attr_dev_mask = 0;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    const size_t smem = router_small_smem();
+    if (dev < 31 && !(attr_dev_mask & (1 << dev))) {
+      cudaError_t e = cudaFuncSetAttribute(router_logits_small_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)smem);
+      if (e != cudaSuccess) return e;
+      attr_dev_mask |= 1 << dev;
+    }
+    dim3 g0((a.E + kSmExp - 1) / kSmExp, (a.T + kSmTok - 1) / kSmTok);
+    router_logits_small_kernel<<<g0, 256, smem, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E);
+  } else {
+    const int dchunk = a.d / a.splits;
+    dim3 g1((a.E + kRtExp - 1) / kRtExp, (a.T + kRtTok - 1) / kRtTok, a.splits);
+    router_logits_kernel<<<g1, 256, 0, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E, dchunk);
+  }
+  const int nsum = a.splits == 0 ? 1 : a.splits;
+  cudaError_t le = launch_ex(router_softmax_kernel, dim3(a.T), dim3(256), 0, s, true,
+                             a.logits_part, nsum, a.bias, a.probs, a.probs_hat, a.topk_idx,
+                             a.topk_gate, a.T, a.E, a.k, a.mode);
+  if (le != cudaSuccess) return le;
   if (a.mode == DMOE_ROUTE_BLOCK) {
-    block_route_kernel<<<a.n_blocks, 256, 0, s>>>(a.probs, a.probs_hat, a.E, a.k, a.B,
-                                                  a.top_p, a.topk_idx, a.topk_gate,
-                                                  a.coreset, a.coreset_size);
+    le = launch_ex(block_route_kernel, dim3(a.n_blocks), dim3(256), 0, s, true, a.probs,
+                   a.probs_hat, a.E, a.k, a.B, a.top_p, a.topk_idx, a.topk_gate, a.coreset,
+                   a.coreset_size);
+    if (le != cudaSuccess) return le;
   } else {
     cudaError_t e = cudaSuccess;
     if (a.coreset != nullptr)
