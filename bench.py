@@ -67,11 +67,12 @@ def layer_bytes(shape, U: float) -> float:
     return (U * 3 * d * I * 2 + 3 * d * Is * 2 + d * E * 4 + E * 4 + T * d * 2 * 2)
 
 
-def gate_up_bytes(shape, U: float) -> float:
-    """Algorithmic bytes of one gate/up launch: gate and up weights of the unique and shared
-    experts, the token rows read once, the bf16 SwiGLU output written."""
-    d, I, Is, T, k = shape.d_model, shape.d_ff, shape.d_ff_shared, shape.T, shape.top_k
-    return U * 2 * d * I * 2 + 2 * d * Is * 2 + T * d * 2 + (T * k * I + T * Is) * 2
+def experts_bytes(shape, U: float) -> float:
+    """Algorithmic bytes of one expert-kernel launch: the gate, up and down weights of the
+    unique and shared experts once, the token rows read once and the output rows written
+    once (bf16)."""
+    d, I, Is, T = shape.d_model, shape.d_ff, shape.d_ff_shared, shape.T
+    return U * 3 * d * I * 2 + 3 * d * Is * 2 + T * d * 2 * 2
 
 
 def layer_flops(shape) -> float:
@@ -195,10 +196,10 @@ class Arm:
         with torch.cuda.graph(g):
             for i in range(n_steps):
                 if events is not None:
-                    self.dm.dmoe_set_profile_events("gate_up", *events[i])
+                    self.dm.dmoe_set_profile_events("experts", *events[i])
                 self.step(first + i)
             if events is not None:
-                self.dm.dmoe_set_profile_events("gate_up", None, None)
+                self.dm.dmoe_set_profile_events("experts", None, None)
         return g
 
 
@@ -470,7 +471,7 @@ def main():
         side[name] = {"us_per_forward": us, "tokens_per_s": T * args.side_steps * world / s2,
                       "unique_experts_mean": u2,
                       "hbm_roofline_frac": layer_bytes(sh, u2) / (us * 1e-6) / 1e9 / hbm,
-                      "gate_up_us": k2 * 1e6 if k2 else None}
+                      "experts_us": k2 * 1e6 if k2 else None}
         del a2
 
     if rank != 0:
@@ -479,7 +480,7 @@ def main():
         return
 
     lbytes = layer_bytes(shape, U_mean)
-    gbytes = gate_up_bytes(shape, U_mean)
+    gbytes = experts_bytes(shape, U_mean)
     achieved = gbytes / kern_s / 1e9 if kern_s else None
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -497,9 +498,9 @@ def main():
                            "frac_measured_hbm": lbytes / (ms_per_step * 1e-3) / 1e9 / hbm,
                            "frac_nominal_8tbs": lbytes / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
                            "peak_source": peak_src},
-        "roofline": {"kernel": "gate_up", "bound": "hbm", "achieved": achieved, "peak": hbm,
+        "roofline": {"kernel": "moe_experts", "bound": "hbm", "achieved": achieved, "peak": hbm,
                      "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
-                     "traffic": traffic_from_profile("gate_up"),
+                     "traffic": traffic_from_profile("moe_experts"),
                      "algorithmic_bytes_per_launch": gbytes,
                      "launch_us": kern_s * 1e6 if kern_s else None,
                      "peak_source": f"{peak_src} hbm_gbs"},
@@ -507,7 +508,7 @@ def main():
         "e2e": None if secs_e2e is None else {"value": tokens_total / secs_e2e, "unit": UNIT,
                 "h2d_bytes_per_step": T * shape.d_model * 2,
                 "d2h_bytes_per_step": T * shape.d_model * 2},
-        "gpu_launches": args.steps * 8,
+        "gpu_launches": args.steps * 7,
         "flops_per_forward": layer_flops(shape),
         "clocks": clocks,
     }

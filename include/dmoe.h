@@ -152,10 +152,9 @@ typedef enum {
   DMOE_KERNEL_ROUTER = 0,     /* router logits, softmax/top-k and Algorithm 1 kernels */
   DMOE_KERNEL_DISPATCH = 1,   /* unique experts and expert -> token lists            */
   DMOE_KERNEL_GATHER = 2,     /* x rows in dispatch order                            */
-  DMOE_KERNEL_GATE_UP = 3,    /* grouped gate/up GEMM + SwiGLU                       */
-  DMOE_KERNEL_DOWN = 4,       /* grouped down GEMM, gate-weighted                    */
-  DMOE_KERNEL_COMBINE = 5,    /* sum over slots + shared expert -> y                 */
-  DMOE_KERNEL_COUNT = 6
+  DMOE_KERNEL_EXPERTS = 3,    /* grouped gate/up GEMM + SwiGLU and down GEMM         */
+  DMOE_KERNEL_COMBINE = 4,    /* gate-weighted sum over slots + shared expert -> y   */
+  DMOE_KERNEL_COUNT = 5
 } dmoe_kernel_id;
 
 /* Profiling aid, not part of the method: while set, every launch of `kernel` made by a

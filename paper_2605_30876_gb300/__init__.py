@@ -201,7 +201,7 @@ def dmoe_get_device_error(workspace, stream=None) -> Tuple[int, Tuple[int, int, 
     return st, (info[0], info[1], info[2])
 
 
-KERNELS = {"router": 0, "dispatch": 1, "gather": 2, "gate_up": 3, "down": 4, "combine": 5}
+KERNELS = {"router": 0, "dispatch": 1, "gather": 2, "experts": 3, "combine": 4}
 
 
 def dmoe_set_profile_events(kernel, ev_begin=None, ev_end=None) -> None:

@@ -94,6 +94,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.xperm = take(2 * T * k * dm);
   w.h = take(2 * T * k * I);
   w.hs = take(2 * T * Is);
+  w.h_ready = take(sizeof(int32_t) * experts_ready_counters((int)T, (int)E));
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
   w.total = off;
@@ -218,6 +219,7 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
   a.h = at<__nv_bfloat16>(ws, plan.h);
   a.hs = at<__nv_bfloat16>(ws, plan.hs);
   a.yslot = at<float>(ws, plan.yslot);
+  a.h_ready = at<int32_t>(ws, plan.h_ready);
   a.yshared = at<float>(ws, plan.yshared);
   a.err = at<DevErrRecord>(ws, plan.err);
   a.T = desc->n_blocks * desc->block_size;

@@ -68,7 +68,8 @@ struct Workspace {
   size_t xperm;        // bf16 [T*k, d]   x gathered in dispatch order
   size_t h;            // bf16 [T*k, I]   SwiGLU intermediate of the routed experts
   size_t hs;           // bf16 [T, I_s]   shared-expert intermediate
-  size_t yslot;        // fp32 [T*k, d]   gate-weighted expert outputs per (token, slot)
+  size_t h_ready;      // int32 [(E+1) * token tiles]: published gate/up tiles
+  size_t yslot;        // fp32 [T*k, d]   expert outputs per (token, slot)
   size_t yshared;      // fp32 [T, d]
   size_t total;
   int router_splits;
@@ -127,11 +128,13 @@ struct ExpertArgs {
   // workspace
   __nv_bfloat16* xperm; __nv_bfloat16* h; __nv_bfloat16* hs;
   float* yslot; float* yshared;
+  int32_t* h_ready;
   DevErrRecord* err;
   // shape
   int T, d, E, k, I, Is, n_max;
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
+int experts_ready_counters(int T, int E);
 
 // profiling events (dmoe_set_profile_events), per host thread
 void prof_begin(int kernel, cudaStream_t s);

@@ -5,23 +5,26 @@
 // tile, streamed by TMA with the 128-byte swizzle), the few tokens routed to an expert are
 // the N operand, K is the reduction dimension, and the fp32 accumulator lives in TMEM.
 //
-//   gather_kernel     x rows in dispatch order -> xperm [T*k, d]
-//   gate/up kernel    per (group, 64 rows of I, token tile): the A tile stacks 64 rows of
-//                     W_gate over the same 64 rows of W_up, so one M=128 MMA chain gives
-//                     gate (TMEM lanes 0-63) and up (lanes 64-127) of those rows; the
-//                     epilogue warps holding "up" pass it through shared memory to the
-//                     warps holding "gate", which write h = silu(gate) * up as bf16 H.
-//   down kernel       per (group, 128 rows of d, token tile): D = W_down * H^T; the
-//                     epilogue stores the fp32 rows per (token, slot)
-//   combine_kernel    y_t = sum over slots (slot order) of g_tj * row + shared -> bf16
+//   gather_kernel       x rows in dispatch order -> xperm [T*k, d]; clears the tile counters
+//   moe_experts_kernel  one persistent launch with two kinds of unit:
+//     gate/up unit      (group, 64 rows of I, token tile): the A tile stacks 64 rows of
+//                       W_gate over the same 64 rows of W_up, so one M=128 MMA chain gives
+//                       gate (TMEM lanes 0-63) and up (lanes 64-127) of those rows; the
+//                       epilogue warps holding "up" pass it through shared memory to the
+//                       warps holding "gate", which write h = silu(gate) * up as bf16 H and
+//                       then publish the tile (h_ready counter)
+//     down unit         (group, 128 rows of d, token tile): D = W_down * H^T; the epilogue
+//                       stores the fp32 rows per (token, slot)
+//   combine_kernel      y_t = sum over slots (slot order) of g_tj * row + shared -> bf16
 //
-// A group is one unique expert (dispatch order) or the shared expert (all T tokens). Both
-// GEMM kernels are persistent (one CTA per SM) and warp-specialised: warp 0 issues TMA,
-// warp 1 issues MMAs, warps 2-5 run the epilogue. The unit list is derived on the device
-// from the dispatch output, so no host round-trip is needed. Consecutive kernels are
-// chained with programmatic dependent launch: each kernel's set-up (barriers, TMEM,
-// tensor-map prefetch) overlaps the previous kernel, and griddepcontrol.wait orders the
-// reads of its outputs.
+// A group is one unique expert (dispatch order) or the shared expert (all T tokens). The
+// expert kernel is warp-specialised: warp 0 issues TMA, warp 1 issues MMAs, warps 2-5 run
+// the epilogue; each pipeline stage carries K = 128 (two 128-B-wide boxes per operand), the
+// access shape that keeps per-SM TMA streaming near its peak. The unit list is derived on
+// the device from the dispatch output, so no host round-trip is needed. Consecutive
+// kernels are chained with programmatic dependent launch: each kernel's set-up (barriers,
+// TMEM, tensor-map prefetch) overlaps the previous kernel, and griddepcontrol.wait orders
+// the reads of its outputs.
 #include <math.h>
 
 #include <mutex>
@@ -33,11 +36,14 @@ namespace dmoe {
 namespace {
 
 constexpr int kThreads = 192;                      // 6 warps
-constexpr int kATileBytes = kTileM * kTileK * 2;   // 16 KB: 128 rows x 64 K
-constexpr int kHalfTileBytes = kATileBytes / 2;    // 8 KB: 64 rows x 64 K
+constexpr int kBoxBytes = 64 * 128;                // one TMA box: 64 rows x 128 B
+constexpr int kKBoxes = 2;                         // K boxes per stage: K = 128 per stage
+constexpr int kStageK = kKBoxes * kTileK;
+constexpr int kATileBytes = kTileM * 128;          // 16 KB: 128 rows x 64 K (one K box)
+constexpr int kAStageBytes = kKBoxes * kATileBytes;  // 32 KB
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
-constexpr int kMaxStages = 12;
+constexpr int kMaxStages = 8;
 constexpr int kXchgStride = 17;                    // floats per row of the exchange buffer
 
 struct GemmParams {
@@ -48,13 +54,22 @@ struct GemmParams {
   __nv_bfloat16* hs;      // [T, Is]
   float* yslot;           // [T*k, d]
   float* yshared;         // [T, d]
+  int32_t* h_ready;       // [(E+1) * ntiles]: gate/up tiles done per (group, token tile)
   DevErrRecord* err;
   int T, d, E, k, I, Is;
   int n_max;              // token tile = rows of the B box
+  int ntiles;             // token tiles per group at most
   int stages;
   int n_acc;              // accumulator buffers in TMEM
   uint32_t tmem_cols;
   int has_shared;
+};
+
+struct Maps {
+  CUtensorMap wg, wu, sg, su;   // gate/up weights, 64-row boxes (routed [E*I,d], shared [Is,d])
+  CUtensorMap wd, sd;           // down weights, 128-row boxes (routed [E*d,I], shared [d,Is])
+  CUtensorMap xp, x;            // gate/up token rows: xperm [T*k,d], x [T,d]
+  CUtensorMap h, hs;            // down token rows: H [T*k,I], Hs [T,Is]
 };
 
 __device__ __forceinline__ void named_bar_sync(int id, int n) {
@@ -76,29 +91,37 @@ __device__ __forceinline__ bool epi_all(bool v) {
   return r != 0;
 }
 
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ int ld_acquire(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
 __device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
 
-template <bool kGateUp>
+// The expert FFN of one forward in one persistent launch. Units: first every gate/up tile
+// (group, 64 rows of I, token tile), then every down tile (group, 128 rows of d, token
+// tile); the shared expert's group comes first in both lists. A CTA takes units
+// blockIdx.x, blockIdx.x + gridDim.x, ... so its gate/up units always precede its down
+// units and a gate/up unit never waits on another unit. A down unit loads its W_down
+// tiles at once and only then waits (bounded) for the gate/up tiles of its token rows to
+// be published (h_ready), so weight streaming of both phases overlaps.
 __global__ void __launch_bounds__(kThreads, 1)
-expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, d] (64-row box) | W_down [E*d, I]
-                   const __grid_constant__ CUtensorMap tm_a1,   // W_up   [E*I, d] (64-row box) | unused
-                   const __grid_constant__ CUtensorMap tm_b,    // xperm [T*k, d] | H [T*k, I]
-                   const __grid_constant__ CUtensorMap tm_sa0,  // W_sgate [Is, d] | W_sdown [d, Is]
-                   const __grid_constant__ CUtensorMap tm_sa1,  // W_sup   [Is, d] | unused
-                   const __grid_constant__ CUtensorMap tm_sb,   // x [T, d] | Hs [T, Is]
-                   const GemmParams p) {
+moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
-  // 1024-B aligned base (the swizzled tiles need it)
   const uint32_t raw_addr = ptx::smem_addr(smem_raw);
-  uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+  uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);  // 1024-B aligned
 
-  constexpr int kRowsPerTile = kGateUp ? kTileM / 2 : kTileM;  // weight rows of I or d per tile
   const int stages = p.stages;
-  const uint32_t b_bytes = (uint32_t)p.n_max * 128u;
+  const uint32_t b_box = (uint32_t)p.n_max * 128u;            // one B box
+  const uint32_t b_stage = kKBoxes * b_box;
   const uint32_t off_a = 0;
-  const uint32_t off_b = off_a + (uint32_t)stages * kATileBytes;
-  const uint32_t off_x = off_b + (uint32_t)stages * b_bytes;           // epilogue exchange
-  const uint32_t x_bytes = kGateUp ? 2u * 64u * kXchgStride * 4u : 0u;  // 2 buffers [64][17] fp32
+  const uint32_t off_b = off_a + (uint32_t)stages * kAStageBytes;
+  const uint32_t off_x = off_b + (uint32_t)stages * b_stage;
+  const uint32_t x_bytes = 2u * 64u * kXchgStride * 4u;        // 2 buffers [64][17] fp32
   const uint32_t off_bar = (off_x + x_bytes + 7u) & ~7u;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + off_bar);
   uint64_t* empty = full + stages;
@@ -108,18 +131,16 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
   int* misc = reinterpret_cast<int*>(drain + 1);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(misc + 0);
   volatile int* s_abort = misc + 1;
-  int* s_sched = misc + 4;                     // G, U, units
-  int* g_prefix = misc + 8;                    // [kMaxGroups + 1] tile prefix
-  int* g_row0 = g_prefix + (kMaxGroups + 1);   // [kMaxGroups]
-  int* g_cnt = g_row0 + kMaxGroups;            // [kMaxGroups]
-  int* g_e = g_cnt + kMaxGroups;               // [kMaxGroups]
+  int* s_sched = misc + 4;                         // G, U, gu_units, dn_units
+  int* gu_prefix = misc + 8;                       // [kMaxGroups + 1], by slot
+  int* dn_prefix = gu_prefix + (kMaxGroups + 1);   // [kMaxGroups + 1], by slot
+  int* g_row0 = dn_prefix + (kMaxGroups + 1);      // by group
+  int* g_cnt = g_row0 + kMaxGroups;
+  int* g_e = g_cnt + kMaxGroups;
   float* xchg = reinterpret_cast<float*>(smem + off_x);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int mtiles_routed = (kGateUp ? p.I : p.d) / kRowsPerTile;
-  const int mtiles_shared = (kGateUp ? p.Is : p.d) / kRowsPerTile;
 
-  // ---------------- set-up that does not read the previous kernel's output
   if (tid == 0) {
     for (int s = 0; s < stages; ++s) {
       ptx::mbar_init(&full[s], 1);
@@ -132,43 +153,42 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
     ptx::mbar_init(drain, 1);
     ptx::fence_mbarrier_init();
     *s_abort = 0;
-    ptx::prefetch_tensormap(&tm_a0);
-    if (kGateUp) ptx::prefetch_tensormap(&tm_a1);
-    ptx::prefetch_tensormap(&tm_b);
-    if (p.has_shared) {
-      ptx::prefetch_tensormap(&tm_sa0);
-      ptx::prefetch_tensormap(&tm_sb);
-    }
+    ptx::prefetch_tensormap(&tm.wg);
+    ptx::prefetch_tensormap(&tm.wu);
+    ptx::prefetch_tensormap(&tm.wd);
+    ptx::prefetch_tensormap(&tm.xp);
+    ptx::prefetch_tensormap(&tm.h);
   }
   if (warp == 1) {
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
   pdl_launch_dependents();
-  pdl_wait();  // the dispatch output (and H for the down kernel) is complete from here on
+  pdl_wait();  // dispatch output and the gathered rows are complete from here on
 
-  // ---------------- the unit list, from the dispatch output
+  // ---------------- groups and unit lists (slot 0 = the shared expert when present)
   if (warp == 0) {
     int U = *p.n_unique;
     if (U < 0 || U > p.E) {
-      if (lane == 0) record_error(p.err, kErrBadDispatch, kGateUp ? kAtGateUp : kAtDown, U);
+      if (lane == 0) record_error(p.err, kErrBadDispatch, kAtGateUp, U);
       U = 0;
     }
     const int G = U + (p.has_shared ? 1 : 0);
-    int carry = 0;
+    int carry_gu = 0, carry_dn = 0;
     for (int base = 0; base < G; base += 32) {
-      const int g = base + lane;
-      int tiles = 0;
-      if (g < G) {
-        int cnt, row0, e, mt;
+      const int slot = base + lane;
+      int gu = 0, dn = 0;
+      if (slot < G) {
+        const int g = p.has_shared ? (slot == 0 ? U : slot - 1) : slot;
+        int cnt, row0, e, Ig;
         if (g < U) {
           row0 = p.offsets[g];
           cnt = p.offsets[g + 1] - row0;
           e = p.unique_ids[g];
-          mt = mtiles_routed;
+          Ig = p.I;
           if (e < 0 || e >= p.E || cnt < 0 || cnt > p.T || row0 < 0 ||
               row0 + cnt > p.T * p.k) {
-            record_error(p.err, kErrBadDispatch, kGateUp ? kAtGateUp : kAtDown, g);
+            record_error(p.err, kErrBadDispatch, kAtGateUp, g);
             cnt = 0;
             e = 0;
             row0 = 0;
@@ -177,50 +197,64 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
           row0 = 0;
           cnt = p.T;
           e = -1;
-          mt = mtiles_shared;
+          Ig = p.Is;
         }
         g_row0[g] = row0;
         g_cnt[g] = cnt;
         g_e[g] = e;
-        tiles = ((cnt + p.n_max - 1) / p.n_max) * mt;
+        const int nt = (cnt + p.n_max - 1) / p.n_max;
+        gu = nt * (Ig / 64);
+        dn = nt * (p.d / kTileM);
       }
-      int incl = tiles;
+      int igu = gu, idn = dn;
 #pragma unroll
       for (int o = 1; o < 32; o <<= 1) {
-        const int u = __shfl_up_sync(0xffffffffu, incl, o);
-        if (lane >= o) incl += u;
+        const int a = __shfl_up_sync(0xffffffffu, igu, o);
+        const int b = __shfl_up_sync(0xffffffffu, idn, o);
+        if (lane >= o) { igu += a; idn += b; }
       }
-      if (g < G) g_prefix[g + 1] = carry + incl;
-      carry += __shfl_sync(0xffffffffu, incl, 31);
+      if (slot < G) {
+        gu_prefix[slot + 1] = carry_gu + igu;
+        dn_prefix[slot + 1] = carry_dn + idn;
+      }
+      carry_gu += __shfl_sync(0xffffffffu, igu, 31);
+      carry_dn += __shfl_sync(0xffffffffu, idn, 31);
     }
     if (lane == 0) {
-      g_prefix[0] = 0;
+      gu_prefix[0] = 0;
+      dn_prefix[0] = 0;
       s_sched[0] = G;
       s_sched[1] = U;
-      s_sched[2] = carry;
+      s_sched[2] = carry_gu;
+      s_sched[3] = carry_dn;
     }
   }
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
-  const int G = s_sched[0], U = s_sched[1], units = s_sched[2];
+  const int G = s_sched[0], U = s_sched[1], n_gu = s_sched[2], n_dn = s_sched[3];
+  const int units = n_gu + n_dn;
 
-  // unit -> (group, m tile, n tile); m varies fastest so that neighbouring CTAs share the
-  // token tile of one expert
-  auto decode = [&](int u, int& g, int& m_idx, int& n_idx) {
-    int lo = 0, hi = G - 1;  // largest g with g_prefix[g] <= u
+  // unit -> phase, group, m tile, n tile
+  struct Unit { bool gu; int g, m, n; };
+  auto decode = [&](int u) -> Unit {
+    Unit r;
+    r.gu = u < n_gu;
+    const int* pre = r.gu ? gu_prefix : dn_prefix;
+    const int v = r.gu ? u : u - n_gu;
+    int lo = 0, hi = G - 1;
     while (lo < hi) {
       const int mid = (lo + hi + 1) >> 1;
-      if (g_prefix[mid] <= u) lo = mid; else hi = mid - 1;
+      if (pre[mid] <= v) lo = mid; else hi = mid - 1;
     }
-    g = lo;
-    const int local = u - g_prefix[g];
-    const int mt = (g < U) ? mtiles_routed : mtiles_shared;
-    n_idx = local / mt;
-    m_idx = local - n_idx * mt;
+    r.g = p.has_shared ? (lo == 0 ? U : lo - 1) : lo;
+    const int mt = r.gu ? ((r.g < U ? p.I : p.Is) / 64) : (p.d / kTileM);
+    const int local = v - pre[lo];
+    r.n = local / mt;
+    r.m = local - r.n * mt;
+    return r;
   };
-  const int where = kGateUp ? kAtGateUp : kAtDown;
   auto wait = [&](uint64_t* bar, uint32_t parity, int value) -> bool {
     if (ptx::mbar_try_wait(bar, parity)) return true;
     const uint64_t t0 = ptx::globaltimer_ns();
@@ -229,7 +263,7 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
       if ((i & 63u) == 0u) {
         if (*s_abort) return false;
         if (ptx::globaltimer_ns() - t0 > kWaitTimeoutNs) {
-          record_error(p.err, kErrTimeout, where, value);
+          record_error(p.err, kErrTimeout, kAtGateUp, value);
           *s_abort = 1;
           return false;
         }
@@ -242,34 +276,107 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
     if (lane == 0) {
       const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
       const uint64_t pol_x = ptx::policy_evict_last();    // activations: re-read by tiles
-      const uint32_t tx_bytes = kATileBytes + b_bytes;
+      const uint32_t tx_bytes = kAStageBytes + b_stage;
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        int g, m_idx, n_idx;
-        decode(u, g, m_idx, n_idx);
-        const bool shared = g >= U;
-        const int Kg = kGateUp ? p.d : (shared ? p.Is : p.I);
-        const int kc = Kg / kTileK;
-        const int arow = shared ? m_idx * kRowsPerTile
-                                : g_e[g] * (kGateUp ? p.I : p.d) + m_idx * kRowsPerTile;
-        const int brow = (shared ? 0 : g_row0[g]) + n_idx * p.n_max;
-        const CUtensorMap* ma0 = shared ? &tm_sa0 : &tm_a0;
-        const CUtensorMap* ma1 = shared ? &tm_sa1 : &tm_a1;
-        const CUtensorMap* mb = shared ? &tm_sb : &tm_b;
-        for (int c = 0; c < kc; ++c) {
-          if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
-          ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-          const int kx = c * kTileK;
-          uint8_t* a_dst = smem + off_a + stage * kATileBytes;
-          ptx::tma_load_2d(a_dst, ma0, &full[stage], kx, arow, pol_w);
-          if (kGateUp)
-            ptx::tma_load_2d(a_dst + kHalfTileBytes, ma1, &full[stage], kx, arow, pol_w);
-          ptx::tma_load_2d(smem + off_b + stage * b_bytes, mb, &full[stage], kx, brow, pol_x);
-          ++issued;
-          if (++stage == stages) { stage = 0; phase ^= 1u; }
+        const Unit un = decode(u);
+        const bool shared = un.g >= U;
+        if (un.gu) {
+          const int arow = shared ? un.m * 64 : g_e[un.g] * p.I + un.m * 64;
+          const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
+          const CUtensorMap* mg = shared ? &tm.sg : &tm.wg;
+          const CUtensorMap* mu = shared ? &tm.su : &tm.wu;
+          const CUtensorMap* mb = shared ? &tm.x : &tm.xp;
+          const int kc = p.d / kStageK;
+          for (int c = 0; c < kc; ++c) {
+            if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
+            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
+            uint8_t* b_dst = smem + off_b + stage * b_stage;
+#pragma unroll
+            for (int kb = 0; kb < kKBoxes; ++kb) {
+              const int kx = c * kStageK + kb * kTileK;
+              ptx::tma_load_2d(a_dst + kb * kATileBytes, mg, &full[stage], kx, arow, pol_w);
+              ptx::tma_load_2d(a_dst + kb * kATileBytes + kBoxBytes, mu, &full[stage], kx, arow,
+                               pol_w);
+              ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], kx, brow, pol_x);
+            }
+            ++issued;
+            if (++stage == stages) { stage = 0; phase ^= 1u; }
+          }
+        } else {
+          const int Kg = shared ? p.Is : p.I;
+          const int arow = shared ? un.m * kTileM : g_e[un.g] * p.d + un.m * kTileM;
+          const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
+          const CUtensorMap* ma = shared ? &tm.sd : &tm.wd;
+          const CUtensorMap* mb = shared ? &tm.hs : &tm.h;
+          const int kc = Kg / kStageK;
+          const int pre = kc < stages ? kc : stages;
+          const int stage0 = stage;
+          const uint32_t phase0 = phase;
+          // weights first: they do not depend on the gate/up phase
+          for (int c = 0; c < pre; ++c) {
+            if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
+            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
+#pragma unroll
+            for (int kb = 0; kb < kKBoxes; ++kb)
+              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], c * kStageK + kb * kTileK,
+                               arow, pol_w);
+            ++issued;
+            if (++stage == stages) { stage = 0; phase ^= 1u; }
+          }
+          if (!ok) break;
+          // then the H rows, once every gate/up tile of this token tile is published
+          const int target = Kg / 64;
+          const int32_t* flag = p.h_ready + un.g * p.ntiles + un.n;
+          if (ld_acquire(flag) < target) {
+            const uint64_t t0 = ptx::globaltimer_ns();
+            while (ld_acquire(flag) < target) {
+              __nanosleep(64);
+              if (*s_abort) { ok = false; break; }
+              if (ptx::globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                record_error(p.err, kErrTimeout, kAtDown, u);
+                *s_abort = 1;
+                ok = false;
+                break;
+              }
+            }
+          }
+          fence_proxy_async_global();
+          int st = stage0;
+          for (int c = 0; c < pre; ++c) {
+            if (ok) {
+              uint8_t* b_dst = smem + off_b + st * b_stage;
+#pragma unroll
+              for (int kb = 0; kb < kKBoxes; ++kb)
+                ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], c * kStageK + kb * kTileK, brow,
+                                 pol_x);
+            } else {
+              // keep the barrier accounting whole: complete the stage without B data
+              ptx::mbar_complete_tx_local(&full[st], b_stage);
+            }
+            if (++st == stages) st = 0;
+          }
+          (void)phase0;
+          if (!ok) break;
+          for (int c = pre; c < kc; ++c) {
+            if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
+            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
+            uint8_t* b_dst = smem + off_b + stage * b_stage;
+#pragma unroll
+            for (int kb = 0; kb < kKBoxes; ++kb) {
+              const int kx = c * kStageK + kb * kTileK;
+              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], kx, arow, pol_w);
+              ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], kx, brow, pol_x);
+            }
+            ++issued;
+            if (++stage == stages) { stage = 0; phase ^= 1u; }
+          }
         }
       }
       if (!ok) {
@@ -292,28 +399,31 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
-      const uint32_t acc_cols = (uint32_t)p.n_max;
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
-        int g, m_idx, n_idx;
-        decode(u, g, m_idx, n_idx);
-        const bool shared = g >= U;
-        const int Kg = kGateUp ? p.d : (shared ? p.Is : p.I);
-        const int kc = Kg / kTileK;
-        const int nvalid = min(p.n_max, g_cnt[g] - n_idx * p.n_max);
+        const Unit un = decode(u);
+        const bool shared = un.g >= U;
+        const int Kg = un.gu ? p.d : (shared ? p.Is : p.I);
+        const int kc = Kg / kStageK;
+        const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
         const uint32_t n_mma = (uint32_t)((nvalid + 15) & ~15);
         const uint32_t idesc = ptx::idesc_bf16(kTileM, n_mma);
         if (!wait(&acc_empty[acc], acc_phase ^ 1u, u)) { ok = false; break; }
         ptx::tc_fence_after();
-        const uint32_t d0 = tmem_base + (uint32_t)acc * acc_cols;
+        const uint32_t d0 = tmem_base + (uint32_t)acc * (uint32_t)p.n_max;
         for (int c = 0; c < kc; ++c) {
           if (!wait(&full[stage], phase, u)) { ok = false; break; }
           ptx::tc_fence_after();
-          const uint32_t a0 = ptx::smem_addr(smem + off_a + stage * kATileBytes);
-          const uint32_t bb = ptx::smem_addr(smem + off_b + stage * b_bytes);
+          if (!*s_abort) {
+            const uint32_t a0 = ptx::smem_addr(smem + off_a + stage * kAStageBytes);
+            const uint32_t b0 = ptx::smem_addr(smem + off_b + stage * b_stage);
 #pragma unroll
-          for (int kk = 0; kk < kTileK / 16; ++kk)
-            ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kk * 32), ptx::sdesc_k_sw128(bb + kk * 32),
-                          idesc, (c > 0 || kk > 0) ? 1u : 0u);
+            for (int kb = 0; kb < kKBoxes; ++kb)
+#pragma unroll
+              for (int kk = 0; kk < kTileK / 16; ++kk)
+                ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kATileBytes + kk * 32),
+                              ptx::sdesc_k_sw128(b0 + kb * b_box + kk * 32), idesc,
+                              (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
+          }
           ptx::mma_commit(&empty[stage]);
           if (++stage == stages) { stage = 0; phase ^= 1u; }
         }
@@ -334,23 +444,22 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
     int acc = 0, xb = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x) {
-      int g, m_idx, n_idx;
-      decode(u, g, m_idx, n_idx);
-      const bool shared = g >= U;
-      const int nvalid = min(p.n_max, g_cnt[g] - n_idx * p.n_max);
+      const Unit un = decode(u);
+      const bool shared = un.g >= U;
+      const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
       const int n_mma = (nvalid + 15) & ~15;
       if (!epi_all(wait(&acc_full[acc], acc_phase, u))) break;
       ptx::tc_fence_after();
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)acc * (uint32_t)p.n_max;
-      const int col0 = n_idx * p.n_max;              // first token column of the tile
-      if (kGateUp) {
+      const int col0 = un.n * p.n_max;              // first token column of the tile
+      if (un.gu) {
         // lanes 0-63: gate rows, lanes 64-127: up rows of the same 64 intermediate units
         const bool is_gate = q < 2;
         const int r64 = (q & 1) * 32 + lane;         // row within the 64-row slice
         const int Ig = shared ? p.Is : p.I;
         __nv_bfloat16* hout = shared ? p.hs : p.h;
-        const int hrow0 = (shared ? 0 : g_row0[g]) + col0;
-        const int icol = m_idx * 64 + r64;
+        const int hrow0 = (shared ? 0 : g_row0[un.g]) + col0;
+        const int icol = un.m * 64 + r64;
         for (int c0 = 0; c0 < n_mma; c0 += 16) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
@@ -370,10 +479,17 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
           }
           xb ^= 1;
         }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&acc_empty[acc]);
+        // publish: the H rows of this tile are visible to TMA loads of other CTAs
+        fence_proxy_async_global();
+        __threadfence();
+        named_bar_sync(2, 128);
+        if (tid == 64) atomicAdd(p.h_ready + un.g * p.ntiles + un.n, 1);
       } else {
-        const int drow = m_idx * kTileM + q * 32 + lane;
+        const int drow = un.m * kTileM + q * 32 + lane;
         float* out = shared ? p.yshared + (size_t)col0 * p.d
-                            : p.yslot + (size_t)(g_row0[g] + col0) * p.d;
+                            : p.yslot + (size_t)(g_row0[un.g] + col0) * p.d;
         for (int c0 = 0; c0 < n_mma; c0 += 16) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
@@ -382,9 +498,9 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
           for (int c = 0; c < 16; ++c)
             if (c0 + c < nvalid) out[(size_t)(c0 + c) * p.d + drow] = v[c];
         }
+        ptx::tc_fence_before();
+        ptx::mbar_arrive(&acc_empty[acc]);
       }
-      ptx::tc_fence_before();
-      ptx::mbar_arrive(&acc_empty[acc]);
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
     }
   }
@@ -398,12 +514,15 @@ expert_gemm_kernel(const __grid_constant__ CUtensorMap tm_a0,   // W_gate [E*I, 
   }
 }
 
-// xperm[r, :] = x[rows[r] / k, :]
+// xperm[r, :] = x[rows[r] / k, :]; block 0 also clears the gate/up tile counters.
 __global__ void __launch_bounds__(256)
 gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ rows,
-              __nv_bfloat16* __restrict__ xperm, int pairs, int k, int d) {
+              __nv_bfloat16* __restrict__ xperm, int32_t* __restrict__ h_ready, int n_ready,
+              int pairs, int k, int d) {
   pdl_launch_dependents();
   pdl_wait();
+  if (blockIdx.x == 0)
+    for (int i = threadIdx.x; i < n_ready; i += blockDim.x) h_ready[i] = 0;
   const int vec = d / 8;  // uint4 per row
   for (int r = blockIdx.x; r < pairs; r += gridDim.x) {
     const int t = rows[r] / k;
@@ -484,10 +603,10 @@ uint32_t pow2_cols(uint32_t c) {
   return r;
 }
 
-size_t gemm_fixed_smem(bool gate_up) {
+size_t experts_fixed_smem() {
   // alignment slack + exchange buffers + barriers + misc/group arrays
-  return 1024 + (gate_up ? 2 * 64 * kXchgStride * 4 : 0) + 8 +
-         8 * (2 * kMaxStages + 9) + sizeof(int) * (8 + 4 * (kMaxGroups + 1)) + 64;
+  return 1024 + 2 * 64 * kXchgStride * 4 + 8 + 8 * (2 * kMaxStages + 9) +
+         sizeof(int) * (8 + 5 * (kMaxGroups + 1)) + 64;
 }
 
 int max_smem_optin() {
@@ -497,53 +616,23 @@ int max_smem_optin() {
   return v;
 }
 
-template <bool kGateUp>
-cudaError_t launch_gemm(const CUtensorMap& a0, const CUtensorMap& a1, const CUtensorMap& b,
-                        const CUtensorMap& sa0, const CUtensorMap& sa1, const CUtensorMap& sb,
-                        GemmParams gp, cudaStream_t s) {
-  const size_t stage_bytes = (size_t)kATileBytes + (size_t)gp.n_max * 128;
-  const size_t fixed = gemm_fixed_smem(kGateUp);
-  const int limit = max_smem_optin();
-  int stages = (int)((limit - (int)fixed) / (int)stage_bytes);
-  if (stages > kMaxStages) stages = kMaxStages;
-  if (stages < 2) return cudaErrorInvalidConfiguration;
-  gp.stages = stages;
-  const uint32_t acc_cols = (uint32_t)gp.n_max;
-  gp.n_acc = (int)(512 / acc_cols);
-  if (gp.n_acc > 4) gp.n_acc = 4;
-  gp.tmem_cols = pow2_cols(gp.n_acc * acc_cols);
-  const size_t smem = fixed + (size_t)stages * stage_bytes;
-  static int attr_dev_mask = 0;  // per-device: the dynamic smem limit is a function attribute
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
-    cudaError_t e = cudaFuncSetAttribute(expert_gemm_kernel<kGateUp>,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
-    if (e != cudaSuccess) return e;
-    if (dev < 31) attr_dev_mask |= 1 << dev;
-  }
-  int grid = device_sm_count();
-  if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
-  const int kid = kGateUp ? DMOE_KERNEL_GATE_UP : DMOE_KERNEL_DOWN;
-  prof_begin(kid, s);
-  cudaError_t e = launch_ex(expert_gemm_kernel<kGateUp>, dim3(grid), dim3(kThreads), smem, s,
-                            true, a0, a1, b, sa0, sa1, sb, gp);
-  prof_end(kid, s);
-  if (e != cudaSuccess) return e;
-  return cudaGetLastError();
-}
-
 }  // namespace
+
+int experts_ready_counters(int T, int E) {
+  const int n_max = expert_n_max(T);
+  return (E + 1) * ((T + n_max - 1) / n_max);
+}
 
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   const int pairs = a.T * a.k;
   const bool has_shared = a.Is > 0;
-  // 1. gather x in dispatch order
+  const int n_ready = experts_ready_counters(a.T, a.E);
+  // 1. gather x in dispatch order; clear the gate/up tile counters
   {
     int grid = pairs < 1024 ? pairs : 1024;
     prof_begin(DMOE_KERNEL_GATHER, s);
     cudaError_t e = launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, true, a.x, a.rows,
-                              a.xperm, pairs, a.k, a.d);
+                              a.xperm, a.h_ready, n_ready, pairs, a.k, a.d);
     prof_end(DMOE_KERNEL_GATHER, s);
     if (e != cudaSuccess) return e;
   }
@@ -555,41 +644,60 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   gp.hs = a.hs;
   gp.yslot = a.yslot;
   gp.yshared = a.yshared;
+  gp.h_ready = a.h_ready;
   gp.err = a.err;
   gp.T = a.T; gp.d = a.d; gp.E = a.E; gp.k = a.k; gp.I = a.I; gp.Is = a.Is;
   gp.n_max = a.n_max;
+  gp.ntiles = (a.T + a.n_max - 1) / a.n_max;
   gp.has_shared = has_shared ? 1 : 0;
 
-  // 2. gate/up + SwiGLU: 64-row boxes of W_gate and W_up stacked in one A tile
-  CUtensorMap m_wg, m_wu, m_xp, m_sg, m_su, m_x;
-  bool ok = make_map(&m_wg, a.w_gate, (uint64_t)a.E * a.I, a.d, 64) &&
-            make_map(&m_wu, a.w_up, (uint64_t)a.E * a.I, a.d, 64) &&
-            make_map(&m_xp, a.xperm, (uint64_t)pairs, a.d, (uint32_t)a.n_max) &&
-            make_map(&m_x, a.x, (uint64_t)a.T, a.d, (uint32_t)a.n_max);
+  // 2. gate/up + SwiGLU and down projection in one persistent launch
+  Maps m;
+  bool ok = make_map(&m.wg, a.w_gate, (uint64_t)a.E * a.I, a.d, 64) &&
+            make_map(&m.wu, a.w_up, (uint64_t)a.E * a.I, a.d, 64) &&
+            make_map(&m.wd, a.w_down, (uint64_t)a.E * a.d, a.I, kTileM) &&
+            make_map(&m.xp, a.xperm, (uint64_t)pairs, a.d, (uint32_t)a.n_max) &&
+            make_map(&m.x, a.x, (uint64_t)a.T, a.d, (uint32_t)a.n_max) &&
+            make_map(&m.h, a.h, (uint64_t)pairs, a.I, (uint32_t)a.n_max);
   if (ok && has_shared)
-    ok = make_map(&m_sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
-         make_map(&m_su, a.ws_up, (uint64_t)a.Is, a.d, 64);
-  if (!has_shared) { m_sg = m_wg; m_su = m_wu; }
+    ok = make_map(&m.sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
+         make_map(&m.su, a.ws_up, (uint64_t)a.Is, a.d, 64) &&
+         make_map(&m.sd, a.ws_down, (uint64_t)a.d, a.Is, kTileM) &&
+         make_map(&m.hs, a.hs, (uint64_t)a.T, a.Is, (uint32_t)a.n_max);
+  if (!has_shared) { m.sg = m.wg; m.su = m.wu; m.sd = m.wd; m.hs = m.h; }
   if (!ok) return cudaErrorInvalidValue;
-  cudaError_t e = launch_gemm<true>(m_wg, m_wu, m_xp, m_sg, m_su, m_x, gp, s);
+
+  const size_t stage_bytes = (size_t)kAStageBytes + (size_t)kKBoxes * a.n_max * 128;
+  const size_t fixed = experts_fixed_smem();
+  const int limit = max_smem_optin();
+  int stages = (int)((limit - (int)fixed) / (int)stage_bytes);
+  if (stages > kMaxStages) stages = kMaxStages;
+  if (stages < 2) return cudaErrorInvalidConfiguration;
+  gp.stages = stages;
+  gp.n_acc = 512 / a.n_max;
+  if (gp.n_acc > 4) gp.n_acc = 4;
+  gp.tmem_cols = pow2_cols((uint32_t)(gp.n_acc * a.n_max));
+  const size_t smem = fixed + (size_t)stages * stage_bytes;
+  static int attr_dev_mask = 0;  // the dynamic smem limit is a per-device function attribute
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
+    cudaError_t e = cudaFuncSetAttribute(moe_experts_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
+    if (e != cudaSuccess) return e;
+    if (dev < 31) attr_dev_mask |= 1 << dev;
+  }
+  int grid = device_sm_count();
+  if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
+  prof_begin(DMOE_KERNEL_EXPERTS, s);
+  cudaError_t e = launch_ex(moe_experts_kernel, dim3(grid), dim3(kThreads), smem, s, true, m, gp);
+  prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
 
-  // 3. down projection
-  CUtensorMap m_wd, m_h, m_sd, m_hs;
-  ok = make_map(&m_wd, a.w_down, (uint64_t)a.E * a.d, a.I, kTileM) &&
-       make_map(&m_h, a.h, (uint64_t)pairs, a.I, (uint32_t)a.n_max);
-  if (ok && has_shared)
-    ok = make_map(&m_sd, a.ws_down, (uint64_t)a.d, a.Is, kTileM) &&
-         make_map(&m_hs, a.hs, (uint64_t)a.T, a.Is, (uint32_t)a.n_max);
-  if (!has_shared) { m_sd = m_wd; m_hs = m_h; }
-  if (!ok) return cudaErrorInvalidValue;
-  e = launch_gemm<false>(m_wd, m_wd, m_h, m_sd, m_sd, m_hs, gp, s);
-  if (e != cudaSuccess) return e;
-
-  // 4. gate-weighted combine
-  dim3 grid((a.d / 4 + 255) / 256, a.T);
+  // 3. gate-weighted combine
+  dim3 cgrid((a.d / 4 + 255) / 256, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
-  e = launch_ex(combine_kernel, grid, dim3(256), 0, s, true, a.yslot, a.yshared, a.pos,
+  e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared, a.pos,
                 a.topk_gate, a.y, a.k, a.d, has_shared ? 1 : 0);
   prof_end(DMOE_KERNEL_COMBINE, s);
   if (e != cudaSuccess) return e;
