@@ -76,7 +76,8 @@ typedef struct {
 } dmoe_layer_desc;
 
 /* Bytes of device workspace needed by every call below for this shape (host only; no
- * CUDA call). One workspace sized for the desc serves all calls on that desc. */
+ * CUDA call). One workspace sized for the desc serves all calls on that desc. A workspace
+ * must be zero-filled once before its first use; every call leaves it reusable. */
 dmoe_status dmoe_workspace_size(const dmoe_layer_desc* desc, size_t* bytes /* host */);
 
 /* Router and routing — §4.2 (s_i = Router(t_i); S_block = aggregation of the s_i;
@@ -180,7 +181,8 @@ dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end
  *  - The first call on each device looks up the array's device address (with that device
  *    current) and caches it; make that first call before any CUDA-graph stream capture.
  *  - All calls share the one array and it keeps the previous call's contents: each call
- *    clears the fault record it uses, and everything else it reads it has written first.
+ *    clears the fault record it uses, its completion counter returns to zero at the end of
+ *    every call, and everything else it reads it has written first.
  *    Calls whose executions overlap on the GPU (two streams, or two host threads) race on
  *    the array and give wrong results: serialise them.
  * Arguments, layouts and errors otherwise as for dmoe_router. */

@@ -12,12 +12,11 @@ thread_local char g_last_error[256] = "";
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
-// Router logits kernel choice: 0 = the full-d small-token kernel (d a multiple of 512 and
-// at most 128 tokens: logits written directly); otherwise the split of the tiled kernel's
-// d-reduction: enough CTAs to spread the W_r read (about 128 tiles), a divisor of d/32, at
-// most 32 partial sums.
+// Router logits kernel choice: 0 = the fused decode-size launch (logits written directly);
+// otherwise the split of the tiled kernel's d-reduction: enough CTAs to spread the W_r read
+// (about 128 tiles), a divisor of d/32, at most 32 partial sums.
 int router_splits(const dmoe_layer_desc& d) {
-  if ((long)d.n_blocks * d.block_size <= 128 && d.d_model % 512 == 0) return 0;
+  if (router_fused_ok(d.n_blocks * d.block_size, d.d_model)) return 0;
   const int tiles = ((d.n_experts + 63) / 64) * ((d.n_blocks * d.block_size + 31) / 32);
   int target = 128 / tiles;
   if (target < 1) target = 1;
@@ -152,7 +151,8 @@ bool all_aligned(std::initializer_list<const void*> ptrs) {
 dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* w_r,
                        const float* bias, int32_t* topk_idx, float* topk_gate, int32_t* coreset,
                        int32_t* coreset_size, float* probs, void* ws, const Workspace& plan,
-                       cudaStream_t s) {
+                       cudaStream_t s, const L2Prefetch& shared_pf = L2Prefetch(),
+                       const DispatchArgs* dsp = nullptr) {
   RouterArgs a{};
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.w_r = w_r;
@@ -174,7 +174,9 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.splits = plan.router_splits;
   a.top_p = desc->top_p;
   a.err = at<DevErrRecord>(ws, plan.err);
-  return cuda_status(launch_router(a, s));
+  a.shared_pf = shared_pf;
+  int32_t* ticket = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + plan.err + kTicketOffset);
+  return cuda_status(launch_router(a, dsp, ticket, s));
 }
 
 dmoe_status run_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx, int32_t* n_unique,
@@ -199,8 +201,10 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
                         const void* ws_up, const void* ws_down, const float* topk_gate,
                         const int32_t* n_unique, const int32_t* unique_ids,
                         const int32_t* offsets, const int32_t* rows, const int32_t* pos,
-                        void* y, void* ws, const Workspace& plan, cudaStream_t s) {
+                        void* y, void* ws, const Workspace& plan, cudaStream_t s,
+                        bool shared_prefetched = false) {
   ExpertArgs a{};
+  a.prefetch_shared = !shared_prefetched;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.w_gate = w_gate;
   a.w_up = w_up;
@@ -323,12 +327,30 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   int32_t* offs = at<int32_t>(workspace, plan.offsets);
   int32_t* rows = at<int32_t>(workspace, plan.rows);
   int32_t* pos = at<int32_t>(workspace, plan.pos);
-  st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s);
-  if (st != DMOE_OK) return st;
-  st = run_dispatch(desc, idx, nu, uid, offs, rows, pos, workspace, plan, s);
+  // In the fused call the shared expert's weights start streaming into L2 with the router.
+  L2Prefetch shared_pf;
+  if (desc->d_ff_shared > 0) {
+    shared_pf.ptr[0] = ws_gate;
+    shared_pf.ptr[1] = ws_up;
+    shared_pf.ptr[2] = ws_down;
+    shared_pf.bytes = (int64_t)desc->d_ff_shared * desc->d_model * 2;
+  }
+  DispatchArgs dsp{};
+  dsp.topk_idx = idx;
+  dsp.n_unique = nu;
+  dsp.unique_ids = uid;
+  dsp.offsets = offs;
+  dsp.rows = rows;
+  dsp.pos = pos;
+  dsp.T = desc->n_blocks * desc->block_size;
+  dsp.E = desc->n_experts;
+  dsp.k = desc->top_k;
+  dsp.err = at<DevErrRecord>(workspace, plan.err);
+  st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
+                  shared_pf, &dsp);
   if (st != DMOE_OK) return st;
   return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid, offs,
-                     rows, pos, y, workspace, plan, s);
+                     rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true);
 }
 
 dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) {

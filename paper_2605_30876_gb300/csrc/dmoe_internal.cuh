@@ -36,6 +36,7 @@ enum DevWhere : int32_t {
   kAtRouter = 1, kAtBlockRoute = 2, kAtDispatch = 3, kAtGateUp = 4, kAtDown = 5,
   kAtCombine = 6, kAtGather = 7,
 };
+constexpr size_t kTicketOffset = 64;
 struct DevErrRecord {
   int32_t code;
   int32_t where;
@@ -54,7 +55,7 @@ __device__ __forceinline__ void record_error(DevErrRecord* rec, int code, int wh
 // workspace layout (byte offsets from the workspace base; every region 256-B aligned)
 // ---------------------------------------------------------------------------------------
 struct Workspace {
-  size_t err;          // DevErrRecord
+  size_t err;          // DevErrRecord; the routing ticket (int32) sits at err + kTicketOffset
   size_t n_unique;     // int32 [1]  (used when the caller does not supply one)
   size_t logits_part;  // fp32 [router_splits, T, E]
   size_t probs;        // fp32 [T, E]
@@ -87,6 +88,35 @@ Workspace plan_workspace(const dmoe_layer_desc& d);
 // ---------------------------------------------------------------------------------------
 // launchers (each defined in its own translation unit)
 // ---------------------------------------------------------------------------------------
+// Weights to pull into L2 ahead of their use (bulk L2 prefetch; all null = none): three
+// matrices of `bytes` each per expert, expert e at ptr[m] + e * bytes.
+struct L2Prefetch {
+  const void* ptr[3] = {nullptr, nullptr, nullptr};
+  int64_t bytes = 0;
+};
+
+__device__ __forceinline__ void prefetch_l2_bulk(const void* p, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
+}
+constexpr int64_t kPrefetchChunk = 64 * 1024;
+
+// Issues chunk `c` (of `per_expert * 3 * n` chunks) of the prefetch list: matrix-major, then
+// expert (by position in `ids`, or 0..n-1 when ids is null), then chunk within the matrix.
+__device__ __forceinline__ void l2_prefetch_chunk(const L2Prefetch& pf, const int32_t* ids,
+                                                  int n, int c) {
+  const int64_t per = (pf.bytes + kPrefetchChunk - 1) / kPrefetchChunk;
+  const int64_t per_mat = per * n;
+  const int m = (int)(c / per_mat);
+  const int64_t r = c - m * per_mat;
+  const int u = (int)(r / per);
+  const int64_t off = (r - (int64_t)u * per) * kPrefetchChunk;
+  const int e = ids != nullptr ? ids[u] : u;
+  const int64_t len = pf.bytes - off < kPrefetchChunk ? pf.bytes - off : kPrefetchChunk;
+  if (m < 3 && pf.ptr[m] != nullptr && len > 0)
+    prefetch_l2_bulk(static_cast<const uint8_t*>(pf.ptr[m]) + (int64_t)e * pf.bytes + off,
+                     (uint32_t)len);
+}
+
 struct RouterArgs {
   const __nv_bfloat16* x;
   const float* w_r;
@@ -101,8 +131,8 @@ struct RouterArgs {
   int T, d, E, k, B, n_blocks, mode, splits;
   float top_p;
   DevErrRecord* err;
+  L2Prefetch shared_pf;   // the shared expert's weights (one "expert")
 };
-cudaError_t launch_router(const RouterArgs& a, cudaStream_t s);
 
 struct DispatchArgs {
   const int32_t* topk_idx;
@@ -115,6 +145,13 @@ struct DispatchArgs {
   DevErrRecord* err;
 };
 cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s);
+
+// Routing of one forward. With `dsp` set, the dispatch is computed too (inside the fused
+// decode-size launch, or by launch_dispatch otherwise). `ticket` is a workspace int that is
+// zero between calls.
+cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t* ticket,
+                          cudaStream_t s);
+bool router_fused_ok(int T, int d);
 
 struct ExpertArgs {
   // inputs
@@ -130,6 +167,7 @@ struct ExpertArgs {
   float* yslot; float* yshared;
   int32_t* h_ready;
   DevErrRecord* err;
+  bool prefetch_shared;   // the shared expert's weights were not prefetched by the router
   // shape
   int T, d, E, k, I, Is, n_max;
 };

@@ -56,6 +56,8 @@ struct GemmParams {
   float* yshared;         // [T, d]
   int32_t* h_ready;       // [(E+1) * ntiles]: gate/up tiles done per (group, token tile)
   DevErrRecord* err;
+  const void* w_down;     // routed W_down, prefetched into L2 for the unique experts
+  const void* ws_gate; const void* ws_up; const void* ws_down;  // shared, prefetched if set
   int T, d, E, k, I, Is;
   int n_max;              // token tile = rows of the B box
   int ntiles;             // token tiles per group at most
@@ -94,6 +96,9 @@ __device__ __forceinline__ bool epi_all(bool v) {
 __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
+__device__ __forceinline__ void red_release_add(int32_t* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
 __device__ __forceinline__ int ld_acquire(const int32_t* p) {
   int v;
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -101,6 +106,19 @@ __device__ __forceinline__ int ld_acquire(const int32_t* p) {
 }
 
 __device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
+
+// Debug builds (-DDMOE_TRACE) record a per-CTA timeline of the expert kernel: slot 0 entry,
+// 1 after the unit list, 62 exit; for the i-th unit of the CTA (i < 8), at 2 + 6i: unit id,
+// producer start, last TMA issued, H ready (down units), last MMA commit, epilogue done;
+// at 50 + i: the epilogue's first TMEM read of that unit.
+#ifdef DMOE_TRACE
+__device__ uint64_t g_trace[kMaxPersistentCtas * 64];
+#define DMOE_TRACE_AT(slot) (g_trace[blockIdx.x * 64 + (slot)] = ptx::globaltimer_ns())
+#define DMOE_TRACE_SET(slot, v) (g_trace[blockIdx.x * 64 + (slot)] = (uint64_t)(v))
+#else
+#define DMOE_TRACE_AT(slot) ((void)0)
+#define DMOE_TRACE_SET(slot, v) ((void)0)
+#endif
 
 // The expert FFN of one forward in one persistent launch. Units: first every gate/up tile
 // (group, 64 rows of I, token tile), then every down tile (group, 128 rows of d, token
@@ -140,6 +158,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   float* xchg = reinterpret_cast<float*>(smem + off_x);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  if (tid == 0) DMOE_TRACE_AT(0);
 
   if (tid == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -235,6 +254,28 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   const uint32_t tmem_base = *s_tmem;
   const int G = s_sched[0], U = s_sched[1], n_gu = s_sched[2], n_dn = s_sched[3];
   const int units = n_gu + n_dn;
+  if (tid == 0) DMOE_TRACE_AT(1);
+  if (tid == 64) {
+    // Pull the down-projection weights of every unique expert into L2 now, spread over all
+    // CTAs: the down units of the second wave then read them from L2, and HBM keeps
+    // streaming while the gate/up results are produced and published.
+    L2Prefetch pf;
+    pf.ptr[2] = p.w_down;
+    pf.bytes = (int64_t)p.d * p.I * 2;
+    const int64_t per = (pf.bytes + kPrefetchChunk - 1) / kPrefetchChunk;
+    const int total = (int)(3 * per * U);
+    for (int c = (int)(2 * per * U) + blockIdx.x; c < total; c += gridDim.x)
+      l2_prefetch_chunk(pf, p.unique_ids, U, c);
+    if (p.ws_gate != nullptr) {
+      L2Prefetch sp;
+      sp.ptr[0] = p.ws_gate;
+      sp.ptr[1] = p.ws_up;
+      sp.ptr[2] = p.ws_down;
+      sp.bytes = (int64_t)p.d * p.Is * 2;
+      const int sper = (int)((sp.bytes + kPrefetchChunk - 1) / kPrefetchChunk);
+      for (int c = blockIdx.x; c < 3 * sper; c += gridDim.x) l2_prefetch_chunk(sp, nullptr, 1, c);
+    }
+  }
 
   // unit -> phase, group, m tile, n tile
   struct Unit { bool gu; int g, m, n; };
@@ -281,9 +322,11 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       uint32_t phase = 0;
       int issued = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int li = 0;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++li) {
         const Unit un = decode(u);
         const bool shared = un.g >= U;
+        if (li < 8) { DMOE_TRACE_SET(2 + 6 * li, u); DMOE_TRACE_AT(3 + 6 * li); }
         if (un.gu) {
           const int arow = shared ? un.m * 64 : g_e[un.g] * p.I + un.m * 64;
           const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
@@ -347,6 +390,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
             }
           }
           fence_proxy_async_global();
+          if (li < 8) DMOE_TRACE_AT(5 + 6 * li);
           int st = stage0;
           for (int c = 0; c < pre; ++c) {
             if (ok) {
@@ -378,6 +422,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
             if (++stage == stages) { stage = 0; phase ^= 1u; }
           }
         }
+        if (li < 8) DMOE_TRACE_AT(4 + 6 * li);
       }
       if (!ok) {
         // let the copies already in flight land before the CTA exits
@@ -399,7 +444,8 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       int stage = 0, acc = 0;
       uint32_t phase = 0, acc_phase = 0;
       bool ok = true;
-      for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
+      int li = 0;
+      for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++li) {
         const Unit un = decode(u);
         const bool shared = un.g >= U;
         const int Kg = un.gu ? p.d : (shared ? p.Is : p.I);
@@ -429,6 +475,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         }
         if (!ok) break;
         ptx::mma_commit(&acc_full[acc]);
+        if (li < 8) DMOE_TRACE_AT(6 + 6 * li);
         if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
       }
       // make sure no MMA is still running when TMEM is released
@@ -441,15 +488,16 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     // ================= epilogue: warps 2..5, TMEM lanes 32*(warp%4) ..
     const int q = warp & 3;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    int acc = 0, xb = 0;
+    int acc = 0, xb = 0, li = 0;
     uint32_t acc_phase = 0;
-    for (int u = blockIdx.x; u < units; u += gridDim.x) {
+    for (int u = blockIdx.x; u < units; u += gridDim.x, ++li) {
       const Unit un = decode(u);
       const bool shared = un.g >= U;
       const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
       const int n_mma = (nvalid + 15) & ~15;
       if (!epi_all(wait(&acc_full[acc], acc_phase, u))) break;
       ptx::tc_fence_after();
+      if (tid == 64 && li < 8) DMOE_TRACE_AT(50 + li);
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)acc * (uint32_t)p.n_max;
       const int col0 = un.n * p.n_max;              // first token column of the tile
       if (un.gu) {
@@ -479,13 +527,14 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           }
           xb ^= 1;
         }
+        if (tid == 64 && li < 4) DMOE_TRACE_AT(54 + li);
         ptx::tc_fence_before();
         ptx::mbar_arrive(&acc_empty[acc]);
-        // publish: the H rows of this tile are visible to TMA loads of other CTAs
-        fence_proxy_async_global();
-        __threadfence();
+        // publish the tile: the barrier orders every epilogue thread's H stores before one
+        // release add; a reader acquires the counter, then fences the async proxy
         named_bar_sync(2, 128);
-        if (tid == 64) atomicAdd(p.h_ready + un.g * p.ntiles + un.n, 1);
+        if (tid == 64 && li < 8) DMOE_TRACE_AT(58 + (li < 4 ? li : 3));
+        if (tid == 64) red_release_add(p.h_ready + un.g * p.ntiles + un.n, 1);
       } else {
         const int drow = un.m * kTileM + q * 32 + lane;
         float* out = shared ? p.yshared + (size_t)col0 * p.d
@@ -501,6 +550,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         ptx::tc_fence_before();
         ptx::mbar_arrive(&acc_empty[acc]);
       }
+      if (tid == 64 && li < 8) DMOE_TRACE_AT(7 + 6 * li);
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
     }
   }
@@ -508,6 +558,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  if (tid == 0) DMOE_TRACE_AT(62);
   if (warp == 1) {
     __syncwarp();
     ptx::tmem_dealloc(tmem_base, p.tmem_cols);
@@ -618,6 +669,17 @@ int max_smem_optin() {
 
 }  // namespace
 
+#ifdef DMOE_TRACE
+extern "C" int dmoe_debug_trace(void* host, size_t bytes) {
+  if (bytes > sizeof(g_trace)) bytes = sizeof(g_trace);
+  return (int)cudaMemcpyFromSymbol(host, g_trace, bytes);
+}
+extern "C" int dmoe_debug_trace_clear() {
+  static uint64_t zeros[kMaxPersistentCtas * 64] = {};
+  return (int)cudaMemcpyToSymbol(g_trace, zeros, sizeof(zeros));
+}
+#endif
+
 int experts_ready_counters(int T, int E) {
   const int n_max = expert_n_max(T);
   return (E + 1) * ((T + n_max - 1) / n_max);
@@ -646,6 +708,12 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   gp.yshared = a.yshared;
   gp.h_ready = a.h_ready;
   gp.err = a.err;
+  gp.w_down = a.w_down;
+  if (has_shared && a.prefetch_shared) {
+    gp.ws_gate = a.ws_gate;
+    gp.ws_up = a.ws_up;
+    gp.ws_down = a.ws_down;
+  }
   gp.T = a.T; gp.d = a.d; gp.E = a.E; gp.k = a.k; gp.I = a.I; gp.Is = a.Is;
   gp.n_max = a.n_max;
   gp.ntiles = (a.T + a.n_max - 1) / a.n_max;

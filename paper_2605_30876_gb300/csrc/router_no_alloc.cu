@@ -111,7 +111,7 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
   a.splits = plan.router_splits;
   a.top_p = desc->top_p;
   a.err = reinterpret_cast<DevErrRecord*>(base + plan.err);
-  e = launch_router(a, s);
+  e = launch_router(a, nullptr, reinterpret_cast<int32_t*>(base + plan.err + kTicketOffset), s);
   if (e != cudaSuccess) {
     set_last_error(e);
     return DMOE_ERR_CUDA;
