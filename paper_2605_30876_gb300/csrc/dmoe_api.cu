@@ -16,7 +16,7 @@ size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 // otherwise the split of the tiled kernel's d-reduction: enough CTAs to spread the W_r read
 // (about 128 tiles), a divisor of d/32, at most 32 partial sums.
 int router_splits(const dmoe_layer_desc& d) {
-  if (router_fused_ok(d.n_blocks * d.block_size, d.d_model)) return 0;
+  if (route_cluster_ok(d.n_blocks * d.block_size, d.d_model, d.n_experts)) return 0;
   const int tiles = ((d.n_experts + 63) / 64) * ((d.n_blocks * d.block_size + 31) / 32);
   int target = 128 / tiles;
   if (target < 1) target = 1;
@@ -80,6 +80,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
     return o;
   };
   w.err = take(sizeof(DevErrRecord));
+  w.tickets = take(sizeof(int32_t) * kRouteTickets);
   w.n_unique = take(sizeof(int32_t));
   w.logits_part = take(sizeof(float) * (w.router_splits == 0 ? 1 : w.router_splits) * T * E);
   w.probs = take(sizeof(float) * T * E);
@@ -159,6 +160,7 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.bias = bias;
   a.logits_part = at<float>(ws, plan.logits_part);
   a.probs = probs != nullptr ? probs : at<float>(ws, plan.probs);
+  a.probs_requested = probs != nullptr;
   a.probs_hat = at<float>(ws, plan.probs_hat);
   a.topk_idx = topk_idx;
   a.topk_gate = topk_gate;
@@ -175,8 +177,7 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.top_p = desc->top_p;
   a.err = at<DevErrRecord>(ws, plan.err);
   a.shared_pf = shared_pf;
-  int32_t* ticket = reinterpret_cast<int32_t*>(static_cast<uint8_t*>(ws) + plan.err + kTicketOffset);
-  return cuda_status(launch_router(a, dsp, ticket, s));
+  return cuda_status(launch_router(a, dsp, at<int32_t>(ws, plan.tickets), s));
 }
 
 dmoe_status run_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx, int32_t* n_unique,

@@ -36,7 +36,7 @@ enum DevWhere : int32_t {
   kAtRouter = 1, kAtBlockRoute = 2, kAtDispatch = 3, kAtGateUp = 4, kAtDown = 5,
   kAtCombine = 6, kAtGather = 7,
 };
-constexpr size_t kTicketOffset = 64;
+constexpr int kRouteTickets = 256;
 struct DevErrRecord {
   int32_t code;
   int32_t where;
@@ -55,7 +55,8 @@ __device__ __forceinline__ void record_error(DevErrRecord* rec, int code, int wh
 // workspace layout (byte offsets from the workspace base; every region 256-B aligned)
 // ---------------------------------------------------------------------------------------
 struct Workspace {
-  size_t err;          // DevErrRecord; the routing ticket (int32) sits at err + kTicketOffset
+  size_t err;          // DevErrRecord
+  size_t tickets;      // int32 [kRouteTickets]: stage counters of the routing launch (zero between calls)
   size_t n_unique;     // int32 [1]  (used when the caller does not supply one)
   size_t logits_part;  // fp32 [router_splits, T, E]
   size_t probs;        // fp32 [T, E]
@@ -117,6 +118,14 @@ __device__ __forceinline__ void l2_prefetch_chunk(const L2Prefetch& pf, const in
                      (uint32_t)len);
 }
 
+// Spreads the chunks of one expert's three matrices over `nctas` CTAs (call from one thread).
+__device__ __forceinline__ void issue_shared_prefetch(const L2Prefetch& pf, int cta, int nctas) {
+  if (pf.bytes > 0) {
+    const int per = (int)((pf.bytes + kPrefetchChunk - 1) / kPrefetchChunk);
+    for (int c = cta; c < 3 * per; c += nctas) l2_prefetch_chunk(pf, nullptr, 1, c);
+  }
+}
+
 struct RouterArgs {
   const __nv_bfloat16* x;
   const float* w_r;
@@ -132,6 +141,7 @@ struct RouterArgs {
   float top_p;
   DevErrRecord* err;
   L2Prefetch shared_pf;   // the shared expert's weights (one "expert")
+  bool probs_requested;   // the caller wants the scores in `probs`
 };
 
 struct DispatchArgs {
@@ -147,11 +157,13 @@ struct DispatchArgs {
 cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s);
 
 // Routing of one forward. With `dsp` set, the dispatch is computed too (inside the fused
-// decode-size launch, or by launch_dispatch otherwise). `ticket` is a workspace int that is
-// zero between calls.
-cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t* ticket,
+// decode-size launch, or by launch_dispatch otherwise). `tickets` is a workspace array of
+// kRouteTickets ints that is zero between calls.
+cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                           cudaStream_t s);
-bool router_fused_ok(int T, int d);
+bool route_cluster_ok(int T, int d, int E);
+cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
+                                 cudaStream_t s);
 
 struct ExpertArgs {
   // inputs
@@ -184,6 +196,24 @@ void prof_end(int kernel, cudaStream_t s);
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_launch_dependents() {
   asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                           cudaStream_t s, int cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = cluster_x;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
 }
 
 template <typename... KArgs, typename... Args>

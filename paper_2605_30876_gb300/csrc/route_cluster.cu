@@ -1,0 +1,302 @@
+// Routing of a decode-sized forward (T <= 64 tokens) in one launch of 8-CTA thread-block
+// clusters (§4.2 router and Algorithm 1 of arXiv 2605.30876, plus the dispatch).
+//
+// Cluster c owns 32 experts; CTA r of the cluster owns the r-th eighth of d:
+//   1. logits: TMA brings the W_r slice (d/8 rows x 32 experts, 128-B rows) and the x
+//      slice (T rows x d/8); fp32 FFMA gives partial logits [T x 32] in shared memory;
+//      CTA r then adds, in rank order, the eight partials of the tokens t = r (mod 8) over
+//      distributed shared memory and writes those logits.
+//   2. one atomic ticket: the last cluster to finish continues; the others exit.
+//   3. scores: one warp per token (8 CTAs x 8 warps = 64 tokens): softmax, top-k (token
+//      mode: the routing; block mode: TopKMask).
+//   4. Algorithm 1 for block b by CTA b mod 8 (blocks in parallel).
+//   5. dispatch by CTA 0 (fused layer call).
+// Stages 3-5 are separated by cluster barriers (release/acquire at cluster scope); data
+// written to global memory by other CTAs is read past the L1 (ld.global.cg).
+#include <math.h>
+
+#include "dispatch_impl.cuh"
+#include "dmoe_internal.cuh"
+#include "routing_device.cuh"
+
+namespace dmoe {
+namespace {
+
+constexpr int kCl = 8;                 // CTAs per cluster (split of d)
+constexpr int kClExp = 32;             // experts per cluster
+constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
+constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
+
+struct ClusterArgs {
+  CUtensorMap wmap;   // W_r [d, E] fp32, box 32 experts x d/8 rows
+  CUtensorMap xmap;   // x [T, d] bf16, box d/8 columns x T rows
+  RouterArgs r;
+  DispatchArgs dsp;   // dsp.n_unique == nullptr: no dispatch
+  int32_t* ticket;    // zero between calls
+};
+
+__device__ __forceinline__ uint32_t s_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;"
+               ::: "memory");
+}
+// address of the same shared variable in CTA `rank` of the cluster
+__device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(s_addr(p)), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ float ld_peer_f32(uint32_t addr) {
+  float v;
+  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
+  return v;
+}
+__device__ __forceinline__ void st_peer_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
+}
+
+__global__ void __launch_bounds__(256, 1)
+route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
+  extern __shared__ __align__(128) uint8_t dsm_raw[];
+  uint8_t* dsm = dsm_raw + ((128u - (s_addr(dsm_raw) & 127u)) & 127u);
+  __shared__ __align__(8) uint64_t s_bar;
+  __shared__ uint32_t s_last;
+  __shared__ float s_part[kClMaxTok * kClExp];                     // partial logits [T][32]
+  __shared__ uint32_t s_bits[(kClMaxTok / 32) * kMaxExperts];
+  __shared__ uint16_t s_base[(kClMaxTok / 32) * kMaxExperts];
+  const RouterArgs& a = f.r;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int T = a.T, E = a.E, k = a.k, B = a.B;
+  const uint32_t rank = cluster_rank();
+  const int DC = a.d / kCl;                          // rows of d in this CTA's slice
+  const int e0 = blockIdx.y * kClExp;
+  const int n_clusters = gridDim.y;
+  pdl_launch_dependents();
+  pdl_wait();
+
+  // ---- 1. partial logits over this CTA's slice of d
+  float* Ws = reinterpret_cast<float*>(dsm);                                   // [DC][32]
+  __nv_bfloat16* Xs = reinterpret_cast<__nv_bfloat16*>(dsm + kClMaxDChunk * kClExp * 4);  // [T][DC]
+  if (tid == 0) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(s_addr(&s_bar)) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.wmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.xmap)) : "memory");
+    const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)T * DC * 2;
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_addr(&s_bar)),
+                 "r"(bytes)
+                 : "memory");
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Ws)),
+        "l"(reinterpret_cast<uint64_t>(&f.wmap)), "r"(s_addr(&s_bar)), "r"(e0),
+        "r"((int)rank * DC)
+        : "memory");
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Xs)),
+        "l"(reinterpret_cast<uint64_t>(&f.xmap)), "r"(s_addr(&s_bar)), "r"((int)rank * DC),
+        "r"(0)
+        : "memory");
+    issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
+  }
+  __syncthreads();
+  {
+    uint64_t t0;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t0));
+    for (;;) {
+      uint32_t ok;
+      asm volatile(
+          "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], 0;\n\t"
+          "selp.u32 %0, 1, 0, p;\n\t}"
+          : "=r"(ok)
+          : "r"(s_addr(&s_bar))
+          : "memory");
+      if (ok) break;
+      uint64_t t;
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+      if (t - t0 > 1000000000ull) {
+        if (tid == 0) record_error(a.err, kErrTimeout, kAtRouter, (int)rank);
+        break;
+      }
+    }
+  }
+  // lane = expert e0 + lane, warp w = tokens w, w + 8, ...
+  constexpr int kTokPerWarp = kClMaxTok / 8;
+  float acc[kTokPerWarp];
+#pragma unroll
+  for (int i = 0; i < kTokPerWarp; ++i) acc[i] = 0.f;
+  const int ntok = (T - warp + 7) / 8;   // tokens of this warp
+  for (int dd = 0; dd < DC; dd += 2) {
+    const float w0 = Ws[dd * kClExp + lane];
+    const float w1 = Ws[(dd + 1) * kClExp + lane];
+#pragma unroll
+    for (int i = 0; i < kTokPerWarp; ++i) {
+      if (i < ntok) {
+        const __nv_bfloat162 xv =
+            *reinterpret_cast<const __nv_bfloat162*>(Xs + (size_t)(warp + 8 * i) * DC + dd);
+        acc[i] = fmaf(__low2float(xv), w0, acc[i]);
+        acc[i] = fmaf(__high2float(xv), w1, acc[i]);
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kTokPerWarp; ++i)
+    if (i < ntok) s_part[(warp + 8 * i) * kClExp + lane] = acc[i];
+  cluster_sync();
+  // CTA r adds the partials of tokens t = r (mod 8), in rank order
+  {
+    const int t = (int)rank + 8 * warp;
+    if (t < T) {
+      float v = 0.f;
+#pragma unroll
+      for (uint32_t q = 0; q < (uint32_t)kCl; ++q)
+        v += ld_peer_f32(peer_addr(&s_part[t * kClExp + lane], q));
+      if (e0 + lane < E) a.logits_part[(size_t)t * E + e0 + lane] = v;
+    }
+  }
+  __threadfence();
+  cluster_sync();  // all logits of this cluster written; peers done reading s_part
+
+  // ---- 2. the last cluster to finish routes the forward
+  if (rank == 0 && tid == 0) {
+    const uint32_t last = (atomicAdd(f.ticket, 1) == n_clusters - 1) ? 1u : 0u;
+    for (uint32_t q = 0; q < (uint32_t)kCl; ++q) st_peer_u32(peer_addr(&s_last, q), last);
+  }
+  cluster_sync();
+  if (!s_last) return;
+  __threadfence();
+
+  // ---- 3. scores: token t = 8 * rank + warp
+  {
+    const int t = 8 * (int)rank + warp;
+    if (t < T) {
+      float* row = reinterpret_cast<float*>(dsm) + warp * kMaxExperts;
+      for (int e = lane; e < E; e += 32) row[e] = __ldcg(a.logits_part + (size_t)t * E + e);
+      __syncwarp();
+      token_route_warp(row, 1, 0, a.bias, E, k, a.mode, a.probs + (size_t)t * E,
+                       a.probs_hat + (size_t)t * E, a.topk_idx + (size_t)t * k,
+                       a.topk_gate + (size_t)t * k);
+    }
+  }
+  __threadfence();
+  cluster_sync();
+
+  // ---- 4. Algorithm 1: block b by CTA b mod 8
+  if (a.mode == DMOE_ROUTE_BLOCK) {
+    for (int b = (int)rank; b < a.n_blocks; b += kCl) {
+      float* P = reinterpret_cast<float*>(dsm);     // [B][E] scores
+      float* H = P + B * E;                         // [B][E] TopKMask
+      for (int i = tid; i < B * E; i += 256) {
+        P[i] = __ldcg(a.probs + (size_t)b * B * E + i);
+        H[i] = __ldcg(a.probs_hat + (size_t)b * B * E + i);
+      }
+      __syncthreads();
+      block_route_cta(0, P, H, E, k, B, a.top_p, a.topk_idx + (size_t)b * B * k,
+                      a.topk_gate + (size_t)b * B * k,
+                      a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
+                      a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
+    }
+  } else if (rank == 0) {
+    if (a.coreset != nullptr)
+      for (int i = tid; i < a.n_blocks * E; i += 256) a.coreset[i] = -1;
+    if (a.coreset_size != nullptr)
+      for (int i = tid; i < a.n_blocks; i += 256) a.coreset_size[i] = 0;
+  }
+  __threadfence();
+  cluster_sync();
+
+  // ---- 5. dispatch
+  if (rank == 0) {
+    if (f.dsp.n_unique != nullptr) {
+      int32_t* idx = reinterpret_cast<int32_t*>(dsm);
+      for (int i = tid; i < T * k; i += 256) idx[i] = __ldcg(a.topk_idx + i);
+      __syncthreads();
+      dispatch_cta(idx, T, E, k, f.dsp.n_unique, f.dsp.unique_ids, f.dsp.offsets, f.dsp.rows,
+                   f.dsp.pos, f.dsp.err, s_bits, s_base);
+    }
+    if (tid == 0) *f.ticket = 0;  // ready for the next call
+  }
+}
+
+typedef CUresult (*EncodeTiledFnC)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFnC encoder() {
+  static EncodeTiledFnC fn = nullptr;
+  if (fn == nullptr) {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFnC>(ptr);
+  }
+  return fn;
+}
+
+size_t route_cluster_smem() {
+  const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2;
+  const size_t stage4 = (size_t)2 * kClMaxTok * kMaxExperts * 4;
+  return (stage1 > stage4 ? stage1 : stage4) + 128;
+}
+
+}  // namespace
+
+bool route_cluster_ok(int T, int d, int E) {
+  return T <= kClMaxTok && d % (kCl * 8) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
+}
+
+cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
+                                 cudaStream_t s) {
+  EncodeTiledFnC enc = encoder();
+  if (enc == nullptr) return cudaErrorInvalidValue;
+  ClusterArgs f{};
+  const int DC = a.d / kCl;
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)a.E, (cuuint64_t)a.d};
+    const cuuint64_t strides[1] = {(cuuint64_t)a.E * 4};
+    const cuuint32_t box[2] = {(cuuint32_t)kClExp, (cuuint32_t)DC};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(&f.wmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(a.w_r), dims, strides,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  {
+    const cuuint64_t dims[2] = {(cuuint64_t)a.d, (cuuint64_t)a.T};
+    const cuuint64_t strides[1] = {(cuuint64_t)a.d * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)DC, (cuuint32_t)a.T};
+    const cuuint32_t estr[2] = {1, 1};
+    if (enc(&f.xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(a.x), dims,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return cudaErrorInvalidValue;
+  }
+  f.r = a;
+  if (dsp != nullptr) f.dsp = *dsp;
+  f.ticket = tickets;
+  const size_t smem = route_cluster_smem();
+  static int mask = 0;
+  int dev = 0;
+  cudaGetDevice(&dev);
+  if (dev >= 31 || !(mask & (1 << dev))) {
+    cudaError_t e = cudaFuncSetAttribute(route_cluster_kernel,
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev < 31) mask |= 1 << dev;
+  }
+  dim3 grid(kCl, (a.E + kClExp - 1) / kClExp);
+  return launch_cluster(route_cluster_kernel, grid, dim3(256), smem, s, kCl, f);
+}
+
+}  // namespace dmoe

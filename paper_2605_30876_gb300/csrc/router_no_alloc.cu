@@ -63,8 +63,9 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
       (coreset_size != nullptr && !ok16(coreset_size)))
     return DMOE_ERR_INVALID_ARG;
 
-  // The router uses the leading regions of the workspace plan: the fault record, the
-  // partial logits, the scores and the masked scores; the next region starts at tk_idx.
+  // The router uses the leading regions of the workspace plan: the fault record, the stage
+  // counters, the partial logits, the scores and the masked scores; the next region starts
+  // at tk_idx.
   const Workspace plan = plan_workspace(*desc);
   const size_t need = plan.tk_idx;
   if (need > kRouterStaticScratchBytes) {
@@ -96,6 +97,7 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
   a.bias = bias;
   a.logits_part = reinterpret_cast<float*>(base + plan.logits_part);
   a.probs = probs != nullptr ? probs : reinterpret_cast<float*>(base + plan.probs);
+  a.probs_requested = probs != nullptr;
   a.probs_hat = reinterpret_cast<float*>(base + plan.probs_hat);
   a.topk_idx = topk_idx;
   a.topk_gate = topk_gate;
@@ -111,7 +113,7 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
   a.splits = plan.router_splits;
   a.top_p = desc->top_p;
   a.err = reinterpret_cast<DevErrRecord*>(base + plan.err);
-  e = launch_router(a, nullptr, reinterpret_cast<int32_t*>(base + plan.err + kTicketOffset), s);
+  e = launch_router(a, nullptr, reinterpret_cast<int32_t*>(base + plan.tickets), s);
   if (e != cudaSuccess) {
     set_last_error(e);
     return DMOE_ERR_CUDA;
