@@ -26,6 +26,25 @@ constexpr int kCl = 8;                 // CTAs per cluster (split of d)
 constexpr int kClExp = 32;             // experts per cluster
 constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
 constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
+static_assert(kClMaxTok * kClMaxDChunk * 2 >= 4 * kClMaxTok * kClExp * 4,
+              "the quarter sums must fit where the bf16 x slice was");
+
+// Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 8 + stage]: 0 entry,
+// 1 TMA landed, 2 partial logits done, 3 logits reduced, 4 ticket, 5 scores, 6 Algorithm 1,
+// 7 dispatch.
+#ifdef DMOE_TRACE
+__device__ uint64_t g_ctrace[64 * 8 * 8];
+#define CT_AT(st)                                                                       \
+  do {                                                                                  \
+    if (threadIdx.x == 0) {                                                             \
+      uint64_t t_;                                                                      \
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                            \
+      g_ctrace[((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 8 + (st)] = t_;          \
+    }                                                                                   \
+  } while (0)
+#else
+#define CT_AT(st) ((void)0)
+#endif
 
 struct ClusterArgs {
   CUtensorMap wmap;   // W_r [d, E] fp32, box 32 experts x d/8 rows
@@ -62,6 +81,43 @@ __device__ __forceinline__ void st_peer_u32(uint32_t addr, uint32_t v) {
   asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
 
+// Partial logits of the CTA's d slice: thread (q, eg, tg) accumulates experts 4eg..4eg+3 of
+// tokens tg*TPT .. tg*TPT+TPT-1 over d in the q-th quarter of the slice and stores them to
+// red[q][t][e] (fp32, [4][kClMaxTok][32]); Ws [DC][32], Xf [T][xs] fp32 in shared memory.
+template <int TPT>
+__device__ __forceinline__ void logits_partial(const float* Ws, const float* Xf, int xs, int DC,
+                                               int T, float* red, int tid) {
+  const int q = tid >> 6, r = tid & 63, eg = r & 7, tg = r >> 3;
+  const int dq = DC / 4, d0 = q * dq;
+  float acc[TPT][4];
+#pragma unroll
+  for (int i = 0; i < TPT; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  int trow[TPT];
+#pragma unroll
+  for (int i = 0; i < TPT; ++i) trow[i] = min(tg * TPT + i, T - 1) * xs;  // clamp: rows >= T unused
+#pragma unroll 4
+  for (int dd = d0; dd < d0 + dq; ++dd) {
+    const float4 w = *reinterpret_cast<const float4*>(Ws + dd * kClExp + eg * 4);
+#pragma unroll
+    for (int i = 0; i < TPT; ++i) {
+      const float xv = Xf[trow[i] + dd];
+      acc[i][0] = fmaf(xv, w.x, acc[i][0]);
+      acc[i][1] = fmaf(xv, w.y, acc[i][1]);
+      acc[i][2] = fmaf(xv, w.z, acc[i][2]);
+      acc[i][3] = fmaf(xv, w.w, acc[i][3]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < TPT; ++i) {
+    const int t = tg * TPT + i;
+    if (t < T)
+      *reinterpret_cast<float4*>(red + ((size_t)q * kClMaxTok + t) * kClExp + eg * 4) =
+          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+  }
+}
+
 __global__ void __launch_bounds__(256, 1)
 route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   extern __shared__ __align__(128) uint8_t dsm_raw[];
@@ -80,6 +136,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   const int n_clusters = gridDim.y;
   pdl_launch_dependents();
   pdl_wait();
+  CT_AT(0);
 
   // ---- 1. partial logits over this CTA's slice of d
   float* Ws = reinterpret_cast<float*>(dsm);                                   // [DC][32]
@@ -128,28 +185,26 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       }
     }
   }
-  // lane = expert e0 + lane, warp w = tokens w, w + 8, ...
-  constexpr int kTokPerWarp = kClMaxTok / 8;
-  float acc[kTokPerWarp];
-#pragma unroll
-  for (int i = 0; i < kTokPerWarp; ++i) acc[i] = 0.f;
-  const int ntok = (T - warp + 7) / 8;   // tokens of this warp
-  for (int dd = 0; dd < DC; dd += 2) {
-    const float w0 = Ws[dd * kClExp + lane];
-    const float w1 = Ws[(dd + 1) * kClExp + lane];
-#pragma unroll
-    for (int i = 0; i < kTokPerWarp; ++i) {
-      if (i < ntok) {
-        const __nv_bfloat162 xv =
-            *reinterpret_cast<const __nv_bfloat162*>(Xs + (size_t)(warp + 8 * i) * DC + dd);
-        acc[i] = fmaf(__low2float(xv), w0, acc[i]);
-        acc[i] = fmaf(__high2float(xv), w1, acc[i]);
-      }
-    }
+  CT_AT(1);
+  // x slice to fp32, rows padded by one float against bank conflicts
+  float* Xf = reinterpret_cast<float*>(dsm + kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2);
+  const int xs = DC + 1;
+  for (int i = tid; i < T * DC; i += 256) Xf[(i / DC) * xs + (i % DC)] = __bfloat162float(Xs[i]);
+  __syncthreads();
+  // register-blocked FFMA: thread = (d quarter q, expert quad eg, token group tg);
+  // 4 experts x TPT tokens per thread, d ascending within the quarter
+  // the four quarter sums go where the bf16 x slice was (dead after the conversion)
+  float* red4 = reinterpret_cast<float*>(Xs);
+  if (T <= 32) logits_partial<4>(Ws, Xf, xs, DC, T, red4, tid);
+  else logits_partial<8>(Ws, Xf, xs, DC, T, red4, tid);
+  __syncthreads();
+  // add the four d quarters in order
+  for (int i = tid; i < T * kClExp; i += 256) {
+    const float* red = red4 + i;
+    s_part[i] = ((red[0] + red[kClMaxTok * kClExp]) + red[2 * kClMaxTok * kClExp]) +
+                red[3 * kClMaxTok * kClExp];
   }
-#pragma unroll
-  for (int i = 0; i < kTokPerWarp; ++i)
-    if (i < ntok) s_part[(warp + 8 * i) * kClExp + lane] = acc[i];
+  CT_AT(2);
   cluster_sync();
   // CTA r adds the partials of tokens t = r (mod 8), in rank order
   {
@@ -164,6 +219,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   }
   __threadfence();
   cluster_sync();  // all logits of this cluster written; peers done reading s_part
+  CT_AT(3);
 
   // ---- 2. the last cluster to finish routes the forward
   if (rank == 0 && tid == 0) {
@@ -173,6 +229,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   cluster_sync();
   if (!s_last) return;
   __threadfence();
+  CT_AT(4);
 
   // ---- 3. scores: token t = 8 * rank + warp
   {
@@ -188,6 +245,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   }
   __threadfence();
   cluster_sync();
+  CT_AT(5);
 
   // ---- 4. Algorithm 1: block b by CTA b mod 8
   if (a.mode == DMOE_ROUTE_BLOCK) {
@@ -212,6 +270,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   }
   __threadfence();
   cluster_sync();
+  CT_AT(6);
 
   // ---- 5. dispatch
   if (rank == 0) {
@@ -223,6 +282,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
                    f.dsp.pos, f.dsp.err, s_bits, s_base);
     }
     if (tid == 0) *f.ticket = 0;  // ready for the next call
+    CT_AT(7);
   }
 }
 
@@ -245,12 +305,19 @@ EncodeTiledFnC encoder() {
 }
 
 size_t route_cluster_smem() {
-  const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2;
+  const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2 +
+                        (size_t)kClMaxTok * (kClMaxDChunk + 1) * 4;
   const size_t stage4 = (size_t)2 * kClMaxTok * kMaxExperts * 4;
   return (stage1 > stage4 ? stage1 : stage4) + 128;
 }
 
 }  // namespace
+
+#ifdef DMOE_TRACE
+extern "C" int dmoe_debug_ctrace(void* host) {
+  return (int)cudaMemcpyFromSymbol(host, g_ctrace, sizeof(g_ctrace));
+}
+#endif
 
 bool route_cluster_ok(int T, int d, int E) {
   return T <= kClMaxTok && d % (kCl * 8) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
