@@ -31,6 +31,7 @@
 
 #include "dmoe_internal.cuh"
 #include "sm100_ptx.cuh"
+#include "trace_log.cuh"
 
 namespace dmoe {
 namespace {
@@ -159,6 +160,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) DMOE_TRACE_AT(0);
+  KLOG(DMOE_KERNEL_EXPERTS, 0);
 
   if (tid == 0) {
     for (int s = 0; s < stages; ++s) {
@@ -559,6 +561,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   __syncthreads();
   ptx::tc_fence_after();
   if (tid == 0) DMOE_TRACE_AT(62);
+  KLOG(DMOE_KERNEL_EXPERTS, 1);
   if (warp == 1) {
     __syncwarp();
     ptx::tmem_dealloc(tmem_base, p.tmem_cols);
@@ -572,6 +575,7 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
               int pairs, int k, int d) {
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(DMOE_KERNEL_GATHER, 0);
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_ready; i += blockDim.x) h_ready[i] = 0;
   const int vec = d / 8;  // uint4 per row
@@ -581,6 +585,7 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
     uint4* dst = reinterpret_cast<uint4*>(xperm + (size_t)r * d);
     for (int i = threadIdx.x; i < vec; i += blockDim.x) dst[i] = src[i];
   }
+  KLOG(DMOE_KERNEL_GATHER, 1);
 }
 
 // y[t, :] = bf16( sum_j g[t,j] * yslot[pos[t*k + j], :] (slot order) + yshared[t, :] )
@@ -590,6 +595,7 @@ combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshare
                __nv_bfloat16* __restrict__ y, int k, int d, int has_shared) {
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(DMOE_KERNEL_COMBINE, 0);
   const int t = blockIdx.y;
   const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
   if (c >= d) return;
@@ -613,6 +619,7 @@ combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshare
   out.x = *reinterpret_cast<uint32_t*>(&lo);
   out.y = *reinterpret_cast<uint32_t*>(&hi);
   *reinterpret_cast<uint2*>(y + (size_t)t * d + c) = out;
+  KLOG(DMOE_KERNEL_COMBINE, 1);
 }
 
 // ------------------------------------------------------------------ host side
@@ -678,6 +685,7 @@ extern "C" int dmoe_debug_trace_clear() {
   static uint64_t zeros[kMaxPersistentCtas * 64] = {};
   return (int)cudaMemcpyToSymbol(g_trace, zeros, sizeof(zeros));
 }
+DMOE_KLOG_EXPORT(dmoe_debug_klog_experts)
 #endif
 
 int experts_ready_counters(int T, int E) {

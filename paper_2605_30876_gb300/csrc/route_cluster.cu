@@ -8,16 +8,20 @@
 //      distributed shared memory and writes those logits.
 //   2. one atomic ticket: the last cluster to finish continues; the others exit.
 //   3. scores: one warp per token (8 CTAs x 8 warps = 64 tokens): softmax, top-k (token
-//      mode: the routing; block mode: TopKMask).
-//   4. Algorithm 1 for block b by CTA b mod 8 (blocks in parallel).
-//   5. dispatch by CTA 0 (fused layer call).
-// Stages 3-5 are separated by cluster barriers (release/acquire at cluster scope); data
-// written to global memory by other CTAs is read past the L1 (ld.global.cg).
+//      mode: the routing; block mode: TopKMask, whose k nonzeros are stored straight into
+//      the shared memory of the CTA that routes the token's block).
+//   4. Algorithm 1 for block b by CTA b mod 8 (blocks in parallel); the scores MaskOutside
+//      needs are read from the scoring CTAs' shared memory.
+//   5. dispatch by CTA 0 (fused layer call) from the top-k ids gathered in its shared memory.
+// Stages 3-5 are separated by cluster barriers (release/acquire at cluster scope) and pass
+// their data through distributed shared memory; only the logits cross clusters, through
+// global memory, read past the L1 (ld.global.cg) after the ticket's acquire.
 #include <math.h>
 
 #include "dispatch_impl.cuh"
 #include "dmoe_internal.cuh"
 #include "routing_device.cuh"
+#include "trace_log.cuh"
 
 namespace dmoe {
 namespace {
@@ -29,17 +33,20 @@ constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
 static_assert(kClMaxTok * kClMaxDChunk * 2 >= 4 * kClMaxTok * kClExp * 4,
               "the quarter sums must fit where the bf16 x slice was");
 
-// Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 8 + stage]: 0 entry,
-// 1 TMA landed, 2 partial logits done, 3 logits reduced, 4 ticket, 5 scores, 6 Algorithm 1,
-// 7 dispatch.
+// Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 32 + stage] (globaltimer;
+// + 16: clock64): 0 entry,
+// 1 TMA landed, 8 x converted, 2 partial logits done, 3 logits reduced, 4 ticket, 5 scores,
+// 6 Algorithm 1, 7 dispatch.
 #ifdef DMOE_TRACE
-__device__ uint64_t g_ctrace[64 * 8 * 8];
+__device__ uint64_t g_ctrace[64 * 8 * 32];
 #define CT_AT(st)                                                                       \
   do {                                                                                  \
     if (threadIdx.x == 0) {                                                             \
       uint64_t t_;                                                                      \
       asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                            \
-      g_ctrace[((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 8 + (st)] = t_;          \
+      const int c_ = ((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 32 + (st);         \
+      g_ctrace[c_] = t_;                                                                \
+      g_ctrace[c_ + 16] = clock64();                                                    \
     }                                                                                   \
   } while (0)
 #else
@@ -80,6 +87,21 @@ __device__ __forceinline__ float ld_peer_f32(uint32_t addr) {
 __device__ __forceinline__ void st_peer_u32(uint32_t addr, uint32_t v) {
   asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
+__device__ __forceinline__ void st_peer_f32(uint32_t addr, float v) {
+  asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+
+// Shared-memory layout after the logits (the W_r / x slices are dead by then), in bytes
+// from the dynamic base: scores of this CTA's tokens, the top-k ids for the dispatch (rank
+// 0), the MaskOutside scratch, and the dense TopKMask rows of the blocks this CTA routes.
+constexpr int kOffP = 0;                                      // f32 [8][kMaxExperts]
+constexpr int kOffIdx = kOffP + 8 * kMaxExperts * 4;          // i32 [kClMaxTok * kMaxTopK]
+constexpr int kOffSv = kOffIdx + kClMaxTok * kMaxTopK * 4;    // f32 [kClMaxTok][32]
+constexpr int kOffSelE = kOffSv + kClMaxTok * 32 * 4;         // i32 [kClMaxTok][kMaxTopK]
+constexpr int kOffSelV = kOffSelE + kClMaxTok * kMaxTopK * 4; // f32 [kClMaxTok][kMaxTopK]
+constexpr int kOffHat = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;  // f32 [kClMaxTok][kMaxExperts]
+static_assert(kOffSelV + kClMaxTok * kMaxTopK * 4 <= kClMaxDChunk * kClExp * 4,
+              "the routing scratch must fit where the W_r slice was");
 
 // Partial logits of the CTA's d slice: thread (q, eg, tg) accumulates experts 4eg..4eg+3 of
 // tokens tg*TPT .. tg*TPT+TPT-1 over d in the q-th quarter of the slice and stores them to
@@ -127,6 +149,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   __shared__ float s_part[kClMaxTok * kClExp];                     // partial logits [T][32]
   __shared__ uint32_t s_bits[(kClMaxTok / 32) * kMaxExperts];
   __shared__ uint16_t s_base[(kClMaxTok / 32) * kMaxExperts];
+  __shared__ float s_bias[kMaxExperts];
   const RouterArgs& a = f.r;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int T = a.T, E = a.E, k = a.k, B = a.B;
@@ -136,6 +159,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   const int n_clusters = gridDim.y;
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(DMOE_KERNEL_ROUTER, 0);
   CT_AT(0);
 
   // ---- 1. partial logits over this CTA's slice of d
@@ -164,6 +188,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         : "memory");
     issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
   }
+  for (int e = tid; e < E; e += 256) s_bias[e] = a.bias != nullptr ? a.bias[e] : 0.f;
   __syncthreads();
   {
     uint64_t t0;
@@ -189,8 +214,22 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   // x slice to fp32, rows padded by one float against bank conflicts
   float* Xf = reinterpret_cast<float*>(dsm + kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2);
   const int xs = DC + 1;
-  for (int i = tid; i < T * DC; i += 256) Xf[(i / DC) * xs + (i % DC)] = __bfloat162float(Xs[i]);
+  {
+    const int DC8 = DC / 8;  // d % 64 == 0: whole groups of eight per row
+    for (int i = tid; i < T * DC8; i += 256) {
+      const int t = i / DC8, c = (i - t * DC8) * 8;
+      const uint4 raw = *reinterpret_cast<const uint4*>(Xs + t * DC + c);
+      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
+      float* dst = Xf + t * xs + c;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        dst[2 * q] = __low2float(p2[q]);
+        dst[2 * q + 1] = __high2float(p2[q]);
+      }
+    }
+  }
   __syncthreads();
+  CT_AT(8);
   // register-blocked FFMA: thread = (d quarter q, expert quad eg, token group tg);
   // 4 experts x TPT tokens per thread, d ascending within the quarter
   // the four quarter sums go where the bf16 x slice was (dead after the conversion)
@@ -204,63 +243,127 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     s_part[i] = ((red[0] + red[kClMaxTok * kClExp]) + red[2 * kClMaxTok * kClExp]) +
                 red[3 * kClMaxTok * kClExp];
   }
+  {  // TopKMask rows start as zeros (scoring warps anywhere in the cluster add the winners)
+    float4* hz = reinterpret_cast<float4*>(dsm + kOffHat);
+    for (int i = tid; i < T * (kMaxExperts / 4); i += 256) hz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+  }
   CT_AT(2);
   cluster_sync();
   // CTA r adds the partials of tokens t = r (mod 8), in rank order
   {
     const int t = (int)rank + 8 * warp;
     if (t < T) {
-      float v = 0.f;
+      float p[kCl];
 #pragma unroll
       for (uint32_t q = 0; q < (uint32_t)kCl; ++q)
-        v += ld_peer_f32(peer_addr(&s_part[t * kClExp + lane], q));
+        p[q] = ld_peer_f32(peer_addr(&s_part[t * kClExp + lane], q));
+      float v = 0.f;
+#pragma unroll
+      for (int q = 0; q < kCl; ++q) v += p[q];
       if (e0 + lane < E) a.logits_part[(size_t)t * E + e0 + lane] = v;
     }
   }
-  __threadfence();
-  cluster_sync();  // all logits of this cluster written; peers done reading s_part
+  // every CTA of the cluster has written its logits and finished reading its peers' s_part
+  // (cluster scope); rank 0 then publishes the cluster at GPU scope
+  cluster_sync();
   CT_AT(3);
 
   // ---- 2. the last cluster to finish routes the forward
   if (rank == 0 && tid == 0) {
+    __threadfence();
     const uint32_t last = (atomicAdd(f.ticket, 1) == n_clusters - 1) ? 1u : 0u;
+    if (last) __threadfence();  // acquire the other clusters' logits
     for (uint32_t q = 0; q < (uint32_t)kCl; ++q) st_peer_u32(peer_addr(&s_last, q), last);
   }
   cluster_sync();
-  if (!s_last) return;
-  __threadfence();
+  if (!s_last) {
+    KLOG(DMOE_KERNEL_ROUTER, 1);
+    return;
+  }
   CT_AT(4);
 
-  // ---- 3. scores: token t = 8 * rank + warp
+  // ---- 3. scores: token t = 8 * rank + warp; its scores stay in this CTA's shared memory
+  // (sP [8 warps][E]) and its TopKMask winners go to the CTA that routes its block
+  float* sP = reinterpret_cast<float*>(dsm + kOffP);
+  int32_t* sIdx = reinterpret_cast<int32_t*>(dsm + kOffIdx);  // [T * k], read in rank 0
+  float* sHat = reinterpret_cast<float*>(dsm + kOffHat);
+  constexpr int J = kMaxExperts / 32;
   {
     const int t = 8 * (int)rank + warp;
     if (t < T) {
-      float* row = reinterpret_cast<float*>(dsm) + warp * kMaxExperts;
-      for (int e = lane; e < E; e += 32) row[e] = __ldcg(a.logits_part + (size_t)t * E + e);
-      __syncwarp();
-      token_route_warp(row, 1, 0, a.bias, E, k, a.mode, a.probs + (size_t)t * E,
-                       a.probs_hat + (size_t)t * E, a.topk_idx + (size_t)t * k,
-                       a.topk_gate + (size_t)t * k);
+      float v[J];
+      int id[J];
+      uint32_t valid = 0;
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        const int e = lane + 32 * j;
+        id[j] = e;
+        v[j] = 0.f;
+        if (e < E) {
+          valid |= 1u << j;
+          v[j] = __ldcg(a.logits_part + (size_t)t * E + e);
+        }
+      }
+#pragma unroll
+      for (int j = 0; j < J; ++j) v[j] = ((valid >> j) & 1u) ? v[j] + s_bias[lane + 32 * j] : -INFINITY;
+      warp_softmax8(v, valid);
+      float* prow = sP + warp * kMaxExperts;
+#pragma unroll
+      for (int j = 0; j < J; ++j)
+        if ((valid >> j) & 1u) {
+          prow[lane + 32 * j] = v[j];
+          if (a.probs_requested) a.probs[(size_t)t * E + lane + 32 * j] = v[j];
+        }
+      int my_idx;
+      float my_val;
+      warp_topk(v, id, valid, k, my_idx, my_val);
+      if (a.mode == DMOE_ROUTE_BLOCK) {
+        // TopKMask: the k winners into the zeroed row of token t in the CTA that routes
+        // its block (block b: CTA b mod 8)
+        if (lane < k)
+          st_peer_f32(peer_addr(sHat + t * kMaxExperts + my_idx, (uint32_t)((t / B) % kCl)),
+                      my_val);
+      } else {
+        float tot = 0.f;
+        for (int r = 0; r < k; ++r) tot += __shfl_sync(0xffffffffu, my_val, r);
+        if (lane < k) {
+          a.topk_idx[(size_t)t * k + lane] = my_idx;
+          a.topk_gate[(size_t)t * k + lane] = my_val / tot;
+          st_peer_u32(peer_addr(&sIdx[t * k + lane], 0), (uint32_t)my_idx);
+        }
+      }
     }
   }
-  __threadfence();
   cluster_sync();
   CT_AT(5);
 
-  // ---- 4. Algorithm 1: block b by CTA b mod 8
+  // ---- 4. Algorithm 1: block b by CTA b mod 8, the block's rows read from the shared
+  // memory of the CTAs that scored them (token t: CTA t / 8, row t mod 8)
   if (a.mode == DMOE_ROUTE_BLOCK) {
+    __shared__ int order[kMaxExperts];
     for (int b = (int)rank; b < a.n_blocks; b += kCl) {
-      float* P = reinterpret_cast<float*>(dsm);     // [B][E] scores
-      float* H = P + B * E;                         // [B][E] TopKMask
-      for (int i = tid; i < B * E; i += 256) {
-        P[i] = __ldcg(a.probs + (size_t)b * B * E + i);
-        H[i] = __ldcg(a.probs_hat + (size_t)b * B * E + i);
-      }
+      const int t0 = b * B;
+      const int size = block_coreset_steps(
+          E, k, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
+          a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
+          a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
+      auto prob = [&](int i, int e) {
+        const int t = t0 + i;
+        return ld_peer_f32(peer_addr(sP + (t & 7) * kMaxExperts + e, (uint32_t)(t >> 3)));
+      };
+      auto out = [&](int i, int r, int e, float g) {
+        const int t = t0 + i;
+        a.topk_idx[(size_t)t * k + r] = e;
+        a.topk_gate[(size_t)t * k + r] = g;
+        st_peer_u32(peer_addr(&sIdx[t * k + r], 0), (uint32_t)e);
+      };
+      if (size <= 32)
+        mask_topk_small(k, B, size, order, prob, out, reinterpret_cast<float*>(dsm + kOffSv),
+                        reinterpret_cast<int*>(dsm + kOffSelE),
+                        reinterpret_cast<float*>(dsm + kOffSelV));
+      else
+        mask_topk_warps(k, B, size, order, prob, out);
       __syncthreads();
-      block_route_cta(0, P, H, E, k, B, a.top_p, a.topk_idx + (size_t)b * B * k,
-                      a.topk_gate + (size_t)b * B * k,
-                      a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
-                      a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
     }
   } else if (rank == 0) {
     if (a.coreset != nullptr)
@@ -268,22 +371,18 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     if (a.coreset_size != nullptr)
       for (int i = tid; i < a.n_blocks; i += 256) a.coreset_size[i] = 0;
   }
-  __threadfence();
   cluster_sync();
   CT_AT(6);
 
   // ---- 5. dispatch
   if (rank == 0) {
-    if (f.dsp.n_unique != nullptr) {
-      int32_t* idx = reinterpret_cast<int32_t*>(dsm);
-      for (int i = tid; i < T * k; i += 256) idx[i] = __ldcg(a.topk_idx + i);
-      __syncthreads();
-      dispatch_cta(idx, T, E, k, f.dsp.n_unique, f.dsp.unique_ids, f.dsp.offsets, f.dsp.rows,
+    if (f.dsp.n_unique != nullptr)
+      dispatch_cta(sIdx, T, E, k, f.dsp.n_unique, f.dsp.unique_ids, f.dsp.offsets, f.dsp.rows,
                    f.dsp.pos, f.dsp.err, s_bits, s_base);
-    }
     if (tid == 0) *f.ticket = 0;  // ready for the next call
     CT_AT(7);
   }
+  KLOG(DMOE_KERNEL_ROUTER, 1);
 }
 
 typedef CUresult (*EncodeTiledFnC)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
@@ -307,7 +406,7 @@ EncodeTiledFnC encoder() {
 size_t route_cluster_smem() {
   const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2 +
                         (size_t)kClMaxTok * (kClMaxDChunk + 1) * 4;
-  const size_t stage4 = (size_t)2 * kClMaxTok * kMaxExperts * 4;
+  const size_t stage4 = (size_t)2 * 8 * kMaxExperts * 4 + (size_t)kClMaxTok * kMaxTopK * 4;
   return (stage1 > stage4 ? stage1 : stage4) + 128;
 }
 
@@ -316,6 +415,11 @@ size_t route_cluster_smem() {
 #ifdef DMOE_TRACE
 extern "C" int dmoe_debug_ctrace(void* host) {
   return (int)cudaMemcpyFromSymbol(host, g_ctrace, sizeof(g_ctrace));
+}
+DMOE_KLOG_EXPORT(dmoe_debug_klog_router)
+extern "C" int dmoe_debug_ctrace_clear() {
+  static uint64_t zeros[64 * 8 * 32];
+  return (int)cudaMemcpyToSymbol(g_ctrace, zeros, sizeof(g_ctrace));
 }
 #endif
 

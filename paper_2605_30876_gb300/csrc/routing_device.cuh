@@ -89,6 +89,26 @@ __device__ __forceinline__ void warp_topk(const float (&v)[8], const int (&id)[8
   }
 }
 
+// Softmax over one token's experts held by a warp (lane holds experts lane + 32j; invalid
+// slots are -inf on entry and 0 on exit): exp(v - max) / sum, fp32, the sum in a fixed order.
+__device__ __forceinline__ void warp_softmax8(float (&v)[kMaxExperts / 32], uint32_t valid) {
+  constexpr int J = kMaxExperts / 32;
+  uint32_t mk = 0;
+#pragma unroll
+  for (int j = 0; j < J; ++j)
+    if ((valid >> j) & 1u) mk = max(mk, order_key(v[j]));
+  const float m = key_value(__reduce_max_sync(0xffffffffu, mk));
+  float sum = 0.f;
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    v[j] = ((valid >> j) & 1u) ? expf(v[j] - m) : 0.f;
+    sum += v[j];
+  }
+  sum = warp_sum(sum);
+#pragma unroll
+  for (int j = 0; j < J; ++j) v[j] = v[j] / sum;
+}
+
 // Router scores and top-k of one token by one warp (E <= 256; lane holds experts lane + 32j).
 // logit(e) = sum over `nsum` partial rows (stride `pstride`) in order, + bias[e].
 // Writes the scores to prow; block mode: TopKMask(s, k) to hrow; token mode: the k experts
@@ -105,32 +125,29 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
   for (int j = 0; j < J; ++j) {
     const int e = lane + 32 * j;
     id[j] = e;
-    float a = -INFINITY;
-    if (e < E) {
-      valid |= 1u << j;
-      a = 0.f;
-      for (int s = 0; s < nsum; ++s) a += lrow[(size_t)s * pstride + e];
-      if (bias != nullptr) a += bias[e];
-    }
-    v[j] = a;
+    v[j] = 0.f;
+    if (e < E) valid |= 1u << j;
   }
-  uint32_t mk = 0;
+  // partial rows outermost: the J loads of one row are independent and go out together
+  for (int s = 0; s < nsum; ++s) {
+    float l[J];
+#pragma unroll
+    for (int j = 0; j < J; ++j) l[j] = ((valid >> j) & 1u) ? lrow[(size_t)s * pstride + lane + 32 * j] : 0.f;
+#pragma unroll
+    for (int j = 0; j < J; ++j) v[j] += l[j];
+  }
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    if ((valid >> j) & 1u) {
+      if (bias != nullptr) v[j] += bias[lane + 32 * j];
+    } else {
+      v[j] = -INFINITY;
+    }
+  }
+  warp_softmax8(v, valid);
 #pragma unroll
   for (int j = 0; j < J; ++j)
-    if ((valid >> j) & 1u) mk = max(mk, order_key(v[j]));
-  const float m = key_value(__reduce_max_sync(0xffffffffu, mk));
-  float sum = 0.f;
-#pragma unroll
-  for (int j = 0; j < J; ++j) {
-    v[j] = ((valid >> j) & 1u) ? expf(v[j] - m) : 0.f;
-    sum += v[j];
-  }
-  sum = warp_sum(sum);
-#pragma unroll
-  for (int j = 0; j < J; ++j) {
-    v[j] = v[j] / sum;
     if ((valid >> j) & 1u) prow[lane + 32 * j] = v[j];
-  }
   int my_idx;
   float my_val;
   warp_topk(v, id, valid, k, my_idx, my_val);
@@ -152,25 +169,38 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 }
 
 // ---------------------------------------------------------------- Algorithm 1, one block
-// Algorithm 1 for block b by a CTA of 256 threads (thread = expert for the block-level
-// steps, one warp per token for MaskOutside + TopK).
-__device__ inline void block_route_cta(int b, const float* probs, const float* probs_hat, int E, int k,
-                                int B, float top_p, int32_t* __restrict__ topk_idx,
-                                float* __restrict__ topk_gate, int32_t* __restrict__ coreset,
-                                int32_t* __restrict__ coreset_size) {
+// Algorithm 1 for one block of B tokens by a CTA of 256 threads. The block's rows come
+// through accessors, so the same steps serve rows in global memory and rows spread over the
+// shared memory of a cluster:
+//   hat(i, e)   TopKMask(s_i, k)[e] of the block's i-th token
+//   prob(i, e)  s_i[e]
+//   out(i, r, e, g)  the r-th selection of token i: expert e with gate g
+
+// Aggregate, Normalize, Sort, Top-P and the k floor (thread = expert). Leaves the coreset in
+// order[0, size) (S~ descending, ties to the lower id) and returns size; writes the coreset
+// outputs when given. `order` is a shared array of kMaxExperts entries.
+template <class HatFn>
+__device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
+                                          int32_t* __restrict__ coreset,
+                                          int32_t* __restrict__ coreset_size) {
   __shared__ __align__(16) float st_s[kMaxExperts];
-  __shared__ int order[kMaxExperts];
   __shared__ int s_size;
   __shared__ float fscr[32];
   const int tid = threadIdx.x;
-  const int t0 = b * B;
   const bool live = tid < E;
 
-  // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k)
+  // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k); eight rows are
+  // fetched at a time so that their loads overlap
   float S = 0.f;
   if (live) {
-#pragma unroll 8
-    for (int i = 0; i < B; ++i) S += probs_hat[(size_t)(t0 + i) * E + tid];
+    for (int i0 = 0; i0 < B; i0 += 8) {
+      float h[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) h[u] = (i0 + u < B) ? hat(i0 + u, tid) : 0.f;
+#pragma unroll
+      for (int u = 0; u < 8; ++u)
+        if (i0 + u < B) S += h[u];
+    }
   }
   // Normalize: L1
   const float tot = block_sum(S, fscr);
@@ -212,14 +242,19 @@ __device__ inline void block_route_cta(int b, const float* probs, const float* p
   }
   __syncthreads();
   const int size = s_size;
-  if (coreset != nullptr && live) coreset[(size_t)b * E + tid] = (tid < size) ? order[tid] : -1;
-  if (coreset_size != nullptr && tid == 0) coreset_size[b] = size;
+  if (coreset != nullptr && live) coreset[tid] = (tid < size) ? order[tid] : -1;
+  if (coreset_size != nullptr && tid == 0) coreset_size[0] = size;
+  return size;
+}
 
-  // MaskOutside + TopK for every token of the block (one warp per token): lane l holds the
-  // coreset members at sorted positions l + 32j
-  const int warp = tid >> 5, lane = tid & 31;
-  for (int i = warp; i < B; i += 8) {
-    const int t = t0 + i;
+// MaskOutside + TopK for every token of the block, one warp per token: lane l holds the
+// coreset members at sorted positions l + 32j; the k best by descending score (ties: lower
+// id), gates renormalised over the k in that order.
+template <class ProbFn, class OutFn>
+__device__ inline void mask_topk_warps(int k, int B, int size, const int* order, ProbFn prob,
+                                       OutFn out) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int i = warp; i < B; i += (int)(blockDim.x >> 5)) {
     float cv[8];
     int ce[8];
     uint32_t valid = 0;
@@ -227,24 +262,96 @@ __device__ inline void block_route_cta(int b, const float* probs, const float* p
     for (int j = 0; j < 8; ++j) {
       const int c = lane + 32 * j;
       ce[j] = 0;
-      cv[j] = 0.f;
       if (c < size) {
         valid |= 1u << j;
         ce[j] = order[c];
-        cv[j] = probs[(size_t)t * E + ce[j]];
       }
     }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) cv[j] = ((valid >> j) & 1u) ? prob(i, ce[j]) : 0.f;
     int my_e;
     float my_v;
     warp_topk(cv, ce, valid, k, my_e, my_v);
     float g = 0.f;
     for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
-    if (lane < k) {
-      topk_idx[(size_t)t * k + lane] = my_e;
-      topk_gate[(size_t)t * k + lane] = my_v / g;
+    if (lane < k) out(i, lane, my_e, my_v / g);
+  }
+}
+
+// The same result for a coreset of at most 32 experts with every (token, member) pair in
+// parallel: a member's rank among its token's members is the number of members that beat it
+// (larger score, or equal score and lower id); ranks below k are the selection. `sv` is a
+// shared [B][32] buffer, `sel_e`/`sel_v` shared [B][kMaxTopK] buffers.
+template <class ProbFn, class OutFn>
+__device__ inline void mask_topk_small(int k, int B, int size, const int* order, ProbFn prob,
+                                       OutFn out, float* sv, int* sel_e, float* sel_v) {
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  const int n = B * size;
+  for (int p0 = tid; p0 < n; p0 += 8 * nthr) {  // eight gathers in flight per thread
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int pidx = p0 + u * nthr;
+      v[u] = pidx < n ? prob(pidx / size, order[pidx % size]) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int pidx = p0 + u * nthr;
+      if (pidx < n) sv[(pidx / size) * 32 + pidx % size] = v[u];
     }
   }
   __syncthreads();
+  for (int pidx = tid; pidx < n; pidx += nthr) {
+    const int i = pidx / size, c = pidx % size;
+    const float* row = sv + i * 32;
+    const float v = row[c];
+    const int e = order[c];
+    int rank = 0;
+    for (int c2 = 0; c2 < size; ++c2) {
+      const float w = row[c2];
+      rank += (w > v || (w == v && order[c2] < e)) ? 1 : 0;
+    }
+    if (rank < k) {
+      sel_e[i * kMaxTopK + rank] = e;
+      sel_v[i * kMaxTopK + rank] = v;
+    }
+  }
+  __syncthreads();
+  for (int pidx = tid; pidx < B * k; pidx += nthr) {
+    const int i = pidx / k, r = pidx % k;
+    float g = 0.f;
+    for (int r2 = 0; r2 < k; ++r2) g += sel_v[i * kMaxTopK + r2];
+    out(i, r, sel_e[i * kMaxTopK + r], sel_v[i * kMaxTopK + r] / g);
+  }
+}
+
+template <class HatFn, class ProbFn, class OutFn>
+__device__ inline void block_route_steps(int E, int k, int B, float top_p, HatFn hat, ProbFn prob,
+                                         OutFn out, int32_t* __restrict__ coreset,
+                                         int32_t* __restrict__ coreset_size) {
+  __shared__ int order[kMaxExperts];
+  const int size = block_coreset_steps(E, k, B, top_p, hat, order, coreset, coreset_size);
+  mask_topk_warps(k, B, size, order, prob, out);
+  __syncthreads();
+}
+
+// Algorithm 1 for block b with the block's rows in global memory ([T, E] row-major).
+__device__ inline void block_route_cta(int b, const float* probs, const float* probs_hat, int E,
+                                       int k, int B, float top_p, int32_t* __restrict__ topk_idx,
+                                       float* __restrict__ topk_gate,
+                                       int32_t* __restrict__ coreset,
+                                       int32_t* __restrict__ coreset_size) {
+  const size_t r0 = (size_t)b * B;
+  block_route_steps(
+      E, k, B, top_p,
+      [&](int i, int e) { return probs_hat[(r0 + i) * E + e]; },
+      [&](int i, int e) { return probs[(r0 + i) * E + e]; },
+      [&](int i, int r, int e, float g) {
+        topk_idx[(r0 + i) * k + r] = e;
+        topk_gate[(r0 + i) * k + r] = g;
+      },
+      coreset != nullptr ? coreset + (size_t)b * E : nullptr,
+      coreset_size != nullptr ? coreset_size + b : nullptr);
 }
 
 }  // namespace dmoe
