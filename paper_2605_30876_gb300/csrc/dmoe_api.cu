@@ -97,6 +97,8 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.h_ready = take(sizeof(int32_t) * experts_ready_counters((int)T, (int)E));
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
+  const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
+  w.hdense = take(dec ? 2 * (E + 1) * (size_t)((T + 15) / 16 * 16) * (I > Is ? I : Is) : 0);
   w.total = off;
   return w;
 }
@@ -225,6 +227,8 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
   a.hs = at<__nv_bfloat16>(ws, plan.hs);
   a.yslot = at<float>(ws, plan.yslot);
   a.h_ready = at<int32_t>(ws, plan.h_ready);
+  a.hdense = at<__nv_bfloat16>(ws, plan.hdense);
+  a.tickets = at<int32_t>(ws, plan.tickets);
   a.yshared = at<float>(ws, plan.yshared);
   a.err = at<DevErrRecord>(ws, plan.err);
   a.T = desc->n_blocks * desc->block_size;
@@ -234,6 +238,7 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
   a.I = desc->d_ff;
   a.Is = desc->d_ff_shared;
   a.n_max = plan.n_max;
+  if (experts_decode_ok(a.T, a.d, a.I, a.Is)) return cuda_status(launch_experts_decode(a, s));
   return cuda_status(launch_experts(a, s));
 }
 

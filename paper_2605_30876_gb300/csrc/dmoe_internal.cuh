@@ -73,6 +73,8 @@ struct Workspace {
   size_t h_ready;      // int32 [(E+1) * token tiles]: published gate/up tiles
   size_t yslot;        // fp32 [T*k, d]   expert outputs per (token, slot)
   size_t yshared;      // fp32 [T, d]
+  size_t hdense;       // bf16 [(E+1) * n_pad, max(I, I_s)]: H per group over all tokens
+                       // (decode-size forwards only)
   size_t total;
   int router_splits;
   int n_max;           // token tile (MMA N) of the expert GEMMs
@@ -178,6 +180,8 @@ struct ExpertArgs {
   __nv_bfloat16* xperm; __nv_bfloat16* h; __nv_bfloat16* hs;
   float* yslot; float* yshared;
   int32_t* h_ready;
+  __nv_bfloat16* hdense;  // decode-size path: H per group over all tokens
+  int32_t* tickets;       // kRouteTickets ints, zero between calls
   DevErrRecord* err;
   bool prefetch_shared;   // the shared expert's weights were not prefetched by the router
   // shape
@@ -185,6 +189,13 @@ struct ExpertArgs {
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E);
+// gate-weighted combine of the expert rows into y (the last launch of both expert paths)
+cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s);
+// Decode-sized forwards (T <= 64): one persistent launch over gate/up and down tiles of
+// every group, all tokens at once (no gather), then the combine.
+bool experts_decode_ok(int T, int d, int I, int Is);
+cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s);
+constexpr int kTicketDecodeExit = 1;   // tickets[1]: CTAs of the decode expert launch done
 
 // profiling events (dmoe_set_profile_events), per host thread
 void prof_begin(int kernel, cudaStream_t s);

@@ -1,0 +1,680 @@
+// Expert FFN of a decode-sized forward (at most 64 tokens) in one persistent launch on
+// tcgen05 tensor cores (§4.2 of arXiv 2605.30876: every unique expert of the forward runs
+// once on the tokens routed to it; plus the shared expert on all tokens).
+//
+// A group is the shared expert (group 0, when present) or the u-th unique expert of the
+// dispatch. With at most 64 tokens every group is computed over all T tokens at once: the
+// B operand of gate/up is x itself (no gather), the extra MMA columns cost nothing next to
+// the weight stream, and the down epilogue keeps only the columns of the tokens routed to
+// the group. The work is a list of units spread round-robin over one CTA per SM:
+//   gate/up unit (group, 64 rows of I): 64 rows of W_gate stacked over the same 64 rows of
+//     W_up, one M = 128 MMA chain over K = d (gate in TMEM lanes 0-63, up in 64-127); the
+//     epilogue writes h = silu(gate) * up as bf16 into the group's H (global, L2-resident)
+//     and publishes the tile on the group's counter;
+//   down unit (group, 128 rows of d): D = W_down tile x H^T over K = I; the producer loads
+//     the weight stages first and the H stages once every gate/up tile of the group is
+//     published; the epilogue stores the fp32 rows per (token, slot).
+// Down units continue the round-robin where the gate/up units stopped, so a CTA that
+// streams a gate/up tile (d x 128 weights) takes at most one down tile (128 x I) and the
+// rest go to CTAs without gate/up work: the weight bytes per SM stay near the mean, every
+// SM streams, and HBM rather than one SM's TMA rate sets the pace.
+//
+// Warp roles (192 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, warps 2-5
+// run the epilogues (TMEM lane quadrant = warp % 4). Every wait is bounded (1 s): a timeout
+// is recorded and the CTA unwinds. The last CTA to finish clears the group counters for
+// the next call.
+#include <math.h>
+
+#include <mutex>
+
+#include "dmoe_internal.cuh"
+#include "sm100_ptx.cuh"
+#include "trace_log.cuh"
+
+namespace dmoe {
+namespace {
+
+constexpr int kThr = 192;
+constexpr int kKB = 2;                          // K boxes per stage: K = 128 per stage
+constexpr int kStageK = kKB * kTileK;
+constexpr int kGateBox = 64 * 128;              // 64 weight rows x 128 B
+constexpr int kABox = kTileM * 128;             // 128 rows x 128 B (gate|up, or W_down)
+constexpr int kAStage = kKB * kABox;            // 32 KB
+constexpr int kMaxStagesD = 6;
+constexpr int kXStride = 17;                    // floats per row of the SwiGLU exchange
+constexpr int kXchgBytes = 2 * 64 * kXStride * 4;
+constexpr uint64_t kTimeoutNs = 1000000000ull;  // 1 s
+constexpr int kMaxTok = 64;                     // tokens of a decode-sized forward
+
+// Debug builds (-DDMOE_TRACE): per-CTA timeline of the first unit of each kind,
+// g_dtrace[cta * 32 + slot] (globaltimer ns): 0 entry, 1 unit list known, 2 gate/up first
+// stage landed, 3 gate/up MMAs committed, 4 gate/up tile published, 5 down weights issued,
+// 6 H ready seen, 7 down MMAs committed, 8 down rows stored, 9 exit, 10 gate/up unit id,
+// 11 down unit id.
+#ifdef DMOE_TRACE
+__device__ uint64_t g_dtrace[kMaxPersistentCtas * 32];
+#define ED_AT(slot) (g_dtrace[blockIdx.x * 32 + (slot)] = ptx::globaltimer_ns())
+#define ED_SET(slot, v) (g_dtrace[blockIdx.x * 32 + (slot)] = (uint64_t)(v))
+#else
+#define ED_AT(slot) ((void)0)
+#define ED_SET(slot, v) ((void)0)
+#endif
+
+struct DParams {
+  const int32_t* n_unique;
+  const int32_t* unique_ids;
+  const int32_t* offsets;
+  const int32_t* rows;
+  __nv_bfloat16* hdense;     // [(E+1) * n_pad, imax]: H of group g in rows g*n_pad ..
+  float* yslot;              // [T*k, d]
+  float* yshared;            // [T, d]
+  int32_t* h_ready;          // [E+1]: published gate/up tiles per group
+  int32_t* exit_ticket;      // zero between calls
+  DevErrRecord* err;
+  int T, d, E, k, I, Is;
+  int imax;                  // max(I, Is): row length of hdense
+  int n_pad;                 // token rows of every B box (multiple of 16)
+  int stages;
+  int has_shared;
+  int n_acc;                 // TMEM accumulators of n_pad columns
+  uint32_t tmem_cols;
+};
+
+struct DMaps {
+  CUtensorMap wg, wu, wd;    // routed: [E*I, d] (64-row boxes) x2, [E*d, I] (128-row boxes)
+  CUtensorMap sg, su, sd;    // shared: [Is, d] x2, [d, Is]
+  CUtensorMap x;             // x [T, d], n_pad-row boxes (rows >= T read as zeros)
+  CUtensorMap h;             // hdense, n_pad-row boxes
+};
+
+// One group of the forward.
+struct Grp {
+  bool shared;
+  int e;      // expert id (routed)
+  int row0;   // first dispatch row (routed)
+  int n;      // tokens routed to the group (T for the shared expert)
+  int Ig;     // intermediate size
+};
+
+__device__ __forceinline__ void named_bar_sync(int id, int n) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+__device__ __forceinline__ void red_release_add(int32_t* p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+__device__ __forceinline__ int ld_acquire(const int32_t* p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+__device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
+
+// AND of `v` over the 128 epilogue threads (named barrier 1), so that warp-collective TMEM
+// loads are taken by all of them or by none.
+__device__ __forceinline__ bool epi_all(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, 128, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v)
+      : "memory");
+  return r != 0;
+}
+
+__global__ void __launch_bounds__(kThr, 1)
+moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DParams p) {
+  extern __shared__ __align__(1024) uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
+  const int S = p.stages;
+  const int bbox = p.n_pad * 128;                 // one K box of token rows
+  const int bstage = kKB * bbox;
+  const int SP = p.n_pad + 1;                     // floats per row of the down staging tile
+  uint8_t* ring_a = smem;
+  uint8_t* ring_b = ring_a + S * kAStage;
+  float* stage_t = reinterpret_cast<float*>(ring_b + S * bstage);   // [128][SP]
+  float* xchg = stage_t + kTileM * SP;
+  int* tok = reinterpret_cast<int*>(xchg + 2 * 64 * kXStride);      // [kMaxTok]
+  uint64_t* full = reinterpret_cast<uint64_t*>(tok + kMaxTok);
+  uint64_t* empty = full + S;
+  uint64_t* acc_full = empty + S;
+  uint64_t* acc_empty = acc_full + 4;
+  uint64_t* drain = acc_empty + 4;
+  uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
+  volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
+  int* s_u = const_cast<int*>(s_abort) + 1;
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nb = gridDim.x, b = blockIdx.x;
+  KLOG(DMOE_KERNEL_EXPERTS, 0);
+  if (tid == 0) ED_AT(0);
+
+  if (tid == 0) {
+    for (int s = 0; s < S; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], 1);
+    }
+    for (int a = 0; a < 4; ++a) {
+      ptx::mbar_init(&acc_full[a], 1);
+      ptx::mbar_init(&acc_empty[a], 128);
+    }
+    ptx::mbar_init(drain, 1);
+    ptx::fence_mbarrier_init();
+    *s_abort = 0;
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(s_tmem, p.tmem_cols);
+    ptx::tmem_relinquish();
+  }
+  pdl_launch_dependents();
+  pdl_wait();   // the dispatch is complete from here on
+  if (tid == 0) {
+    int u = __ldcg(p.n_unique);
+    if (u < 0 || u > p.E) {
+      record_error(p.err, kErrBadDispatch, kAtGateUp, u);
+      u = 0;
+    }
+    *s_u = u;
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  const uint32_t tmem_base = *s_tmem;
+  const int U = *s_u;
+  const int G = U + p.has_shared;
+  const int ngu_s = p.has_shared ? p.Is / 64 : 0, ngu_r = p.I / 64;
+  const int ndn = p.d / kTileM;
+  const int NGU = ngu_s + U * ngu_r;
+  const int ND = G * ndn;
+  // first down unit of this CTA: the round-robin continues after the NGU gate/up units
+  const int v0 = ((b - NGU % nb) % nb + nb) % nb;
+  if (tid == 0) ED_AT(1);
+
+  auto group = [&](int gi) -> Grp {
+    Grp g;
+    if (gi < p.has_shared) {
+      g.shared = true;
+      g.e = 0;
+      g.row0 = 0;
+      g.n = p.T;
+      g.Ig = p.Is;
+      return g;
+    }
+    const int u = gi - p.has_shared;
+    int row0 = __ldcg(p.offsets + u);
+    int n = __ldcg(p.offsets + u + 1) - row0;
+    int e = __ldcg(p.unique_ids + u);
+    if (e < 0 || e >= p.E || n < 0 || n > p.T || row0 < 0 || row0 + n > p.T * p.k) {
+      record_error(p.err, kErrBadDispatch, kAtGateUp, u);
+      n = 0;
+      e = 0;
+      row0 = 0;
+    }
+    g.shared = false;
+    g.e = e;
+    g.row0 = row0;
+    g.n = n;
+    g.Ig = p.I;
+    return g;
+  };
+  // gate/up unit -> (group, 64-row tile)
+  auto gu_unit = [&](int u, int& gi, int& m) {
+    if (u < ngu_s) {
+      gi = 0;
+      m = u;
+    } else {
+      gi = p.has_shared + (u - ngu_s) / ngu_r;
+      m = (u - ngu_s) % ngu_r;
+    }
+  };
+  auto wait = [&](uint64_t* bar, uint32_t parity, int value) -> bool {
+    if (*s_abort) return false;
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = ptx::globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+      if (ptx::mbar_try_wait(bar, parity)) return true;
+      if ((i & 63u) == 0u) {
+        if (*s_abort) return false;
+        if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {
+          record_error(p.err, kErrTimeout, kAtGateUp, value);
+          *s_abort = 1;
+          return false;
+        }
+      }
+    }
+  };
+  const int kc = p.d / kStageK;      // stages of one gate/up tile
+
+  if (warp == 0 && lane == 0) {
+    // ================= TMA producer
+    const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
+    const uint64_t pol_x = ptx::policy_evict_last();    // x and H: re-read by many tiles
+    int stage = 0, issued = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    bool first = true;
+    for (int u = b; u < NGU && ok; u += nb) {
+      int gi, m;
+      gu_unit(u, gi, m);
+      const Grp g = group(gi);
+      const CUtensorMap* mg = g.shared ? &tm.sg : &tm.wg;
+      const CUtensorMap* mu = g.shared ? &tm.su : &tm.wu;
+      const int arow = (g.shared ? 0 : g.e * p.I) + m * 64;
+      if (first) ED_SET(10, u);
+      for (int c = 0; c < kc; ++c) {
+        if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+        ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
+        uint8_t* a_dst = ring_a + stage * kAStage;
+        uint8_t* b_dst = ring_b + stage * bstage;
+#pragma unroll
+        for (int kb = 0; kb < kKB; ++kb) {
+          const int kx = c * kStageK + kb * kTileK;
+          ptx::tma_load_2d(a_dst + kb * kABox, mg, &full[stage], kx, arow, pol_w);
+          ptx::tma_load_2d(a_dst + kb * kABox + kGateBox, mu, &full[stage], kx, arow, pol_w);
+          ptx::tma_load_2d(b_dst + kb * bbox, &tm.x, &full[stage], kx, 0, pol_x);
+        }
+        ++issued;
+        if (++stage == S) { stage = 0; phase ^= 1u; }
+      }
+      first = false;
+    }
+    first = true;
+    for (int v = v0; v < ND && ok; v += nb) {
+      const int gi = v / ndn, i = v % ndn;
+      const Grp g = group(gi);
+      const CUtensorMap* md = g.shared ? &tm.sd : &tm.wd;
+      const int arow = (g.shared ? 0 : g.e * p.d) + i * kTileM;
+      const int ndk = g.Ig / kStageK;
+      const int pre = ndk < S ? ndk : S;
+      const int st0 = stage;
+      if (first) ED_SET(11, v);
+      // weights first: they do not depend on the gate/up phase
+      int done = 0;
+      for (int c = 0; c < pre; ++c, ++done) {
+        if (!wait(&empty[stage], phase ^ 1u, v)) { ok = false; break; }
+        ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
+        uint8_t* a_dst = ring_a + stage * kAStage;
+#pragma unroll
+        for (int kb = 0; kb < kKB; ++kb)
+          ptx::tma_load_2d(a_dst + kb * kABox, md, &full[stage], c * kStageK + kb * kTileK, arow,
+                           pol_w);
+        ++issued;
+        if (++stage == S) { stage = 0; phase ^= 1u; }
+      }
+      if (first) ED_AT(5);
+      // then the H rows, once every gate/up tile of the group is published
+      const int target = g.Ig / 64;
+      if (ok && ld_acquire(p.h_ready + gi) < target) {
+        const uint64_t t0 = ptx::globaltimer_ns();
+        while (ld_acquire(p.h_ready + gi) < target) {
+          if (*s_abort) { ok = false; break; }
+          if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {
+            record_error(p.err, kErrTimeout, kAtDown, v);
+            *s_abort = 1;
+            ok = false;
+            break;
+          }
+        }
+      }
+      fence_proxy_async_global();
+      if (first) ED_AT(6);
+      {
+        int st = st0;
+        for (int c = 0; c < done; ++c) {
+          if (ok) {
+            uint8_t* b_dst = ring_b + st * bstage;
+#pragma unroll
+            for (int kb = 0; kb < kKB; ++kb)
+              ptx::tma_load_2d(b_dst + kb * bbox, &tm.h, &full[st], c * kStageK + kb * kTileK,
+                               gi * p.n_pad, pol_x);
+          } else {
+            // keep the barrier accounting whole: complete the stage without B data
+            ptx::mbar_complete_tx_local(&full[st], bstage);
+          }
+          if (++st == S) st = 0;
+        }
+      }
+      for (int c = pre; c < ndk && ok; ++c) {
+        if (!wait(&empty[stage], phase ^ 1u, v)) { ok = false; break; }
+        ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
+        uint8_t* a_dst = ring_a + stage * kAStage;
+        uint8_t* b_dst = ring_b + stage * bstage;
+#pragma unroll
+        for (int kb = 0; kb < kKB; ++kb) {
+          const int kx = c * kStageK + kb * kTileK;
+          ptx::tma_load_2d(a_dst + kb * kABox, md, &full[stage], kx, arow, pol_w);
+          ptx::tma_load_2d(b_dst + kb * bbox, &tm.h, &full[stage], kx, gi * p.n_pad, pol_x);
+        }
+        ++issued;
+        if (++stage == S) { stage = 0; phase ^= 1u; }
+      }
+      first = false;
+    }
+    if (!ok) {
+      // let the copies already in flight land before the CTA exits
+      int st = stage;
+      uint32_t ph = phase;
+      const int n = issued < S ? issued : S;
+      for (int i = 0; i < n; ++i) {
+        if (--st < 0) { st = S - 1; ph ^= 1u; }
+        const uint64_t t0 = ptx::globaltimer_ns();
+        while (!ptx::mbar_try_wait(&full[st], ph) &&
+               ptx::globaltimer_ns() - t0 < kTimeoutNs / 10) {
+        }
+      }
+    }
+  } else if (warp == 1 && lane == 0) {
+    // ================= MMA issuer
+    int stage = 0, acc = 0;
+    uint32_t phase = 0, acc_phase = 0;
+    bool ok = true, first = true;
+    auto run = [&](int nstages, int n, int value, bool gu) {
+      const uint32_t n_mma = (uint32_t)(n > 0 ? ((n + 15) & ~15) : 16);
+      const uint32_t idesc = ptx::idesc_bf16(kTileM, n_mma);
+      if (!wait(&acc_empty[acc], acc_phase ^ 1u, value)) { ok = false; return; }
+      ptx::tc_fence_after();
+      const uint32_t d0 = tmem_base + (uint32_t)(acc * p.n_pad);
+      for (int c = 0; c < nstages; ++c) {
+        if (!wait(&full[stage], phase, value)) { ok = false; return; }
+        if (gu && first && c == 0) ED_AT(2);
+        ptx::tc_fence_after();
+        const uint32_t a0 = ptx::smem_addr(ring_a + stage * kAStage);
+        const uint32_t b0 = ptx::smem_addr(ring_b + stage * bstage);
+#pragma unroll
+        for (int kb = 0; kb < kKB; ++kb)
+#pragma unroll
+          for (int kk = 0; kk < kTileK / 16; ++kk)
+            ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kABox + kk * 32),
+                          ptx::sdesc_k_sw128(b0 + kb * bbox + kk * 32), idesc,
+                          (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
+        ptx::mma_commit(&empty[stage]);
+        if (++stage == S) { stage = 0; phase ^= 1u; }
+      }
+      ptx::mma_commit(&acc_full[acc]);
+      if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
+    };
+    for (int u = b; u < NGU && ok; u += nb) {
+      int gi, m;
+      gu_unit(u, gi, m);
+      // all T token columns: the B box is x (rows >= T are zeros)
+      run(kc, p.T, u, true);
+      if (first) ED_AT(3);
+      first = false;
+    }
+    first = true;
+    for (int v = v0; v < ND && ok; v += nb) {
+      const Grp g = group(v / ndn);
+      run(g.Ig / kStageK, p.T, v, false);
+      if (first) ED_AT(7);
+      first = false;
+    }
+    // no MMA may still run when TMEM is released
+    ptx::mma_commit(drain);
+    const uint64_t t0 = ptx::globaltimer_ns();
+    while (!ptx::mbar_try_wait(drain, 0) && ptx::globaltimer_ns() - t0 < kTimeoutNs) {
+    }
+  } else if (warp >= 2) {
+    // ================= epilogue: warps 2..5, TMEM lanes 32*(warp%4) ..
+    const int q = warp & 3;
+    const int et = tid - 64;                      // 0..127
+    const int row = q * 32 + lane;                // accumulator row of this thread
+    const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    const bool is_gate = q < 2;
+    const int r64 = (q & 1) * 32 + lane;          // row within the 64-row slice
+    const int n_mma = (p.T + 15) & ~15;
+    int acc = 0, xb = 0;
+    uint32_t acc_phase = 0;
+    bool first = true;
+    for (int u = b; u < NGU; u += nb) {
+      int gi, m;
+      gu_unit(u, gi, m);
+      const bool ok = epi_all(wait(&acc_full[acc], acc_phase, u));
+      if (!ok) break;
+      ptx::tc_fence_after();
+      const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
+      __nv_bfloat16* hg = p.hdense + (size_t)gi * p.n_pad * p.imax + m * 64 + r64;
+      for (int c0 = 0; c0 < n_mma; c0 += 16) {
+        float v[16];
+        ptx::tmem_ld16(tbase + c0, v);
+        ptx::tmem_ld_wait();
+        float* buf = xchg + xb * (64 * kXStride);
+        if (!is_gate) {
+#pragma unroll
+          for (int c = 0; c < 16; ++c) buf[r64 * kXStride + c] = v[c];
+        }
+        named_bar_sync(2, 128);
+        if (is_gate) {
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            hg[(size_t)(c0 + c) * p.imax] = __float2bfloat16(silu_f(v[c]) * buf[r64 * kXStride + c]);
+        }
+        xb ^= 1;
+      }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&acc_empty[acc]);
+      if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
+      // publish the tile: the barrier orders every epilogue thread's H stores before one
+      // release add; a reader acquires the counter, then fences the async proxy
+      named_bar_sync(2, 128);
+      if (et == 0) {
+        red_release_add(p.h_ready + gi, 1);
+        if (first) ED_AT(4);
+      }
+      first = false;
+    }
+    first = true;
+    for (int v = v0; v < ND; v += nb) {
+      const int gi = v / ndn, i = v % ndn;
+      const Grp g = group(gi);
+      if (!g.shared && et < g.n) tok[et] = __ldcg(p.rows + g.row0 + et) / p.k;
+      const bool ok = epi_all(wait(&acc_full[acc], acc_phase, v));   // also orders tok[]
+      if (!ok) break;
+      ptx::tc_fence_after();
+      const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
+      const int drow = i * kTileM + row;
+      if (g.shared) {
+        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+          float vv[16];
+          ptx::tmem_ld16(tbase + c0, vv);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            if (c0 + c < p.T) p.yshared[(size_t)(c0 + c) * p.d + drow] = vv[c];
+        }
+      } else {
+        // the accumulator column of token t is the group's output for t: keep the routed
+        // ones, in dispatch order, through this thread's own staging row
+        float* srow = stage_t + row * SP;
+        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+          float vv[16];
+          ptx::tmem_ld16(tbase + c0, vv);
+          ptx::tmem_ld_wait();
+#pragma unroll
+          for (int c = 0; c < 16; ++c) srow[c0 + c] = vv[c];
+        }
+        float* out = p.yslot + (size_t)g.row0 * p.d + drow;
+        for (int r = 0; r < g.n; ++r) {
+          const int t = tok[r];
+          if (t >= 0 && t < p.T) out[(size_t)r * p.d] = srow[t];
+        }
+      }
+      ptx::tc_fence_before();
+      ptx::mbar_arrive(&acc_empty[acc]);
+      if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
+      named_bar_sync(2, 128);   // tok[] is rewritten by the next unit
+      if (first && et == 0) ED_AT(8);
+      first = false;
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  if (warp == 1) {
+    __syncwarp();
+    ptx::tmem_dealloc(tmem_base, p.tmem_cols);
+  }
+  if (tid == 0) {
+    // the last CTA clears the group counters for the next call
+    __threadfence();
+    if (atomicAdd(p.exit_ticket, 1) == nb - 1) {
+      for (int gi = 0; gi <= p.E; ++gi) p.h_ready[gi] = 0;
+      __threadfence();
+      *p.exit_ticket = 0;
+    }
+    ED_AT(9);
+  }
+  KLOG(DMOE_KERNEL_EXPERTS, 1);
+}
+
+// ------------------------------------------------------------------ host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+// bf16 matrix [rows, cols] row-major (row pitch `pitch` elements), box = 64 columns (128 B)
+// x box_rows rows, 128-B swizzle.
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+              uint64_t pitch = 0) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {(pitch ? pitch : cols) * 2};
+  const cuuint32_t box[2] = {64, box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int max_smem_optin() {
+  int dev = 0, v = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&v, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  return v;
+}
+
+uint32_t pow2_cols(uint32_t n) {
+  uint32_t c = 32;
+  while (c < n) c <<= 1;
+  return c;
+}
+
+// Shared memory besides the ring: staging tile, SwiGLU exchange, token list, barriers.
+size_t fixed_smem(int n_pad, int stages) {
+  return 1024 /* alignment */ + (size_t)kTileM * (n_pad + 1) * 4 + kXchgBytes + kMaxTok * 4 +
+         (size_t)(2 * stages + 9) * 8 + 64;
+}
+
+int plan_stages(int T) {
+  const int n_pad = ((T + 15) / 16) * 16;
+  const long avail = (long)max_smem_optin() - (long)fixed_smem(n_pad, kMaxStagesD);
+  int stages = (int)(avail / (kAStage + kKB * n_pad * 128));
+  return stages > kMaxStagesD ? kMaxStagesD : stages;
+}
+
+}  // namespace
+
+#ifdef DMOE_TRACE
+DMOE_KLOG_EXPORT(dmoe_debug_klog_decode)
+extern "C" int dmoe_debug_dtrace(void* host) {
+  return (int)cudaMemcpyFromSymbol(host, g_dtrace, sizeof(g_dtrace));
+}
+extern "C" int dmoe_debug_dtrace_clear() {
+  static uint64_t zeros[kMaxPersistentCtas * 32];
+  return (int)cudaMemcpyToSymbol(g_dtrace, zeros, sizeof(zeros));
+}
+#endif
+
+bool experts_decode_ok(int T, int d, int I, int Is) {
+  if (T < 1 || T > kMaxTok || d % kTileM != 0 || I % kStageK != 0 || (Is > 0 && Is % kStageK != 0))
+    return false;
+  return plan_stages(T) >= 2;
+}
+
+cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
+  const bool has_shared = a.Is > 0;
+  const int stages = plan_stages(a.T);
+  if (stages < 2) return cudaErrorInvalidConfiguration;
+  const int n_pad = ((a.T + 15) / 16) * 16;
+  const int imax = a.I > a.Is ? a.I : a.Is;
+
+  DMaps m;
+  bool ok = make_map(&m.wg, a.w_gate, (uint64_t)a.E * a.I, a.d, 64) &&
+            make_map(&m.wu, a.w_up, (uint64_t)a.E * a.I, a.d, 64) &&
+            make_map(&m.wd, a.w_down, (uint64_t)a.E * a.d, a.I, kTileM) &&
+            make_map(&m.x, a.x, (uint64_t)a.T, a.d, (uint32_t)n_pad) &&
+            make_map(&m.h, a.hdense, (uint64_t)(a.E + 1) * n_pad, (uint64_t)imax,
+                     (uint32_t)n_pad);
+  if (ok && has_shared)
+    ok = make_map(&m.sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
+         make_map(&m.su, a.ws_up, (uint64_t)a.Is, a.d, 64) &&
+         make_map(&m.sd, a.ws_down, (uint64_t)a.d, a.Is, kTileM);
+  if (!has_shared) { m.sg = m.wg; m.su = m.wu; m.sd = m.wd; }
+  if (!ok) return cudaErrorInvalidValue;
+
+  DParams p{};
+  p.n_unique = a.n_unique;
+  p.unique_ids = a.unique_ids;
+  p.offsets = a.offsets;
+  p.rows = a.rows;
+  p.hdense = a.hdense;
+  p.yslot = a.yslot;
+  p.yshared = a.yshared;
+  p.h_ready = a.h_ready;
+  p.exit_ticket = a.tickets + kTicketDecodeExit;
+  p.err = a.err;
+  p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
+  p.imax = imax;
+  p.n_pad = n_pad;
+  p.stages = stages;
+  p.has_shared = has_shared ? 1 : 0;
+  p.n_acc = 512 / n_pad > 4 ? 4 : 512 / n_pad;
+  p.tmem_cols = pow2_cols((uint32_t)(p.n_acc * n_pad));
+  const size_t smem =
+      (size_t)stages * (kAStage + (size_t)kKB * n_pad * 128) + fixed_smem(n_pad, stages);
+
+  static std::mutex mu;
+  static int attr_dev_mask = 0;  // the dynamic smem limit is a per-device function attribute
+  int dev = 0;
+  cudaGetDevice(&dev);
+  {
+    std::lock_guard<std::mutex> lock(mu);
+    if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
+      cudaError_t e = cudaFuncSetAttribute(moe_decode_kernel,
+                                           cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           max_smem_optin());
+      if (e != cudaSuccess) return e;
+      if (dev < 31) attr_dev_mask |= 1 << dev;
+    }
+  }
+  int grid = device_sm_count();
+  if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
+  prof_begin(DMOE_KERNEL_EXPERTS, s);
+  cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
+  prof_end(DMOE_KERNEL_EXPERTS, s);
+  if (e != cudaSuccess) return e;
+  return launch_combine(a, s);
+}
+
+}  // namespace dmoe

@@ -771,10 +771,14 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   if (e != cudaSuccess) return e;
 
   // 3. gate-weighted combine
+  return launch_combine(a, s);
+}
+
+cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s) {
   dim3 cgrid((a.d / 4 + 255) / 256, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
-  e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared, a.pos,
-                a.topk_gate, a.y, a.k, a.d, has_shared ? 1 : 0);
+  cudaError_t e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared,
+                            a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0);
   prof_end(DMOE_KERNEL_COMBINE, s);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

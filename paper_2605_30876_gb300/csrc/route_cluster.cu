@@ -306,7 +306,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       }
 #pragma unroll
       for (int j = 0; j < J; ++j) v[j] = ((valid >> j) & 1u) ? v[j] + s_bias[lane + 32 * j] : -INFINITY;
+      CT_AT(9);
       warp_softmax8(v, valid);
+      CT_AT(10);
       float* prow = sP + warp * kMaxExperts;
 #pragma unroll
       for (int j = 0; j < J; ++j)
@@ -317,6 +319,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       int my_idx;
       float my_val;
       warp_topk(v, id, valid, k, my_idx, my_val);
+      CT_AT(11);
       if (a.mode == DMOE_ROUTE_BLOCK) {
         // TopKMask: the k winners into the zeroed row of token t in the CTA that routes
         // its block (block b: CTA b mod 8)
@@ -357,6 +360,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         a.topk_gate[(size_t)t * k + r] = g;
         st_peer_u32(peer_addr(&sIdx[t * k + r], 0), (uint32_t)e);
       };
+      CT_AT(12);
       if (size <= 32)
         mask_topk_small(k, B, size, order, prob, out, reinterpret_cast<float*>(dsm + kOffSv),
                         reinterpret_cast<int*>(dsm + kOffSelE),
@@ -371,6 +375,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     if (a.coreset_size != nullptr)
       for (int i = tid; i < a.n_blocks; i += 256) a.coreset_size[i] = 0;
   }
+  CT_AT(13);
   cluster_sync();
   CT_AT(6);
 
