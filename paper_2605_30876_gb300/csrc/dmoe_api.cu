@@ -85,6 +85,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.logits_part = take(sizeof(float) * (w.router_splits == 0 ? 1 : w.router_splits) * T * E);
   w.probs = take(sizeof(float) * T * E);
   w.probs_hat = take(sizeof(float) * T * E);
+  w.cand = take(sizeof(uint2) * T * ((E + 31) / 32) * k);
   w.tk_idx = take(sizeof(int32_t) * T * k);
   w.tk_gate = take(sizeof(float) * T * k);
   w.unique_ids = take(sizeof(int32_t) * E);
@@ -164,6 +165,7 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.probs = probs != nullptr ? probs : at<float>(ws, plan.probs);
   a.probs_requested = probs != nullptr;
   a.probs_hat = at<float>(ws, plan.probs_hat);
+  a.cand = at<uint2>(ws, plan.cand);
   a.topk_idx = topk_idx;
   a.topk_gate = topk_gate;
   a.coreset = coreset;

@@ -61,6 +61,8 @@ struct Workspace {
   size_t logits_part;  // fp32 [router_splits, T, E]
   size_t probs;        // fp32 [T, E]
   size_t probs_hat;    // fp32 [T, E]   TopKMask(s_i, k)
+  size_t cand;         // uint2 [T, ceil(E/32), k]: decode-size routing, each 32-expert group's
+                       // k best (order key, id) per token
   size_t tk_idx;       // int32 [T, k] routed experts (when the caller does not supply)
   size_t tk_gate;      // fp32 [T, k]
   size_t unique_ids;   // int32 [E]
@@ -135,6 +137,7 @@ struct RouterArgs {
   float* logits_part;
   float* probs;        // [T, E]
   float* probs_hat;    // [T, E] (block mode)
+  uint2* cand;         // [T, ceil(E/32), k] (decode-size routing)
   int32_t* topk_idx;   // [T, k] final routing
   float* topk_gate;    // [T, k]
   int32_t* coreset;    // [n_blocks, E] or null

@@ -171,7 +171,6 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
-  pdl_launch_dependents();
   pdl_wait();   // the dispatch is complete from here on
   if (tid == 0) {
     int u = __ldcg(p.n_unique);
@@ -515,6 +514,9 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  // the combine may start now: launched earlier, its waiting CTAs would share SMs with the
+  // routing launch of this forward and slow it down
+  pdl_launch_dependents();
   if (warp == 1) {
     __syncwarp();
     ptx::tmem_dealloc(tmem_base, p.tmem_cols);

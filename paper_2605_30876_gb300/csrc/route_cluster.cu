@@ -18,6 +18,33 @@
 // global memory, read past the L1 (ld.global.cg) after the ticket's acquire.
 #include <math.h>
 
+// Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 64 + stage] (stage 0:
+// globaltimer, others: 1 = reached; + 32: clock64): 0 entry, 1 TMA landed, 8 x converted,
+// 2 partial logits done, 3 logits reduced, 4 ticket, 9 score loads issued, 10 softmax,
+// 11 top-k, 5 scores, 12 coreset, 13 MaskOutside, 6 Algorithm 1, 7 dispatch; 16-24: steps
+// inside the dispatch, the coreset and MaskOutside (DMOE_STAMP in the shared headers).
+#ifdef DMOE_TRACE
+#include <stdint.h>
+__device__ uint64_t g_ctrace[64 * 8 * 64];
+#define CT_AT(st)                                                                       \
+  do {                                                                                  \
+    if (threadIdx.x == 0) {                                                             \
+      const int c_ = ((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 64 + (st);         \
+      if ((st) == 0) {                                                                  \
+        uint64_t t_;                                                                    \
+        asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                          \
+        g_ctrace[c_] = t_;                                                              \
+      } else {                                                                          \
+        g_ctrace[c_] = 1;                                                               \
+      }                                                                                 \
+      g_ctrace[c_ + 32] = clock64();                                                    \
+    }                                                                                   \
+  } while (0)
+#define DMOE_STAMP(st) CT_AT(st)
+#else
+#define CT_AT(st) ((void)0)
+#endif
+
 #include "dispatch_impl.cuh"
 #include "dmoe_internal.cuh"
 #include "routing_device.cuh"
@@ -30,28 +57,11 @@ constexpr int kCl = 8;                 // CTAs per cluster (split of d)
 constexpr int kClExp = 32;             // experts per cluster
 constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
 constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
+constexpr int kClMaxCand = (kMaxExperts / kClExp) * kMaxTopK;   // candidates of one token
 static_assert(kClMaxTok * kClMaxDChunk * 2 >= 4 * kClMaxTok * kClExp * 4,
               "the quarter sums must fit where the bf16 x slice was");
 
-// Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 32 + stage] (globaltimer;
-// + 16: clock64): 0 entry,
-// 1 TMA landed, 8 x converted, 2 partial logits done, 3 logits reduced, 4 ticket, 5 scores,
-// 6 Algorithm 1, 7 dispatch.
-#ifdef DMOE_TRACE
-__device__ uint64_t g_ctrace[64 * 8 * 32];
-#define CT_AT(st)                                                                       \
-  do {                                                                                  \
-    if (threadIdx.x == 0) {                                                             \
-      uint64_t t_;                                                                      \
-      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                            \
-      const int c_ = ((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 32 + (st);         \
-      g_ctrace[c_] = t_;                                                                \
-      g_ctrace[c_ + 16] = clock64();                                                    \
-    }                                                                                   \
-  } while (0)
-#else
-#define CT_AT(st) ((void)0)
-#endif
+
 
 struct ClusterArgs {
   CUtensorMap wmap;   // W_r [d, E] fp32, box 32 experts x d/8 rows
@@ -93,14 +103,13 @@ __device__ __forceinline__ void st_peer_f32(uint32_t addr, float v) {
 
 // Shared-memory layout after the logits (the W_r / x slices are dead by then), in bytes
 // from the dynamic base: scores of this CTA's tokens, the top-k ids for the dispatch (rank
-// 0), the MaskOutside scratch, and the dense TopKMask rows of the blocks this CTA routes.
+// 0), the coreset of each token's block, and the dense TopKMask rows of the blocks this CTA
+// routes.
 constexpr int kOffP = 0;                                      // f32 [8][kMaxExperts]
 constexpr int kOffIdx = kOffP + 8 * kMaxExperts * 4;          // i32 [kClMaxTok * kMaxTopK]
-constexpr int kOffSv = kOffIdx + kClMaxTok * kMaxTopK * 4;    // f32 [kClMaxTok][32]
-constexpr int kOffSelE = kOffSv + kClMaxTok * 32 * 4;         // i32 [kClMaxTok][kMaxTopK]
-constexpr int kOffSelV = kOffSelE + kClMaxTok * kMaxTopK * 4; // f32 [kClMaxTok][kMaxTopK]
+constexpr int kOffCore = kOffIdx + kClMaxTok * kMaxTopK * 4;  // i32 [8][1 + kMaxExperts]
 constexpr int kOffHat = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;  // f32 [kClMaxTok][kMaxExperts]
-static_assert(kOffSelV + kClMaxTok * kMaxTopK * 4 <= kClMaxDChunk * kClExp * 4,
+static_assert(kOffCore + 8 * (1 + kMaxExperts) * 4 <= kClMaxDChunk * kClExp * 4,
               "the routing scratch must fit where the W_r slice was");
 
 // Partial logits of the CTA's d slice: thread (q, eg, tg) accumulates experts 4eg..4eg+3 of
@@ -147,9 +156,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ uint32_t s_last;
   __shared__ float s_part[kClMaxTok * kClExp];                     // partial logits [T][32]
-  __shared__ uint32_t s_bits[(kClMaxTok / 32) * kMaxExperts];
-  __shared__ uint16_t s_base[(kClMaxTok / 32) * kMaxExperts];
   __shared__ float s_bias[kMaxExperts];
+  __shared__ uint32_t s_loc[8][32];                  // one token's keys per warp
+  __shared__ uint2 s_cand[8][kClMaxCand];            // merge: one token's candidates per warp
   const RouterArgs& a = f.r;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int T = a.T, E = a.E, k = a.k, B = a.B;
@@ -215,18 +224,16 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   float* Xf = reinterpret_cast<float*>(dsm + kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2);
   const int xs = DC + 1;
   {
-    const int DC8 = DC / 8;  // d % 64 == 0: whole groups of eight per row
-    for (int i = tid; i < T * DC8; i += 256) {
-      const int t = i / DC8, c = (i - t * DC8) * 8;
-      const uint4 raw = *reinterpret_cast<const uint4*>(Xs + t * DC + c);
-      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-      float* dst = Xf + t * xs + c;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        dst[2 * q] = __low2float(p2[q]);
-        dst[2 * q + 1] = __high2float(p2[q]);
+    // warp per row, lanes on consecutive bf16 pairs: conflict-free loads, 2-way stores
+    const int DC2 = DC / 2;
+    const __nv_bfloat162* X2 = reinterpret_cast<const __nv_bfloat162*>(Xs);
+    for (int t = warp; t < T; t += 8)
+      for (int c2 = lane; c2 < DC2; c2 += 32) {
+        const __nv_bfloat162 v2 = X2[t * DC2 + c2];
+        float* dst = Xf + t * xs + 2 * c2;
+        dst[0] = __low2float(v2);
+        dst[1] = __high2float(v2);
       }
-    }
   }
   __syncthreads();
   CT_AT(8);
@@ -249,7 +256,10 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   }
   CT_AT(2);
   cluster_sync();
-  // CTA r adds the partials of tokens t = r (mod 8), in rank order
+  // CTA r adds the partials of tokens t = r (mod 8), in rank order, adds the bias, and keeps
+  // the cluster's k best experts of the token (candidates for the top-k over all experts:
+  // any expert of the top-k is among the k best of its own cluster)
+  uint2* cand = a.cand;   // [T][clusters][k]: (order key, id)
   {
     const int t = (int)rank + 8 * warp;
     if (t < T) {
@@ -260,7 +270,21 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       float v = 0.f;
 #pragma unroll
       for (int q = 0; q < kCl; ++q) v += p[q];
-      if (e0 + lane < E) a.logits_part[(size_t)t * E + e0 + lane] = v;
+      const bool ok = e0 + lane < E;
+      v += ok ? s_bias[e0 + lane] : 0.f;
+      if (ok) a.logits_part[(size_t)t * E + e0 + lane] = v;
+      const uint32_t key = ok ? order_key(v) : 0u;
+      s_loc[warp][lane] = key;
+      __syncwarp();
+      int r = 0;
+#pragma unroll 8
+      for (int j = 0; j < 32; ++j) {
+        const uint32_t kj = s_loc[warp][j];
+        r += (kj > key || (kj == key && j < lane)) ? 1 : 0;
+      }
+      if (r < k)
+        cand[((size_t)t * n_clusters + blockIdx.y) * k + r] =
+            make_uint2(key, ok ? (uint32_t)(e0 + lane) : 0xffffffffu);
     }
   }
   // every CTA of the cluster has written its logits and finished reading its peers' s_part
@@ -270,9 +294,10 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 
   // ---- 2. the last cluster to finish routes the forward
   if (rank == 0 && tid == 0) {
-    __threadfence();
-    const uint32_t last = (atomicAdd(f.ticket, 1) == n_clusters - 1) ? 1u : 0u;
-    if (last) __threadfence();  // acquire the other clusters' logits
+    // release this cluster's logits and candidates, acquire the others' (GPU scope)
+    uint32_t old;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(f.ticket) : "memory");
+    const uint32_t last = (old == (uint32_t)n_clusters - 1) ? 1u : 0u;
     for (uint32_t q = 0; q < (uint32_t)kCl; ++q) st_peer_u32(peer_addr(&s_last, q), last);
   }
   cluster_sync();
@@ -291,34 +316,70 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   {
     const int t = 8 * (int)rank + warp;
     if (t < T) {
+      const int nc = n_clusters * k;                       // candidates of the token
+      const uint2* tc = cand + (size_t)t * nc;
+      uint2 cd[kClMaxCand / 32];
+#pragma unroll
+      for (int q = 0; q < kClMaxCand / 32; ++q) {
+        const int ci = lane + 32 * q;
+        cd[q] = ci < nc ? __ldcg(tc + ci) : make_uint2(0u, 0xffffffffu);
+      }
       float v[J];
-      int id[J];
       uint32_t valid = 0;
 #pragma unroll
       for (int j = 0; j < J; ++j) {
         const int e = lane + 32 * j;
-        id[j] = e;
-        v[j] = 0.f;
+        v[j] = -INFINITY;
         if (e < E) {
           valid |= 1u << j;
-          v[j] = __ldcg(a.logits_part + (size_t)t * E + e);
+          v[j] = __ldcg(a.logits_part + (size_t)t * E + e);   // logit + bias
         }
       }
-#pragma unroll
-      for (int j = 0; j < J; ++j) v[j] = ((valid >> j) & 1u) ? v[j] + s_bias[lane + 32 * j] : -INFINITY;
       CT_AT(9);
-      warp_softmax8(v, valid);
-      CT_AT(10);
+      // scores: softmax over all experts (row kept in shared memory for MaskOutside)
+      float mx = -INFINITY;
+#pragma unroll
+      for (int j = 0; j < J; ++j) mx = fmaxf(mx, v[j]);
+      const float M = key_value(__reduce_max_sync(0xffffffffu, order_key(mx)));
+      float sum = 0.f;
+#pragma unroll
+      for (int j = 0; j < J; ++j) {
+        v[j] = ((valid >> j) & 1u) ? __expf(v[j] - M) : 0.f;
+        sum += v[j];
+      }
+      const float inv = 1.f / warp_sum(sum);
       float* prow = sP + warp * kMaxExperts;
 #pragma unroll
       for (int j = 0; j < J; ++j)
         if ((valid >> j) & 1u) {
-          prow[lane + 32 * j] = v[j];
-          if (a.probs_requested) a.probs[(size_t)t * E + lane + 32 * j] = v[j];
+          const float pv = v[j] * inv;
+          prow[lane + 32 * j] = pv;
+          if (a.probs_requested) a.probs[(size_t)t * E + lane + 32 * j] = pv;
         }
-      int my_idx;
-      float my_val;
-      warp_topk(v, id, valid, k, my_idx, my_val);
+      CT_AT(10);
+      // top-k over the clusters' candidates: each cluster's list is sorted (best first), so
+      // k rounds of a tournament over the list heads (lane c holds cluster c's head; larger
+      // score, ties to the lower id) give the winners in order; a winner's score is computed
+      // exactly as in the row above
+#pragma unroll
+      for (int q = 0; q < kClMaxCand / 32; ++q) s_cand[warp][lane + 32 * q] = cd[q];
+      __syncwarp();
+      int head = 0;
+      uint2 hc = lane < n_clusters ? s_cand[warp][lane * k] : make_uint2(0u, 0xffffffffu);
+      int my_idx = -1;
+      float my_val = 0.f;
+      for (int r = 0; r < k; ++r) {
+        const uint32_t kmax = __reduce_max_sync(0xffffffffu, hc.x);
+        const uint32_t imin = __reduce_min_sync(0xffffffffu, hc.x == kmax ? hc.y : 0xffffffffu);
+        if (lane == r) {
+          my_idx = (int)imin;
+          my_val = __expf(key_value(kmax) - M) * inv;
+        }
+        if (hc.x == kmax && hc.y == imin) {
+          ++head;
+          hc = head < k ? s_cand[warp][lane * k + head] : make_uint2(0u, 0xffffffffu);
+        }
+      }
       CT_AT(11);
       if (a.mode == DMOE_ROUTE_BLOCK) {
         // TopKMask: the k winners into the zeroed row of token t in the CTA that routes
@@ -340,34 +401,71 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   cluster_sync();
   CT_AT(5);
 
-  // ---- 4. Algorithm 1: block b by CTA b mod 8, the block's rows read from the shared
-  // memory of the CTAs that scored them (token t: CTA t / 8, row t mod 8)
+  // ---- 4. Algorithm 1: block b by CTA b mod 8 (Aggregate .. Top-P and the k floor), then
+  // MaskOutside + TopK by the warp that scored each token, on its own score row
   if (a.mode == DMOE_ROUTE_BLOCK) {
     __shared__ int order[kMaxExperts];
+    int* sCore = reinterpret_cast<int*>(dsm + kOffCore);    // [8 warps][1 + kMaxExperts]
     for (int b = (int)rank; b < a.n_blocks; b += kCl) {
       const int t0 = b * B;
       const int size = block_coreset_steps(
           E, k, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
-      auto prob = [&](int i, int e) {
-        const int t = t0 + i;
-        return ld_peer_f32(peer_addr(sP + (t & 7) * kMaxExperts + e, (uint32_t)(t >> 3)));
-      };
-      auto out = [&](int i, int r, int e, float g) {
-        const int t = t0 + i;
-        a.topk_idx[(size_t)t * k + r] = e;
-        a.topk_gate[(size_t)t * k + r] = g;
-        st_peer_u32(peer_addr(&sIdx[t * k + r], 0), (uint32_t)e);
-      };
-      CT_AT(12);
-      if (size <= 32)
-        mask_topk_small(k, B, size, order, prob, out, reinterpret_cast<float*>(dsm + kOffSv),
-                        reinterpret_cast<int*>(dsm + kOffSelE),
-                        reinterpret_cast<float*>(dsm + kOffSelV));
-      else
-        mask_topk_warps(k, B, size, order, prob, out);
+      // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
+      // warp t mod 8): size, then the members in sorted order
+      for (int i = tid; i < B * (size + 1); i += 256) {
+        const int tt = t0 + i / (size + 1), c = i % (size + 1);
+        st_peer_u32(peer_addr(sCore + (tt & 7) * (1 + kMaxExperts) + c, (uint32_t)(tt >> 3)),
+                    (uint32_t)(c == 0 ? size : order[c - 1]));
+      }
       __syncthreads();
+    }
+    CT_AT(12);
+    cluster_sync();
+    {
+      const int t = 8 * (int)rank + warp;
+      if (t < T) {
+        const int* core = sCore + warp * (1 + kMaxExperts);
+        const int size = core[0];
+        const float* prow = sP + warp * kMaxExperts;
+        int my_e = -1;
+        float my_v = 0.f;
+        if (size <= 32) {
+          // one member per lane: k rounds of a tournament (larger score, ties to lower id)
+          const int e = lane < size ? core[1 + lane] : -1;
+          uint32_t key = e >= 0 ? order_key(prow[e]) : 0u;
+          for (int r = 0; r < k; ++r) {
+            const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+            const uint32_t imin =
+                __reduce_min_sync(0xffffffffu, key == kmax ? (uint32_t)e : 0xffffffffu);
+            if (lane == r) {
+              my_e = (int)imin;
+              my_v = key_value(kmax);
+            }
+            if (key == kmax && (uint32_t)e == imin) key = 0u;
+          }
+        } else {
+          float cv[8];
+          int ce[8];
+          uint32_t valid = 0;
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const int c = lane + 32 * j;
+            ce[j] = c < size ? core[1 + c] : 0;
+            if (c < size) valid |= 1u << j;
+            cv[j] = c < size ? prow[ce[j]] : 0.f;
+          }
+          warp_topk(cv, ce, valid, k, my_e, my_v);
+        }
+        float g = 0.f;
+        for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
+        if (lane < k) {
+          a.topk_idx[(size_t)t * k + lane] = my_e;
+          a.topk_gate[(size_t)t * k + lane] = my_v / g;
+          st_peer_u32(peer_addr(&sIdx[t * k + lane], 0), (uint32_t)my_e);
+        }
+      }
     }
   } else if (rank == 0) {
     if (a.coreset != nullptr)
@@ -382,8 +480,8 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   // ---- 5. dispatch
   if (rank == 0) {
     if (f.dsp.n_unique != nullptr)
-      dispatch_cta(sIdx, T, E, k, f.dsp.n_unique, f.dsp.unique_ids, f.dsp.offsets, f.dsp.rows,
-                   f.dsp.pos, f.dsp.err, s_bits, s_base);
+      dispatch_small_cta(sIdx, T, E, k, f.dsp.n_unique, f.dsp.unique_ids, f.dsp.offsets,
+                         f.dsp.rows, f.dsp.pos, f.dsp.err);
     if (tid == 0) *f.ticket = 0;  // ready for the next call
     CT_AT(7);
   }
@@ -423,7 +521,7 @@ extern "C" int dmoe_debug_ctrace(void* host) {
 }
 DMOE_KLOG_EXPORT(dmoe_debug_klog_router)
 extern "C" int dmoe_debug_ctrace_clear() {
-  static uint64_t zeros[64 * 8 * 32];
+  static uint64_t zeros[64 * 8 * 64];
   return (int)cudaMemcpyToSymbol(g_ctrace, zeros, sizeof(g_ctrace));
 }
 #endif

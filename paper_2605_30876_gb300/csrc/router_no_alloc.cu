@@ -64,8 +64,8 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
     return DMOE_ERR_INVALID_ARG;
 
   // The router uses the leading regions of the workspace plan: the fault record, the stage
-  // counters, the partial logits, the scores and the masked scores; the next region starts
-  // at tk_idx.
+  // counters, the partial logits, the scores, the masked scores and the top-k candidates;
+  // the next region starts at tk_idx.
   const Workspace plan = plan_workspace(*desc);
   const size_t need = plan.tk_idx;
   if (need > kRouterStaticScratchBytes) {
@@ -99,6 +99,7 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
   a.probs = probs != nullptr ? probs : reinterpret_cast<float*>(base + plan.probs);
   a.probs_requested = probs != nullptr;
   a.probs_hat = reinterpret_cast<float*>(base + plan.probs_hat);
+  a.cand = reinterpret_cast<uint2*>(base + plan.cand);
   a.topk_idx = topk_idx;
   a.topk_gate = topk_gate;
   a.coreset = coreset;

@@ -3,6 +3,10 @@
 // and Algorithm 1 for one diffusion block by one CTA of 256 threads.
 #pragma once
 
+#ifndef DMOE_STAMP
+#define DMOE_STAMP(st) ((void)0)
+#endif
+
 #include <math.h>
 
 #include "block_reduce.cuh"
@@ -90,23 +94,24 @@ __device__ __forceinline__ void warp_topk(const float (&v)[8], const int (&id)[8
 }
 
 // Softmax over one token's experts held by a warp (lane holds experts lane + 32j; invalid
-// slots are -inf on entry and 0 on exit): exp(v - max) / sum, fp32, the sum in a fixed order.
+// slots are -inf on entry and 0 on exit): exp(v - max) * (1 / sum), fp32, the sum in a fixed
+// order (exp by the hardware exponential: a few ulp, far inside the routing tolerance).
 __device__ __forceinline__ void warp_softmax8(float (&v)[kMaxExperts / 32], uint32_t valid) {
   constexpr int J = kMaxExperts / 32;
-  uint32_t mk = 0;
+  float mx = -INFINITY;
 #pragma unroll
   for (int j = 0; j < J; ++j)
-    if ((valid >> j) & 1u) mk = max(mk, order_key(v[j]));
-  const float m = key_value(__reduce_max_sync(0xffffffffu, mk));
+    if ((valid >> j) & 1u) mx = fmaxf(mx, v[j]);
+  const float m = key_value(__reduce_max_sync(0xffffffffu, order_key(mx)));
   float sum = 0.f;
 #pragma unroll
   for (int j = 0; j < J; ++j) {
-    v[j] = ((valid >> j) & 1u) ? expf(v[j] - m) : 0.f;
+    v[j] = ((valid >> j) & 1u) ? __expf(v[j] - m) : 0.f;
     sum += v[j];
   }
-  sum = warp_sum(sum);
+  const float inv = 1.f / warp_sum(sum);
 #pragma unroll
-  for (int j = 0; j < J; ++j) v[j] = v[j] / sum;
+  for (int j = 0; j < J; ++j) v[j] *= inv;
 }
 
 // Router scores and top-k of one token by one warp (E <= 256; lane holds experts lane + 32j).
@@ -179,14 +184,21 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 // Aggregate, Normalize, Sort, Top-P and the k floor (thread = expert). Leaves the coreset in
 // order[0, size) (S~ descending, ties to the lower id) and returns size; writes the coreset
 // outputs when given. `order` is a shared array of kMaxExperts entries.
+//
+// The sort is by ranks: every nonzero S~ counts the nonzero entries that beat it (larger, or
+// equal with a lower id), all in parallel; the zero entries follow in id order. Top-P then
+// accumulates the sorted values in order in fp32 (one thread) and stops at the first running
+// sum >= p (p >= 1: at the last nonzero entry); the floor extends the coreset to k entries.
 template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
                                           int32_t* __restrict__ coreset_size) {
   __shared__ __align__(16) float st_s[kMaxExperts];
+  __shared__ uint2 nz_kid[kMaxExperts];   // nonzero entries: (order key, id), ids ascending
+  __shared__ int wcnt[2][8];
   __shared__ int s_size;
   __shared__ float fscr[32];
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool live = tid < E;
 
   // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k); eight rows are
@@ -204,44 +216,62 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
   }
   // Normalize: L1
   const float tot = block_sum(S, fscr);
+  DMOE_STAMP(19);
   const float st = live ? S / tot : 0.f;
-  if (live) st_s[tid] = st;
+  // compact the nonzero entries (and count the zero ones), in id order
+  const bool nz = live && st > 0.f;
+  const bool z = live && !nz;
+  const uint32_t bnz = __ballot_sync(0xffffffffu, nz), bz = __ballot_sync(0xffffffffu, z);
+  __syncthreads();   // wcnt and the lists are rewritten by a later block of the same CTA
+  if (lane == 0) {
+    wcnt[0][warp] = __popc(bnz);
+    wcnt[1][warp] = __popc(bz);
+  }
   __syncthreads();
-  // Sort + Top-P + floor by one warp: the experts are taken in sorted order (S~ descending,
-  // ties to the lower id) while the running fp32 sum is accumulated in that order; the
-  // p rule stops at the first running sum >= p (p >= 1: at the last nonzero entry), the
-  // floor then continues to k entries.
-  if (tid < 32) {
-    Cand8 c;
-    int nz = 0;
-#pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const int e = tid + 32 * j;
-      const bool ok = e < E;
-      const float x = ok ? st_s[e] : 0.f;
-      c.key[j] = ok ? order_key(x) : 0u;
-      c.id[j] = ok ? (uint32_t)e : 0xffffffffu;
-      nz += (ok && x > 0.f) ? 1 : 0;
+  int pnz = __popc(bnz & ((1u << lane) - 1u)), pz = __popc(bz & ((1u << lane) - 1u)), nnz = 0, nzero = 0;
+  for (int w = 0; w < (int)(blockDim.x >> 5); ++w) {
+    if (w < warp) {
+      pnz += wcnt[0][w];
+      pz += wcnt[1][w];
     }
-    const int nnz = __reduce_add_sync(0xffffffffu, nz);
-    cand_sort(c);
-    float cum = 0.f;
-    int m = (top_p >= 1.f) ? nnz : -1;
-    int cnt = 0;
-    for (;;) {
-      const int target = (m < 0) ? E : max(m, k);
-      if (cnt >= target) break;
-      uint32_t kmax, imin;
-      cand_pop(c, kmax, imin);
-      if (tid == 0) order[cnt] = (int)imin;
-      cum += key_value(kmax);
-      ++cnt;
-      if (m < 0 && (cum >= top_p || cnt >= nnz)) m = min(cnt, nnz);
+    nnz += wcnt[0][w];
+    nzero += wcnt[1][w];
+  }
+  if (nz) nz_kid[pnz] = make_uint2(order_key(st), (uint32_t)tid);
+  __syncthreads();
+  DMOE_STAMP(20);
+  // ranks of the nonzero entries -> sorted positions; zero entries after them by id
+  if (nz) {
+    const uint32_t key = order_key(st);
+    int r = 0;
+#pragma unroll 8
+    for (int j = 0; j < nnz; ++j) {
+      const uint2 kj = nz_kid[j];
+      r += (kj.x > key || (kj.x == key && kj.y < (uint32_t)tid)) ? 1 : 0;
     }
-    if (tid == 0) s_size = max(m, k);
+    order[r] = tid;
+    st_s[r] = st;
+  }
+  if (z) order[nnz + pz] = tid;
+  __syncthreads();
+  DMOE_STAMP(21);
+  if (tid == 0) {
+    int m = nnz;
+    if (top_p < 1.f) {
+      float cum = 0.f;
+      for (int r = 0; r < nnz; ++r) {
+        cum += st_s[r];
+        if (cum >= top_p) {
+          m = r + 1;
+          break;
+        }
+      }
+    }
+    s_size = max(m, k);
   }
   __syncthreads();
   const int size = s_size;
+  (void)nzero;
   if (coreset != nullptr && live) coreset[tid] = (tid < size) ? order[tid] : -1;
   if (coreset_size != nullptr && tid == 0) coreset_size[0] = size;
   return size;
@@ -301,6 +331,7 @@ __device__ inline void mask_topk_small(int k, int B, int size, const int* order,
     }
   }
   __syncthreads();
+  DMOE_STAMP(23);
   for (int pidx = tid; pidx < n; pidx += nthr) {
     const int i = pidx / size, c = pidx % size;
     const float* row = sv + i * 32;
@@ -317,6 +348,7 @@ __device__ inline void mask_topk_small(int k, int B, int size, const int* order,
     }
   }
   __syncthreads();
+  DMOE_STAMP(24);
   for (int pidx = tid; pidx < B * k; pidx += nthr) {
     const int i = pidx / k, r = pidx % k;
     float g = 0.f;
