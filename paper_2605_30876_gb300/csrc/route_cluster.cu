@@ -58,8 +58,9 @@ constexpr int kClExp = 32;             // experts per cluster
 constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
 constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
 constexpr int kClMaxCand = (kMaxExperts / kClExp) * kMaxTopK;   // candidates of one token
-static_assert(kClMaxTok * kClMaxDChunk * 2 >= 4 * kClMaxTok * kClExp * 4,
-              "the quarter sums must fit where the bf16 x slice was");
+static_assert(kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2 >=
+                  8 * kClMaxTok * kClExp * 4,
+              "the eighth sums must fit where the W_r and x slices were");
 
 
 
@@ -112,40 +113,58 @@ constexpr int kOffHat = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2
 static_assert(kOffCore + 8 * (1 + kMaxExperts) * 4 <= kClMaxDChunk * kClExp * 4,
               "the routing scratch must fit where the W_r slice was");
 
-// Partial logits of the CTA's d slice: thread (q, eg, tg) accumulates experts 4eg..4eg+3 of
-// tokens tg*TPT .. tg*TPT+TPT-1 over d in the q-th quarter of the slice and stores them to
-// red[q][t][e] (fp32, [4][kClMaxTok][32]); Ws [DC][32], Xf [T][xs] fp32 in shared memory.
+// Partial logits of the CTA's d slice: warp w takes the w-th eighth of the slice; lane
+// (tg = lane / 4, eg = lane % 4) accumulates experts 8eg .. 8eg+7 of tokens tg, tg+8, ...
+// (TPT of them) over that eighth, d ascending, four d at a time (one 16-B load of x per
+// token and two of W_r per d), and stores them to red[w][t][e] ([8][kClMaxTok][32] fp32).
+// Ws [DC][32] and Xf [T][xs] are fp32 in shared memory, xs = DC + 4 (16-B rows, and rows
+// tg + 8i fall in distinct banks).
 template <int TPT>
 __device__ __forceinline__ void logits_partial(const float* Ws, const float* Xf, int xs, int DC,
-                                               int T, float* red, int tid) {
-  const int q = tid >> 6, r = tid & 63, eg = r & 7, tg = r >> 3;
-  const int dq = DC / 4, d0 = q * dq;
-  float acc[TPT][4];
+                                               int T, float* red, int warp, int lane) {
+  const int eg = lane & 3, tg = lane >> 2;
+  const int de = DC / 8, d0 = warp * de;
+  float acc[TPT][8];
 #pragma unroll
   for (int i = 0; i < TPT; ++i)
 #pragma unroll
-    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
-  int trow[TPT];
+    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
+  const float* xr[TPT];
 #pragma unroll
-  for (int i = 0; i < TPT; ++i) trow[i] = min(tg * TPT + i, T - 1) * xs;  // clamp: rows >= T unused
-#pragma unroll 4
-  for (int dd = d0; dd < d0 + dq; ++dd) {
-    const float4 w = *reinterpret_cast<const float4*>(Ws + dd * kClExp + eg * 4);
+  for (int i = 0; i < TPT; ++i) xr[i] = Xf + min(tg + 8 * i, T - 1) * xs;  // rows >= T unused
+  const float* wr = Ws + eg * 8;
+#pragma unroll 2
+  for (int dd = d0; dd < d0 + de; dd += 4) {
+    float4 xv[TPT];
 #pragma unroll
-    for (int i = 0; i < TPT; ++i) {
-      const float xv = Xf[trow[i] + dd];
-      acc[i][0] = fmaf(xv, w.x, acc[i][0]);
-      acc[i][1] = fmaf(xv, w.y, acc[i][1]);
-      acc[i][2] = fmaf(xv, w.z, acc[i][2]);
-      acc[i][3] = fmaf(xv, w.w, acc[i][3]);
+    for (int i = 0; i < TPT; ++i) xv[i] = *reinterpret_cast<const float4*>(xr[i] + dd);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const float4 wa = *reinterpret_cast<const float4*>(wr + (dd + u) * kClExp);
+      const float4 wb = *reinterpret_cast<const float4*>(wr + (dd + u) * kClExp + 4);
+#pragma unroll
+      for (int i = 0; i < TPT; ++i) {
+        const float x = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
+        acc[i][0] = fmaf(x, wa.x, acc[i][0]);
+        acc[i][1] = fmaf(x, wa.y, acc[i][1]);
+        acc[i][2] = fmaf(x, wa.z, acc[i][2]);
+        acc[i][3] = fmaf(x, wa.w, acc[i][3]);
+        acc[i][4] = fmaf(x, wb.x, acc[i][4]);
+        acc[i][5] = fmaf(x, wb.y, acc[i][5]);
+        acc[i][6] = fmaf(x, wb.z, acc[i][6]);
+        acc[i][7] = fmaf(x, wb.w, acc[i][7]);
+      }
     }
   }
+  __syncthreads();   // every warp is done with W_r: red overwrites it
 #pragma unroll
   for (int i = 0; i < TPT; ++i) {
-    const int t = tg * TPT + i;
-    if (t < T)
-      *reinterpret_cast<float4*>(red + ((size_t)q * kClMaxTok + t) * kClExp + eg * 4) =
-          make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+    const int t = tg + 8 * i;
+    if (t < T) {
+      float* dst = red + ((size_t)warp * kClMaxTok + t) * kClExp + eg * 8;
+      *reinterpret_cast<float4*>(dst) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
+      *reinterpret_cast<float4*>(dst + 4) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
+    }
   }
 }
 
@@ -220,35 +239,33 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     }
   }
   CT_AT(1);
-  // x slice to fp32, rows padded by one float against bank conflicts
+  // x slice to fp32 in rows of DC + 4 floats (16-B aligned; see logits_partial)
   float* Xf = reinterpret_cast<float*>(dsm + kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2);
-  const int xs = DC + 1;
-  {
-    // warp per row, lanes on consecutive bf16 pairs: conflict-free loads, 2-way stores
-    const int DC2 = DC / 2;
-    const __nv_bfloat162* X2 = reinterpret_cast<const __nv_bfloat162*>(Xs);
-    for (int t = warp; t < T; t += 8)
-      for (int c2 = lane; c2 < DC2; c2 += 32) {
-        const __nv_bfloat162 v2 = X2[t * DC2 + c2];
-        float* dst = Xf + t * xs + 2 * c2;
-        dst[0] = __low2float(v2);
-        dst[1] = __high2float(v2);
-      }
-  }
+  const int xs = DC + 4;
+  for (int t = warp; t < T; t += 8)
+    for (int c8 = lane; c8 < DC / 8; c8 += 32) {
+      const uint4 raw = *reinterpret_cast<const uint4*>(Xs + t * DC + c8 * 8);
+      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
+      float4* dst = reinterpret_cast<float4*>(Xf + t * xs + c8 * 8);
+      dst[0] = make_float4(__low2float(p2[0]), __high2float(p2[0]), __low2float(p2[1]),
+                           __high2float(p2[1]));
+      dst[1] = make_float4(__low2float(p2[2]), __high2float(p2[2]), __low2float(p2[3]),
+                           __high2float(p2[3]));
+    }
   __syncthreads();
   CT_AT(8);
-  // register-blocked FFMA: thread = (d quarter q, expert quad eg, token group tg);
-  // 4 experts x TPT tokens per thread, d ascending within the quarter
-  // the four quarter sums go where the bf16 x slice was (dead after the conversion)
-  float* red4 = reinterpret_cast<float*>(Xs);
-  if (T <= 32) logits_partial<4>(Ws, Xf, xs, DC, T, red4, tid);
-  else logits_partial<8>(Ws, Xf, xs, DC, T, red4, tid);
+  // register-blocked FFMA over eighths of the slice; the eighth sums go where the W_r and x
+  // slices were (logits_partial synchronises the CTA before it stores them)
+  float* red8 = reinterpret_cast<float*>(dsm);
+  if (T <= 32) logits_partial<4>(Ws, Xf, xs, DC, T, red8, warp, lane);
+  else logits_partial<8>(Ws, Xf, xs, DC, T, red8, warp, lane);
   __syncthreads();
-  // add the four d quarters in order
+  // add the eight partial sums in order
   for (int i = tid; i < T * kClExp; i += 256) {
-    const float* red = red4 + i;
-    s_part[i] = ((red[0] + red[kClMaxTok * kClExp]) + red[2 * kClMaxTok * kClExp]) +
-                red[3 * kClMaxTok * kClExp];
+    float v = 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) v += red8[q * kClMaxTok * kClExp + i];
+    s_part[i] = v;
   }
   {  // TopKMask rows start as zeros (scoring warps anywhere in the cluster add the winners)
     float4* hz = reinterpret_cast<float4*>(dsm + kOffHat);
@@ -508,7 +525,7 @@ EncodeTiledFnC encoder() {
 
 size_t route_cluster_smem() {
   const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2 +
-                        (size_t)kClMaxTok * (kClMaxDChunk + 1) * 4;
+                        (size_t)kClMaxTok * (kClMaxDChunk + 4) * 4;
   const size_t stage4 = (size_t)2 * 8 * kMaxExperts * 4 + (size_t)kClMaxTok * kMaxTopK * 4;
   return (stage1 > stage4 ? stage1 : stage4) + 128;
 }
@@ -527,7 +544,8 @@ extern "C" int dmoe_debug_ctrace_clear() {
 #endif
 
 bool route_cluster_ok(int T, int d, int E) {
-  return T <= kClMaxTok && d % (kCl * 8) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
+  // d % 256: each CTA's slice splits into eight runs of whole float4 groups
+  return T <= kClMaxTok && d % (kCl * 32) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
 }
 
 cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
