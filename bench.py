@@ -514,7 +514,7 @@ def main():
         "e2e": None if secs_e2e is None else {"value": tokens_total / secs_e2e, "unit": UNIT,
                 "h2d_bytes_per_step": T * shape.d_model * 2,
                 "d2h_bytes_per_step": T * shape.d_model * 2},
-        "gpu_launches": args.steps * 7,
+        "gpu_launches": args.steps * dm.dmoe_layer_forward_launches(arm.layers[0].desc),
         "flops_per_forward": layer_flops(shape),
         "clocks": clocks,
     }

@@ -148,6 +148,11 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x,
                                int32_t* n_unique, int32_t* unique_ids,
                                void* workspace, size_t workspace_bytes, void* stream);
 
+/* Number of kernel launches one dmoe_layer_forward call makes for `desc` (the decode-size
+ * path: routing 1, experts 1, combine 1). Returns -1 for an invalid or unsupported desc.
+ * Host-only, no GPU needed. */
+int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc);
+
 /* Kernels of the forward, for dmoe_set_profile_events. */
 typedef enum {
   DMOE_KERNEL_ROUTER = 0,     /* router logits, softmax/top-k and Algorithm 1 kernels */

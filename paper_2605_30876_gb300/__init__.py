@@ -18,6 +18,7 @@ __all__ = [
     "DMOE_ROUTE_TOKEN", "DMOE_ROUTE_BLOCK", "DmoeError", "LayerDesc", "make_desc",
     "dmoe_workspace_size", "dmoe_router", "dmoe_dispatch", "dmoe_moe_forward",
     "dmoe_layer_forward", "dmoe_get_device_error", "dmoe_status_string", "dmoe_abi_version",
+    "dmoe_layer_forward_launches",
     "alloc_workspace", "LIB_PATH", "dmoe_set_profile_events", "KERNELS",
 ]
 
@@ -86,6 +87,8 @@ def _load() -> ctypes.CDLL:
     lib.dmoe_last_error_message.restype = ctypes.c_char_p
     lib.dmoe_abi_version.argtypes = []
     lib.dmoe_abi_version.restype = ctypes.c_int32
+    lib.dmoe_layer_forward_launches.argtypes = [ctypes.POINTER(LayerDesc)]
+    lib.dmoe_layer_forward_launches.restype = ctypes.c_int32
     lib.dmoe_set_profile_events.argtypes = [ctypes.c_int32, P, P]
     lib.dmoe_set_profile_events.restype = st
     return lib
@@ -219,3 +222,8 @@ def dmoe_status_string(status: int) -> str:
 
 def dmoe_abi_version() -> int:
     return _lib.dmoe_abi_version()
+
+
+def dmoe_layer_forward_launches(desc) -> int:
+    """Kernel launches of one dmoe_layer_forward call for `desc` (-1: invalid desc)."""
+    return _lib.dmoe_layer_forward_launches(ctypes.byref(desc))

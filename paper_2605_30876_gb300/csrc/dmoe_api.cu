@@ -405,4 +405,22 @@ const char* dmoe_last_error_message(void) { return g_last_error; }
 
 int32_t dmoe_abi_version(void) { return DMOE_ABI_VERSION; }
 
+int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc) {
+  if (check_desc(desc) != DMOE_OK) return -1;
+  const int T = desc->n_blocks * desc->block_size;
+  int n = 0;
+  if (route_cluster_ok(T, desc->d_model, desc->n_experts)) {
+    n += 1;                                                   // routing with the dispatch
+  } else {
+    n += 2;                                                   // logits, softmax / top-k
+    n += desc->mode == DMOE_ROUTE_BLOCK ? 1 : 0;              // Algorithm 1
+    n += 1;                                                   // dispatch
+  }
+  if (experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared))
+    n += 2;                                                   // experts, combine
+  else
+    n += 3;                                                   // gather, experts, combine
+  return n;
+}
+
 }  // extern "C"
