@@ -268,12 +268,12 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
     return secs, kern, clocks
 
 
-def traffic_from_profile(kernel: str):
+def traffic_from_profile(kernel: str, source: str):
     """dram bytes per launch from the committed ncu summary, if it was taken on the current
     source of the kernel (matching source hash); else None."""
     import hashlib
     path = os.path.join(ROOT, "profiles", f"{kernel}_layer_block.txt")
-    src = os.path.join(ROOT, "paper_2605_30876_gb300", "csrc", "expert_ffn.cu")
+    src = os.path.join(ROOT, "paper_2605_30876_gb300", "csrc", source)
     try:
         h = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
         vals = {}
@@ -504,9 +504,9 @@ def main():
                            "frac_measured_hbm": lbytes / (ms_per_step * 1e-3) / 1e9 / hbm,
                            "frac_nominal_8tbs": lbytes / (ms_per_step * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
                            "peak_source": peak_src},
-        "roofline": {"kernel": "moe_experts", "bound": "hbm", "achieved": achieved, "peak": hbm,
-                     "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
-                     "traffic": traffic_from_profile("moe_experts"),
+        "roofline": {"kernel": "moe_decode_kernel", "bound": "hbm", "achieved": achieved,
+                     "peak": hbm, "unit": "GB/s", "frac": (achieved / hbm) if achieved else None,
+                     "traffic": traffic_from_profile("moe_decode", "expert_decode.cu"),
                      "algorithmic_bytes_per_launch": gbytes,
                      "launch_us": kern_s * 1e6 if kern_s else None,
                      "peak_source": f"{peak_src} hbm_gbs"},
