@@ -110,7 +110,20 @@ __device__ __forceinline__ int ld_acquire(const int32_t* p) {
   asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
   return v;
 }
-__device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
+// silu with the fast divide: H is rounded to bf16 right after
+__device__ __forceinline__ float silu_f(float z) { return __fdividef(z, 1.f + __expf(-z)); }
+// 2-D tiled bulk store of a shared-memory box to global memory, tracked by a bulk group
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void* src, int32_t x,
+                                             int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+          reinterpret_cast<uint64_t>(map)),
+      "r"(ptx::smem_addr(src)), "r"(x), "r"(y)
+      : "memory");
+}
+__device__ __forceinline__ void bulk_commit_wait_all() {
+  asm volatile("cp.async.bulk.commit_group;\n\tcp.async.bulk.wait_group 0;" ::: "memory");
+}
 
 // AND of `v` over the 128 epilogue threads (named barrier 1), so that warp-collective TMEM
 // loads are taken by all of them or by none.
@@ -436,7 +449,9 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (!ok) break;
       ptx::tc_fence_after();
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
-      __nv_bfloat16* hg = p.hdense + (size_t)gi * p.n_pad * p.imax + m * 64 + r64;
+      // the H tile (n_pad token rows x 64 columns, bf16) is laid out in the staging tile
+      // exactly as the 128-byte-swizzled box of the H tensor map, then stored by TMA
+      uint8_t* hbox = reinterpret_cast<uint8_t*>(stage_t);
       for (int c0 = 0; c0 < n_mma; c0 += 16) {
         float v[16];
         ptx::tmem_ld16(tbase + c0, v);
@@ -449,21 +464,30 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
         named_bar_sync(2, 128);
         if (is_gate) {
 #pragma unroll
-          for (int c = 0; c < 16; ++c)
-            hg[(size_t)(c0 + c) * p.imax] = __float2bfloat16(silu_f(v[c]) * buf[r64 * kXStride + c]);
+          for (int c = 0; c < 16; ++c) {
+            const int t = c0 + c;
+            *reinterpret_cast<__nv_bfloat16*>(hbox + t * 128 + (((r64 >> 3) ^ (t & 7)) << 4) +
+                                              (r64 & 7) * 2) =
+                __float2bfloat16(silu_f(v[c]) * buf[r64 * kXStride + c]);
+          }
         }
         xb ^= 1;
       }
       ptx::tc_fence_before();
       ptx::mbar_arrive(&acc_empty[acc]);
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
-      // publish the tile: the barrier orders every epilogue thread's H stores before one
-      // release add; a reader acquires the counter, then fences the async proxy
+      // publish the tile: one bulk store of the box, waited to completion, then one release
+      // add; a reader acquires the counter, then fences the async proxy
+      ptx::fence_proxy_async_smem();
       named_bar_sync(2, 128);
       if (et == 0) {
+        tma_store_2d(&tm.h, hbox, m * 64, gi * p.n_pad);
+        bulk_commit_wait_all();
+        fence_proxy_async_global();
         red_release_add(p.h_ready + gi, 1);
         if (first) ED_AT(4);
       }
+      named_bar_sync(2, 128);   // the box is rewritten by the next tile
       first = false;
     }
     first = true;
@@ -497,6 +521,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
           for (int c = 0; c < 16; ++c) srow[c0 + c] = vv[c];
         }
         float* out = p.yslot + (size_t)g.row0 * p.d + drow;
+#pragma unroll 8
         for (int r = 0; r < g.n; ++r) {
           const int t = tok[r];
           if (t >= 0 && t < p.T) out[(size_t)r * p.d] = srow[t];

@@ -588,7 +588,9 @@ cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, i
     if (dev < 31) mask |= 1 << dev;
   }
   dim3 grid(kCl, (a.E + kClExp - 1) / kClExp);
-  return launch_cluster(route_cluster_kernel, grid, dim3(256), smem, s, kCl, f);
+  // programmatic dependent launch: the set-up overlaps the previous kernel on the stream;
+  // the kernel waits for it (griddepcontrol.wait) before it reads anything
+  return launch_cluster(route_cluster_kernel, grid, dim3(256), smem, s, kCl, true, f);
 }
 
 }  // namespace dmoe
