@@ -58,15 +58,12 @@ constexpr int kClExp = 32;             // experts per cluster
 constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
 constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
 constexpr int kClMaxCand = (kMaxExperts / kClExp) * kMaxTopK;   // candidates of one token
-static_assert(kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2 >=
-                  8 * kClMaxTok * kClExp * 4,
-              "the eighth sums must fit where the W_r and x slices were");
 
 
 
 struct ClusterArgs {
   CUtensorMap wmap;   // W_r [d, E] fp32, box 32 experts x d/8 rows
-  CUtensorMap xmap;   // x [T, d] bf16, box d/8 columns x T rows
+  CUtensorMap xmap;   // x [T, d] bf16, box 64 columns x round16(T) rows, 128-B swizzle
   RouterArgs r;
   DispatchArgs dsp;   // dsp.n_unique == nullptr: no dispatch
   int32_t* ticket;    // zero between calls
@@ -110,68 +107,28 @@ constexpr int kOffP = 0;                                      // f32 [8][kMaxExp
 constexpr int kOffIdx = kOffP + 8 * kMaxExperts * 4;          // i32 [kClMaxTok * kMaxTopK]
 constexpr int kOffCore = kOffIdx + kClMaxTok * kMaxTopK * 4;  // i32 [8][1 + kMaxExperts]
 constexpr int kOffHat = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;  // f32 [kClMaxTok][kMaxExperts]
+// logits phase: the three bf16 parts of the W_r slice, [3][32 experts][kWtStride bytes]
+constexpr int kOffWt = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;
 static_assert(kOffCore + 8 * (1 + kMaxExperts) * 4 <= kClMaxDChunk * kClExp * 4,
               "the routing scratch must fit where the W_r slice was");
 
-// Partial logits of the CTA's d slice: warp w takes the w-th eighth of the slice; lane
-// (tg = lane / 4, eg = lane % 4) accumulates experts 8eg .. 8eg+7 of tokens tg, tg+8, ...
-// (TPT of them) over that eighth, d ascending, four d at a time (one 16-B load of x per
-// token and two of W_r per d), and stores them to red[w][t][e] ([8][kClMaxTok][32] fp32).
-// Ws [DC][32] and Xf [T][xs] are fp32 in shared memory, xs = DC + 4 (16-B rows, and rows
-// tg + 8i fall in distinct banks).
-template <int TPT>
-__device__ __forceinline__ void logits_partial(const float* Ws, const float* Xf, int xs, int DC,
-                                               int T, float* red, int warp, int lane) {
-  const int eg = lane & 3, tg = lane >> 2;
-  const int de = DC / 8, d0 = warp * de;
-  float acc[TPT][8];
-#pragma unroll
-  for (int i = 0; i < TPT; ++i)
-#pragma unroll
-    for (int j = 0; j < 8; ++j) acc[i][j] = 0.f;
-  const float* xr[TPT];
-#pragma unroll
-  for (int i = 0; i < TPT; ++i) xr[i] = Xf + min(tg + 8 * i, T - 1) * xs;  // rows >= T unused
-  const float* wr = Ws + eg * 8;
-#pragma unroll 2
-  for (int dd = d0; dd < d0 + de; dd += 4) {
-    float4 xv[TPT];
-#pragma unroll
-    for (int i = 0; i < TPT; ++i) xv[i] = *reinterpret_cast<const float4*>(xr[i] + dd);
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      const float4 wa = *reinterpret_cast<const float4*>(wr + (dd + u) * kClExp);
-      const float4 wb = *reinterpret_cast<const float4*>(wr + (dd + u) * kClExp + 4);
-#pragma unroll
-      for (int i = 0; i < TPT; ++i) {
-        const float x = u == 0 ? xv[i].x : u == 1 ? xv[i].y : u == 2 ? xv[i].z : xv[i].w;
-        acc[i][0] = fmaf(x, wa.x, acc[i][0]);
-        acc[i][1] = fmaf(x, wa.y, acc[i][1]);
-        acc[i][2] = fmaf(x, wa.z, acc[i][2]);
-        acc[i][3] = fmaf(x, wa.w, acc[i][3]);
-        acc[i][4] = fmaf(x, wb.x, acc[i][4]);
-        acc[i][5] = fmaf(x, wb.y, acc[i][5]);
-        acc[i][6] = fmaf(x, wb.z, acc[i][6]);
-        acc[i][7] = fmaf(x, wb.w, acc[i][7]);
-      }
-    }
-  }
-  __syncthreads();   // every warp is done with W_r: red overwrites it
-#pragma unroll
-  for (int i = 0; i < TPT; ++i) {
-    const int t = tg + 8 * i;
-    if (t < T) {
-      float* dst = red + ((size_t)warp * kClMaxTok + t) * kClExp + eg * 8;
-      *reinterpret_cast<float4*>(dst) = make_float4(acc[i][0], acc[i][1], acc[i][2], acc[i][3]);
-      *reinterpret_cast<float4*>(dst + 4) = make_float4(acc[i][4], acc[i][5], acc[i][6], acc[i][7]);
-    }
-  }
+constexpr int kWtStride = kClMaxDChunk * 2 + 16;   // bytes per expert row of a W_r part
+
+// bf16 tensor-core product D[16 x 8] += A[16 x 16] B[16 x 8] (fp32 accumulators)
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
+                                               uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+      "{%8, %9}, {%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
 __global__ void __launch_bounds__(256, 1)
 route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
-  extern __shared__ __align__(128) uint8_t dsm_raw[];
-  uint8_t* dsm = dsm_raw + ((128u - (s_addr(dsm_raw) & 127u)) & 127u);
+  // 1024-B aligned: the swizzled x boxes take their swizzle phase from the address
+  extern __shared__ __align__(1024) uint8_t dsm_raw[];
+  uint8_t* dsm = dsm_raw + ((1024u - (s_addr(dsm_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ uint32_t s_last;
   __shared__ float s_part[kClMaxTok * kClExp];                     // partial logits [T][32]
@@ -192,13 +149,15 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 
   // ---- 1. partial logits over this CTA's slice of d
   float* Ws = reinterpret_cast<float*>(dsm);                                   // [DC][32]
-  __nv_bfloat16* Xs = reinterpret_cast<__nv_bfloat16*>(dsm + kClMaxDChunk * kClExp * 4);  // [T][DC]
+  // x slice: boxes of 64 columns x T16 rows with the 128-byte swizzle
+  uint8_t* Xs = dsm + kClMaxDChunk * kClExp * 4;
+  const int T16 = (T + 15) & ~15, nxb = (DC + 63) / 64;
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(s_addr(&s_bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.wmap)) : "memory");
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.xmap)) : "memory");
-    const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)T * DC * 2;
+    const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)nxb * T16 * 128;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_addr(&s_bar)),
                  "r"(bytes)
                  : "memory");
@@ -208,12 +167,13 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         "l"(reinterpret_cast<uint64_t>(&f.wmap)), "r"(s_addr(&s_bar)), "r"(e0),
         "r"((int)rank * DC)
         : "memory");
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Xs)),
-        "l"(reinterpret_cast<uint64_t>(&f.xmap)), "r"(s_addr(&s_bar)), "r"((int)rank * DC),
-        "r"(0)
-        : "memory");
+    for (int bx = 0; bx < nxb; ++bx)
+      asm volatile(
+          "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+          " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Xs) + (uint32_t)(bx * T16 * 128)),
+          "l"(reinterpret_cast<uint64_t>(&f.xmap)), "r"(s_addr(&s_bar)),
+          "r"((int)rank * DC + 64 * bx), "r"(0)
+          : "memory");
     issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
   }
   for (int e = tid; e < E; e += 256) s_bias[e] = a.bias != nullptr ? a.bias[e] : 0.f;
@@ -239,34 +199,64 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     }
   }
   CT_AT(1);
-  // x slice to fp32 in rows of DC + 4 floats (16-B aligned; see logits_partial)
-  float* Xf = reinterpret_cast<float*>(dsm + kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2);
-  const int xs = DC + 4;
-  for (int t = warp; t < T; t += 8)
-    for (int c8 = lane; c8 < DC / 8; c8 += 32) {
-      const uint4 raw = *reinterpret_cast<const uint4*>(Xs + t * DC + c8 * 8);
-      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-      float4* dst = reinterpret_cast<float4*>(Xf + t * xs + c8 * 8);
-      dst[0] = make_float4(__low2float(p2[0]), __high2float(p2[0]), __low2float(p2[1]),
-                           __high2float(p2[1]));
-      dst[1] = make_float4(__low2float(p2[2]), __high2float(p2[2]), __low2float(p2[3]),
-                           __high2float(p2[3]));
-    }
+  // W_r slice -> three bf16 parts (hi + mid + lo = w to 2^-27), transposed to
+  // [expert][d] rows of kWtStride bytes (the column-major B operand, padded against bank
+  // conflicts); x * part is exact in fp32, so the three products summed in fp32 give the
+  // fp32 logit
+  uint8_t* Wt = dsm + kOffWt;
+  for (int q = tid; q < kClExp * (DC / 2); q += 256) {
+    const int n = q % kClExp, kp = q / kClExp;
+    const float w0 = Ws[(2 * kp) * kClExp + n], w1 = Ws[(2 * kp + 1) * kClExp + n];
+    const __nv_bfloat16 h0 = __float2bfloat16_rn(w0), h1 = __float2bfloat16_rn(w1);
+    const float r0 = w0 - __bfloat162float(h0), r1 = w1 - __bfloat162float(h1);
+    const __nv_bfloat16 m0 = __float2bfloat16_rn(r0), m1 = __float2bfloat16_rn(r1);
+    const __nv_bfloat16 l0 = __float2bfloat16_rn(r0 - __bfloat162float(m0));
+    const __nv_bfloat16 l1 = __float2bfloat16_rn(r1 - __bfloat162float(m1));
+    uint8_t* row = Wt + n * kWtStride + kp * 4;
+    *reinterpret_cast<__nv_bfloat162*>(row) = __halves2bfloat162(h0, h1);
+    *reinterpret_cast<__nv_bfloat162*>(row + kClExp * kWtStride) = __halves2bfloat162(m0, m1);
+    *reinterpret_cast<__nv_bfloat162*>(row + 2 * kClExp * kWtStride) = __halves2bfloat162(l0, l1);
+  }
   __syncthreads();
   CT_AT(8);
-  // register-blocked FFMA over eighths of the slice; the eighth sums go where the W_r and x
-  // slices were (logits_partial synchronises the CTA before it stores them)
-  float* red8 = reinterpret_cast<float*>(dsm);
-  if (T <= 32) logits_partial<4>(Ws, Xf, xs, DC, T, red8, warp, lane);
-  else logits_partial<8>(Ws, Xf, xs, DC, T, red8, warp, lane);
-  __syncthreads();
-  // add the eight partial sums in order
-  for (int i = tid; i < T * kClExp; i += 256) {
-    float v = 0.f;
+  // tensor cores (mma.sync m16n8k16): warp tile = 16 tokens x 8 experts over the whole
+  // slice; per 16-wide K step the hi, mid and lo parts in that order
+  {
+    const int g = lane >> 2, tq = lane & 3;
+    const int ntile = (T16 / 16) * (kClExp / 8);
+    for (int tile = warp; tile < ntile; tile += 8) {
+      const int mt = tile / (kClExp / 8), nt = tile % (kClExp / 8);
+      const int r0 = mt * 16 + g;                   // A rows r0, r0 + 8 (same swizzle phase)
+      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      const uint8_t* brow = Wt + (nt * 8 + g) * kWtStride + tq * 4;
+      for (int k0 = 0; k0 < DC; k0 += 16) {
+        const int bx = k0 >> 6, c = (k0 & 63) >> 3;   // box, 16-B chunk of k0
+        const uint8_t* xb = Xs + bx * T16 * 128;
+        uint32_t af[4];
+        af[0] = *reinterpret_cast<const uint32_t*>(xb + r0 * 128 + ((c ^ (r0 & 7)) << 4) + tq * 4);
+        af[1] = *reinterpret_cast<const uint32_t*>(xb + (r0 + 8) * 128 + ((c ^ (r0 & 7)) << 4) + tq * 4);
+        af[2] = *reinterpret_cast<const uint32_t*>(xb + r0 * 128 + (((c + 1) ^ (r0 & 7)) << 4) + tq * 4);
+        af[3] = *reinterpret_cast<const uint32_t*>(xb + (r0 + 8) * 128 + (((c + 1) ^ (r0 & 7)) << 4) + tq * 4);
 #pragma unroll
-    for (int q = 0; q < 8; ++q) v += red8[q * kClMaxTok * kClExp + i];
-    s_part[i] = v;
+        for (int part = 0; part < 3; ++part) {
+          const uint8_t* bp = brow + part * kClExp * kWtStride + k0 * 2;
+          mma_bf16_16816(acc, af, *reinterpret_cast<const uint32_t*>(bp),
+                         *reinterpret_cast<const uint32_t*>(bp + 16));
+        }
+      }
+      // D rows r0, r0 + 8; columns 2tq, 2tq + 1 of the tile
+      const int e = nt * 8 + 2 * tq;
+      if (r0 < T) {
+        s_part[r0 * kClExp + e] = acc[0];
+        s_part[r0 * kClExp + e + 1] = acc[1];
+      }
+      if (r0 + 8 < T) {
+        s_part[(r0 + 8) * kClExp + e] = acc[2];
+        s_part[(r0 + 8) * kClExp + e + 1] = acc[3];
+      }
+    }
   }
+  __syncthreads();
   {  // TopKMask rows start as zeros (scoring warps anywhere in the cluster add the winners)
     float4* hz = reinterpret_cast<float4*>(dsm + kOffHat);
     for (int i = tid; i < T * (kMaxExperts / 4); i += 256) hz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
@@ -524,10 +514,9 @@ EncodeTiledFnC encoder() {
 }
 
 size_t route_cluster_smem() {
-  const size_t stage1 = (size_t)kClMaxDChunk * kClExp * 4 + (size_t)kClMaxTok * kClMaxDChunk * 2 +
-                        (size_t)kClMaxTok * (kClMaxDChunk + 4) * 4;
-  const size_t stage4 = (size_t)2 * 8 * kMaxExperts * 4 + (size_t)kClMaxTok * kMaxTopK * 4;
-  return (stage1 > stage4 ? stage1 : stage4) + 128;
+  const size_t stage1 = (size_t)kOffWt + 3 * (size_t)kClExp * (kClMaxDChunk * 2 + 16);
+  const size_t stage4 = (size_t)kOffHat + (size_t)kClMaxTok * kMaxExperts * 4;
+  return (stage1 > stage4 ? stage1 : stage4) + 1024;
 }
 
 }  // namespace
@@ -567,10 +556,10 @@ cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, i
   {
     const cuuint64_t dims[2] = {(cuuint64_t)a.d, (cuuint64_t)a.T};
     const cuuint64_t strides[1] = {(cuuint64_t)a.d * 2};
-    const cuuint32_t box[2] = {(cuuint32_t)DC, (cuuint32_t)a.T};
+    const cuuint32_t box[2] = {64u, (cuuint32_t)((a.T + 15) & ~15)};
     const cuuint32_t estr[2] = {1, 1};
     if (enc(&f.xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(a.x), dims,
-            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
