@@ -185,10 +185,11 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 // order[0, size) (S~ descending, ties to the lower id) and returns size; writes the coreset
 // outputs when given. `order` is a shared array of kMaxExperts entries.
 //
-// The sort is by ranks: every nonzero S~ counts the nonzero entries that beat it (larger, or
-// equal with a lower id), all in parallel; the zero entries follow in id order. Top-P then
-// accumulates the sorted values in order in fp32 (one thread) and stops at the first running
-// sum >= p (p >= 1: at the last nonzero entry); the floor extends the coreset to k entries.
+// Top-P accumulates the sorted values in order in fp32 and stops at the first running sum
+// >= p (p >= 1: at the last nonzero entry); the floor extends the coreset to k entries
+// (zero entries in id order). For p < 1 one warp takes the entries in sorted order by a
+// tournament until both rules are met; for p >= 1 every nonzero S~ counts the nonzero
+// entries that beat it (larger, or equal with a lower id), all in parallel.
 template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
@@ -218,6 +219,61 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
   const float tot = block_sum(S, fscr);
   DMOE_STAMP(19);
   const float st = live ? S / tot : 0.f;
+  if (top_p < 1.f) {
+    // p < 1: the coreset is a short sorted prefix. Warp 0 takes the entries in sorted order
+    // by a tournament (lane l holds experts l + 32j and its best remaining one; each round
+    // the warp's best by two single-instruction reductions) and keeps the running sum.
+    if (live) st_s[tid] = st;
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t key[8];
+      int nz = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int e = lane + 32 * j;
+        const float x = e < E ? st_s[e] : 0.f;
+        key[j] = e < E ? order_key(x) : 0u;
+        nz += (e < E && x > 0.f) ? 1 : 0;
+      }
+      const int nnz = __reduce_add_sync(0xffffffffu, nz);
+      uint32_t bk = 0u;
+      int bj = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if (key[j] > bk) { bk = key[j]; bj = j; }   // ties: the lower id (lower j) stays
+      float cum = 0.f;
+      int m = -1, cnt = 0;
+      for (;;) {
+        const int target = (m < 0) ? E : max(m, k);
+        if (cnt >= target) break;
+        const uint32_t kmax = __reduce_max_sync(0xffffffffu, bk);
+        const uint32_t imin =
+            __reduce_min_sync(0xffffffffu, bk == kmax ? (uint32_t)(lane + 32 * bj) : 0xffffffffu);
+        if (lane == 0) order[cnt] = (int)imin;
+        cum += key_value(kmax);
+        ++cnt;
+        if (m < 0 && (cum >= top_p || cnt >= nnz)) m = min(cnt, nnz);
+        if (bk == kmax && (uint32_t)(lane + 32 * bj) == imin) {
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (j == bj) key[j] = 0u;
+          bk = 0u;
+          bj = 0;
+#pragma unroll
+          for (int j = 0; j < 8; ++j)
+            if (key[j] > bk) { bk = key[j]; bj = j; }
+        }
+      }
+      if (lane == 0) s_size = max(m, k);
+    }
+    __syncthreads();
+    const int size = s_size;
+    if (coreset != nullptr && live) coreset[tid] = (tid < size) ? order[tid] : -1;
+    if (coreset_size != nullptr && tid == 0) coreset_size[0] = size;
+    __syncthreads();   // st_s and order are rewritten by a later block of the same CTA
+    return size;
+  }
+  // p >= 1: every nonzero entry is in; sort them by ranks in parallel.
   // compact the nonzero entries (and count the zero ones), in id order
   const bool nz = live && st > 0.f;
   const bool z = live && !nz;
