@@ -7,17 +7,21 @@
 // B operand of gate/up is x itself (no gather), the extra MMA columns cost nothing next to
 // the weight stream, and the down epilogue keeps only the columns of the tokens routed to
 // the group. The work is a list of units spread round-robin over one CTA per SM:
-//   gate/up unit (group, 64 rows of I): 64 rows of W_gate stacked over the same 64 rows of
-//     W_up, one M = 128 MMA chain over K = d (gate in TMEM lanes 0-63, up in 64-127); the
-//     epilogue writes h = silu(gate) * up as bf16 into the group's H (global, L2-resident)
-//     and publishes the tile on the group's counter;
+//   gate/up unit (group, hg rows of I, hg = 64 or 32): hg rows of W_gate stacked over the
+//     same hg rows of W_up, one M = 2 hg MMA chain over K = d (gate in the first hg rows of
+//     the accumulator, up in the rest); the epilogue writes h = silu(gate) * up as bf16 into
+//     the group's H (global, L2-resident) and publishes the tile on the group's counter;
 //   down unit (group, 128 rows of d): D = W_down tile x H^T over K = I; the producer loads
 //     the weight stages first and the H stages once every gate/up tile of the group is
 //     published; the epilogue stores the fp32 rows per (token, slot).
-// Down units continue the round-robin where the gate/up units stopped, so a CTA that
-// streams a gate/up tile (d x 128 weights) takes at most one down tile (128 x I) and the
-// rest go to CTAs without gate/up work: the weight bytes per SM stay near the mean, every
-// SM streams, and HBM rather than one SM's TMA rate sets the pace.
+// Down units continue the round-robin where the gate/up units stopped. hg is chosen on the
+// device once the unique-expert count is known: 32 when the 32-row gate/up units still fit
+// in one round over the CTAs, else 64. With few unique experts the 64-row units would
+// leave half of the SMs on down tiles only, and one SM's TMA rate, not HBM, would set the
+// pace of the gate/up stream; the 32-row units put a gate/up tile on every SM and keep the
+// weight bytes per SM near the mean. Every stage carries 32 KB of weights: K = 128 for
+// hg = 64 and for the down tiles, K = 256 for hg = 32 (four 128-B boxes per weight row,
+// which also streams faster from HBM than two).
 //
 // Warp roles (192 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, warps 2-5
 // run the epilogues (TMEM lane quadrant = warp % 4). Every wait is bounded (1 s): a timeout
@@ -35,11 +39,11 @@ namespace dmoe {
 namespace {
 
 constexpr int kThr = 192;
-constexpr int kKB = 2;                          // K boxes per stage: K = 128 per stage
+constexpr int kKB = 2;                          // K boxes per down stage: K = 128
 constexpr int kStageK = kKB * kTileK;
-constexpr int kGateBox = 64 * 128;              // 64 weight rows x 128 B
-constexpr int kABox = kTileM * 128;             // 128 rows x 128 B (gate|up, or W_down)
-constexpr int kAStage = kKB * kABox;            // 32 KB
+constexpr int kABox = kTileM * 128;             // 128 rows x 128 B (W_down)
+constexpr int kAStage = kKB * kABox;            // 32 KB of weights in every stage
+constexpr int kMaxKBG = 4;                      // K boxes per gate/up stage (hg = 32)
 constexpr int kMaxStagesD = 6;
 constexpr int kXStride = 17;                    // floats per row of the SwiGLU exchange
 constexpr int kXchgBytes = 2 * 64 * kXStride * 4;
@@ -74,7 +78,8 @@ struct DParams {
   int T, d, E, k, I, Is;
   int imax;                  // max(I, Is): row length of hdense
   int n_pad;                 // token rows of every B box (multiple of 16)
-  int stages;
+  int ring_bytes;            // pipeline ring (multiple of 1 KB)
+  int h32_ok;                // 32-row gate/up units allowed (d % 256 == 0, >= 3 slots fit)
   int has_shared;
   int n_acc;                 // TMEM accumulators of n_pad columns
   uint32_t tmem_cols;
@@ -83,8 +88,11 @@ struct DParams {
 struct DMaps {
   CUtensorMap wg, wu, wd;    // routed: [E*I, d] (64-row boxes) x2, [E*d, I] (128-row boxes)
   CUtensorMap sg, su, sd;    // shared: [Is, d] x2, [d, Is]
+  CUtensorMap wg32, wu32;    // routed gate/up, 32-row boxes
+  CUtensorMap sg32, su32;    // shared gate/up, 32-row boxes
   CUtensorMap x;             // x [T, d], n_pad-row boxes (rows >= T read as zeros)
-  CUtensorMap h;             // hdense, n_pad-row boxes
+  CUtensorMap h;             // hdense, n_pad-row boxes, 128-B swizzle (down B operand)
+  CUtensorMap hst;           // hdense, 32 columns x n_pad rows, no swizzle (tile stores)
 };
 
 // One group of the forward.
@@ -144,18 +152,17 @@ __global__ void __launch_bounds__(kThr, 1)
 moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (ptx::smem_addr(smem_raw) & 1023u)) & 1023u);
-  const int S = p.stages;
   const int bbox = p.n_pad * 128;                 // one K box of token rows
-  const int bstage = kKB * bbox;
+  const int bstage = kKB * bbox;                  // B bytes of a down stage
   const int SP = p.n_pad + 1;                     // floats per row of the down staging tile
-  uint8_t* ring_a = smem;
-  uint8_t* ring_b = ring_a + S * kAStage;
-  float* stage_t = reinterpret_cast<float*>(ring_b + S * bstage);   // [128][SP]
+  // ring of S slots [32 KB of weights | token boxes]; S and the slot size follow hg below
+  uint8_t* ring = smem;
+  float* stage_t = reinterpret_cast<float*>(ring + p.ring_bytes);  // [128][SP]
   float* xchg = stage_t + kTileM * SP;
   int* tok = reinterpret_cast<int*>(xchg + 2 * 64 * kXStride);      // [kMaxTok]
   uint64_t* full = reinterpret_cast<uint64_t*>(tok + kMaxTok);
-  uint64_t* empty = full + S;
-  uint64_t* acc_full = empty + S;
+  uint64_t* empty = full + kMaxStagesD;
+  uint64_t* acc_full = empty + kMaxStagesD;
   uint64_t* acc_empty = acc_full + 4;
   uint64_t* drain = acc_empty + 4;
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
@@ -168,7 +175,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   if (tid == 0) ED_AT(0);
 
   if (tid == 0) {
-    for (int s = 0; s < S; ++s) {
+    for (int s = 0; s < kMaxStagesD; ++s) {
       ptx::mbar_init(&full[s], 1);
       ptx::mbar_init(&empty[s], 1);
     }
@@ -199,7 +206,17 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   const uint32_t tmem_base = *s_tmem;
   const int U = *s_u;
   const int G = U + p.has_shared;
-  const int ngu_s = p.has_shared ? p.Is / 64 : 0, ngu_r = p.I / 64;
+  // gate/up unit height: 32 rows of I when even the 32-row units fit in one round over the
+  // CTAs (a forward with few unique experts), else 64
+  const int ngu64 = (p.has_shared ? p.Is / 64 : 0) + U * (p.I / 64);
+  const int hg = (p.h32_ok && 2 * ngu64 <= nb) ? 32 : 64;
+  const int kbg = kTileM / hg;                    // K boxes per gate/up stage (32 KB)
+  const int slot = kAStage + kbg * bbox;
+  const int S = p.ring_bytes / slot < kMaxStagesD ? p.ring_bytes / slot : kMaxStagesD;
+  auto slot_a = [&](int st) { return ring + st * slot; };
+  auto slot_b = [&](int st) { return ring + st * slot + kAStage; };
+  const int abox_g = 2 * hg * 128;                // one K box of the stacked gate|up rows
+  const int ngu_s = p.has_shared ? p.Is / hg : 0, ngu_r = p.I / hg;
   const int ndn = p.d / kTileM;
   const int NGU = ngu_s + U * ngu_r;
   const int ND = G * ndn;
@@ -260,7 +277,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       }
     }
   };
-  const int kc = p.d / kStageK;      // stages of one gate/up tile
+  const int kc = p.d / (kbg * kTileK);   // stages of one gate/up tile
 
   if (warp == 0 && lane == 0) {
     // ================= TMA producer
@@ -274,20 +291,21 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       int gi, m;
       gu_unit(u, gi, m);
       const Grp g = group(gi);
-      const CUtensorMap* mg = g.shared ? &tm.sg : &tm.wg;
-      const CUtensorMap* mu = g.shared ? &tm.su : &tm.wu;
-      const int arow = (g.shared ? 0 : g.e * p.I) + m * 64;
+      const CUtensorMap* mg =
+          hg == 32 ? (g.shared ? &tm.sg32 : &tm.wg32) : (g.shared ? &tm.sg : &tm.wg);
+      const CUtensorMap* mu =
+          hg == 32 ? (g.shared ? &tm.su32 : &tm.wu32) : (g.shared ? &tm.su : &tm.wu);
+      const int arow = (g.shared ? 0 : g.e * p.I) + m * hg;
       if (first) ED_SET(10, u);
       for (int c = 0; c < kc; ++c) {
         if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
-        ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
-        uint8_t* a_dst = ring_a + stage * kAStage;
-        uint8_t* b_dst = ring_b + stage * bstage;
-#pragma unroll
-        for (int kb = 0; kb < kKB; ++kb) {
-          const int kx = c * kStageK + kb * kTileK;
-          ptx::tma_load_2d(a_dst + kb * kABox, mg, &full[stage], kx, arow, pol_w);
-          ptx::tma_load_2d(a_dst + kb * kABox + kGateBox, mu, &full[stage], kx, arow, pol_w);
+        ptx::mbar_arrive_expect_tx(&full[stage], kAStage + kbg * bbox);
+        uint8_t* a_dst = slot_a(stage);
+        uint8_t* b_dst = slot_b(stage);
+        for (int kb = 0; kb < kbg; ++kb) {
+          const int kx = (c * kbg + kb) * kTileK;
+          ptx::tma_load_2d(a_dst + kb * abox_g, mg, &full[stage], kx, arow, pol_w);
+          ptx::tma_load_2d(a_dst + kb * abox_g + hg * 128, mu, &full[stage], kx, arow, pol_w);
           ptx::tma_load_2d(b_dst + kb * bbox, &tm.x, &full[stage], kx, 0, pol_x);
         }
         ++issued;
@@ -310,7 +328,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       for (int c = 0; c < pre; ++c, ++done) {
         if (!wait(&empty[stage], phase ^ 1u, v)) { ok = false; break; }
         ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
-        uint8_t* a_dst = ring_a + stage * kAStage;
+        uint8_t* a_dst = slot_a(stage);
 #pragma unroll
         for (int kb = 0; kb < kKB; ++kb)
           ptx::tma_load_2d(a_dst + kb * kABox, md, &full[stage], c * kStageK + kb * kTileK, arow,
@@ -320,7 +338,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       }
       if (first) ED_AT(5);
       // then the H rows, once every gate/up tile of the group is published
-      const int target = g.Ig / 64;
+      const int target = g.Ig / hg;
       if (ok && ld_acquire(p.h_ready + gi) < target) {
         const uint64_t t0 = ptx::globaltimer_ns();
         while (ld_acquire(p.h_ready + gi) < target) {
@@ -339,7 +357,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
         int st = st0;
         for (int c = 0; c < done; ++c) {
           if (ok) {
-            uint8_t* b_dst = ring_b + st * bstage;
+            uint8_t* b_dst = slot_b(st);
 #pragma unroll
             for (int kb = 0; kb < kKB; ++kb)
               ptx::tma_load_2d(b_dst + kb * bbox, &tm.h, &full[st], c * kStageK + kb * kTileK,
@@ -354,8 +372,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       for (int c = pre; c < ndk && ok; ++c) {
         if (!wait(&empty[stage], phase ^ 1u, v)) { ok = false; break; }
         ptx::mbar_arrive_expect_tx(&full[stage], kAStage + bstage);
-        uint8_t* a_dst = ring_a + stage * kAStage;
-        uint8_t* b_dst = ring_b + stage * bstage;
+        uint8_t* a_dst = slot_a(stage);
+        uint8_t* b_dst = slot_b(stage);
 #pragma unroll
         for (int kb = 0; kb < kKB; ++kb) {
           const int kx = c * kStageK + kb * kTileK;
@@ -385,9 +403,10 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     int stage = 0, acc = 0;
     uint32_t phase = 0, acc_phase = 0;
     bool ok = true, first = true;
-    auto run = [&](int nstages, int n, int value, bool gu) {
-      const uint32_t n_mma = (uint32_t)(n > 0 ? ((n + 15) & ~15) : 16);
-      const uint32_t idesc = ptx::idesc_bf16(kTileM, n_mma);
+    // nstages stages of kboxes K boxes each; A boxes abox bytes apart, M = mrows
+    auto run = [&](int nstages, int kboxes, int abox, uint32_t mrows, int value, bool gu) {
+      const uint32_t n_mma = (uint32_t)((p.T + 15) & ~15);
+      const uint32_t idesc = ptx::idesc_bf16(mrows, n_mma);
       if (!wait(&acc_empty[acc], acc_phase ^ 1u, value)) { ok = false; return; }
       ptx::tc_fence_after();
       const uint32_t d0 = tmem_base + (uint32_t)(acc * p.n_pad);
@@ -395,13 +414,12 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
         if (!wait(&full[stage], phase, value)) { ok = false; return; }
         if (gu && first && c == 0) ED_AT(2);
         ptx::tc_fence_after();
-        const uint32_t a0 = ptx::smem_addr(ring_a + stage * kAStage);
-        const uint32_t b0 = ptx::smem_addr(ring_b + stage * bstage);
-#pragma unroll
-        for (int kb = 0; kb < kKB; ++kb)
+        const uint32_t a0 = ptx::smem_addr(slot_a(stage));
+        const uint32_t b0 = ptx::smem_addr(slot_b(stage));
+        for (int kb = 0; kb < kboxes; ++kb)
 #pragma unroll
           for (int kk = 0; kk < kTileK / 16; ++kk)
-            ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kABox + kk * 32),
+            ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * abox + kk * 32),
                           ptx::sdesc_k_sw128(b0 + kb * bbox + kk * 32), idesc,
                           (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
         ptx::mma_commit(&empty[stage]);
@@ -414,14 +432,14 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       int gi, m;
       gu_unit(u, gi, m);
       // all T token columns: the B box is x (rows >= T are zeros)
-      run(kc, p.T, u, true);
+      run(kc, kbg, abox_g, (uint32_t)(2 * hg), u, true);
       if (first) ED_AT(3);
       first = false;
     }
     first = true;
     for (int v = v0; v < ND && ok; v += nb) {
       const Grp g = group(v / ndn);
-      run(g.Ig / kStageK, p.T, v, false);
+      run(g.Ig / kStageK, kKB, kABox, (uint32_t)kTileM, v, false);
       if (first) ED_AT(7);
       first = false;
     }
@@ -437,7 +455,12 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     const int row = q * 32 + lane;                // accumulator row of this thread
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     const bool is_gate = q < 2;
-    const int r64 = (q & 1) * 32 + lane;          // row within the 64-row slice
+    // gate/up accumulator (M = 2 hg): row r sits in TMEM lane r for M = 128 and in lane
+    // 32 (r / 16) + r % 16 for M = 64, so each quadrant holds rq = hg / 2 rows in its first
+    // rq lanes: gate rows in quadrants 0-1, the matching up rows in quadrants 2-3
+    const int rq = hg / 2;
+    const bool g_act = lane < rq;
+    const int rr = (q & 1) * rq + lane;           // row within the hg-row slice
     const int n_mma = (p.T + 15) & ~15;
     int acc = 0, xb = 0;
     uint32_t acc_phase = 0;
@@ -449,27 +472,25 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (!ok) break;
       ptx::tc_fence_after();
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
-      // the H tile (n_pad token rows x 64 columns, bf16) is laid out in the staging tile
-      // exactly as the 128-byte-swizzled box of the H tensor map, then stored by TMA
+      // the H tile (n_pad token rows x hg columns, bf16) is laid out in the staging tile as
+      // hg / 32 row-major boxes of 32 columns, then stored by TMA
       uint8_t* hbox = reinterpret_cast<uint8_t*>(stage_t);
       for (int c0 = 0; c0 < n_mma; c0 += 16) {
         float v[16];
         ptx::tmem_ld16(tbase + c0, v);
         ptx::tmem_ld_wait();
         float* buf = xchg + xb * (64 * kXStride);
-        if (!is_gate) {
+        if (!is_gate && g_act) {
 #pragma unroll
-          for (int c = 0; c < 16; ++c) buf[r64 * kXStride + c] = v[c];
+          for (int c = 0; c < 16; ++c) buf[rr * kXStride + c] = v[c];
         }
         named_bar_sync(2, 128);
-        if (is_gate) {
+        if (is_gate && g_act) {
+          uint8_t* hcol = hbox + (rr >> 5) * p.n_pad * 64 + (rr & 31) * 2;
 #pragma unroll
-          for (int c = 0; c < 16; ++c) {
-            const int t = c0 + c;
-            *reinterpret_cast<__nv_bfloat16*>(hbox + t * 128 + (((r64 >> 3) ^ (t & 7)) << 4) +
-                                              (r64 & 7) * 2) =
-                __float2bfloat16(silu_f(v[c]) * buf[r64 * kXStride + c]);
-          }
+          for (int c = 0; c < 16; ++c)
+            *reinterpret_cast<__nv_bfloat16*>(hcol + (c0 + c) * 64) =
+                __float2bfloat16(silu_f(v[c]) * buf[rr * kXStride + c]);
         }
         xb ^= 1;
       }
@@ -481,7 +502,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       ptx::fence_proxy_async_smem();
       named_bar_sync(2, 128);
       if (et == 0) {
-        tma_store_2d(&tm.h, hbox, m * 64, gi * p.n_pad);
+        for (int j = 0; j < hg / 32; ++j)
+          tma_store_2d(&tm.hst, hbox + j * p.n_pad * 64, m * hg + 32 * j, gi * p.n_pad);
         bulk_commit_wait_all();
         fence_proxy_async_global();
         red_release_add(p.h_ready + gi, 1);
@@ -579,18 +601,19 @@ EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// bf16 matrix [rows, cols] row-major (row pitch `pitch` elements), box = 64 columns (128 B)
-// x box_rows rows, 128-B swizzle.
+// bf16 matrix [rows, cols] row-major, box = 64 columns (128 B) x box_rows rows with the
+// 128-B swizzle, or (plain) box_cols columns x box_rows rows without swizzle.
 bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
-              uint64_t pitch = 0) {
+              bool plain = false, uint32_t box_cols = 64) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return false;
   const cuuint64_t dims[2] = {cols, rows};
-  const cuuint64_t strides[1] = {(pitch ? pitch : cols) * 2};
-  const cuuint32_t box[2] = {64, box_rows};
+  const cuuint64_t strides[1] = {cols * 2};
+  const cuuint32_t box[2] = {plain ? box_cols : 64u, box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             plain ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -614,16 +637,26 @@ uint32_t pow2_cols(uint32_t n) {
 }
 
 // Shared memory besides the ring: staging tile, SwiGLU exchange, token list, barriers.
-size_t fixed_smem(int n_pad, int stages) {
+size_t fixed_smem(int n_pad) {
   return 1024 /* alignment */ + (size_t)kTileM * (n_pad + 1) * 4 + kXchgBytes + kMaxTok * 4 +
-         (size_t)(2 * stages + 9) * 8 + 64;
+         (size_t)(2 * kMaxStagesD + 9) * 8 + 64;
 }
 
-int plan_stages(int T) {
+// Pipeline ring: the shared memory left by the fixed part. A slot holds 32 KB of weights
+// and two K boxes of token rows (64-row gate/up units, down tiles) or four (32-row gate/up
+// units, K = 256 per stage; allowed when d is a multiple of 256 and three slots fit).
+struct Ring {
+  int bytes, stages2, h32_ok;
+};
+Ring plan_ring(int T, int d) {
   const int n_pad = ((T + 15) / 16) * 16;
-  const long avail = (long)max_smem_optin() - (long)fixed_smem(n_pad, kMaxStagesD);
-  int stages = (int)(avail / (kAStage + kKB * n_pad * 128));
-  return stages > kMaxStagesD ? kMaxStagesD : stages;
+  long avail = (long)max_smem_optin() - (long)fixed_smem(n_pad);
+  avail = avail > 0 ? (avail & ~1023L) : 0;
+  Ring r;
+  r.bytes = (int)avail;
+  r.stages2 = (int)(avail / (kAStage + kKB * n_pad * 128));
+  r.h32_ok = d % (kMaxKBG * kTileK) == 0 && avail / (kAStage + kMaxKBG * n_pad * 128) >= 3;
+  return r;
 }
 
 }  // namespace
@@ -642,28 +675,34 @@ extern "C" int dmoe_debug_dtrace_clear() {
 bool experts_decode_ok(int T, int d, int I, int Is) {
   if (T < 1 || T > kMaxTok || d % kTileM != 0 || I % kStageK != 0 || (Is > 0 && Is % kStageK != 0))
     return false;
-  return plan_stages(T) >= 2;
+  return plan_ring(T, d).stages2 >= 2;
 }
 
 cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   const bool has_shared = a.Is > 0;
-  const int stages = plan_stages(a.T);
-  if (stages < 2) return cudaErrorInvalidConfiguration;
+  const Ring ring = plan_ring(a.T, a.d);
+  if (ring.stages2 < 2) return cudaErrorInvalidConfiguration;
   const int n_pad = ((a.T + 15) / 16) * 16;
   const int imax = a.I > a.Is ? a.I : a.Is;
 
   DMaps m;
   bool ok = make_map(&m.wg, a.w_gate, (uint64_t)a.E * a.I, a.d, 64) &&
             make_map(&m.wu, a.w_up, (uint64_t)a.E * a.I, a.d, 64) &&
+            make_map(&m.wg32, a.w_gate, (uint64_t)a.E * a.I, a.d, 32) &&
+            make_map(&m.wu32, a.w_up, (uint64_t)a.E * a.I, a.d, 32) &&
             make_map(&m.wd, a.w_down, (uint64_t)a.E * a.d, a.I, kTileM) &&
             make_map(&m.x, a.x, (uint64_t)a.T, a.d, (uint32_t)n_pad) &&
             make_map(&m.h, a.hdense, (uint64_t)(a.E + 1) * n_pad, (uint64_t)imax,
-                     (uint32_t)n_pad);
+                     (uint32_t)n_pad) &&
+            make_map(&m.hst, a.hdense, (uint64_t)(a.E + 1) * n_pad, (uint64_t)imax,
+                     (uint32_t)n_pad, true, 32);
   if (ok && has_shared)
     ok = make_map(&m.sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
          make_map(&m.su, a.ws_up, (uint64_t)a.Is, a.d, 64) &&
+         make_map(&m.sg32, a.ws_gate, (uint64_t)a.Is, a.d, 32) &&
+         make_map(&m.su32, a.ws_up, (uint64_t)a.Is, a.d, 32) &&
          make_map(&m.sd, a.ws_down, (uint64_t)a.d, a.Is, kTileM);
-  if (!has_shared) { m.sg = m.wg; m.su = m.wu; m.sd = m.wd; }
+  if (!has_shared) { m.sg = m.wg; m.su = m.wu; m.sd = m.wd; m.sg32 = m.wg32; m.su32 = m.wu32; }
   if (!ok) return cudaErrorInvalidValue;
 
   DParams p{};
@@ -680,12 +719,12 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
   p.imax = imax;
   p.n_pad = n_pad;
-  p.stages = stages;
+  p.ring_bytes = ring.bytes;
+  p.h32_ok = ring.h32_ok;
   p.has_shared = has_shared ? 1 : 0;
   p.n_acc = 512 / n_pad > 4 ? 4 : 512 / n_pad;
   p.tmem_cols = pow2_cols((uint32_t)(p.n_acc * n_pad));
-  const size_t smem =
-      (size_t)stages * (kAStage + (size_t)kKB * n_pad * 128) + fixed_smem(n_pad, stages);
+  const size_t smem = (size_t)ring.bytes + fixed_smem(n_pad);
 
   static std::mutex mu;
   static int attr_dev_mask = 0;  // the dynamic smem limit is a per-device function attribute
