@@ -192,13 +192,14 @@ struct ExpertArgs {
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E);
-// gate-weighted combine of the expert rows into y (the last launch of both expert paths)
-cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s);
+// gate-weighted combine of the expert rows into y (the last launch of both expert paths);
+// it also clears zero[0 .. n_zero) once the launch before it has ended
+cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = nullptr,
+                           int n_zero = 0);
 // Decode-sized forwards (T <= 64): one persistent launch over gate/up and down tiles of
 // every group, all tokens at once (no gather), then the combine.
 bool experts_decode_ok(int T, int d, int I, int Is);
 cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s);
-constexpr int kTicketDecodeExit = 1;   // tickets[1]: CTAs of the decode expert launch done
 
 // profiling events (dmoe_set_profile_events), per host thread
 void prof_begin(int kernel, cudaStream_t s);

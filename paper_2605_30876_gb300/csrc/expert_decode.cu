@@ -25,8 +25,8 @@
 //
 // Warp roles (192 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, warps 2-5
 // run the epilogues (TMEM lane quadrant = warp % 4). Every wait is bounded (1 s): a timeout
-// is recorded and the CTA unwinds. The last CTA to finish clears the group counters for
-// the next call.
+// is recorded and the CTA unwinds. The combine launch that follows clears the group
+// counters for the next call.
 #include <math.h>
 
 #include <mutex>
@@ -72,8 +72,8 @@ struct DParams {
   __nv_bfloat16* hdense;     // [(E+1) * n_pad, imax]: H of group g in rows g*n_pad ..
   float* yslot;              // [T*k, d]
   float* yshared;            // [T, d]
-  int32_t* h_ready;          // [E+1]: published gate/up tiles per group
-  int32_t* exit_ticket;      // zero between calls
+  int32_t* h_ready;          // [E+1]: published gate/up tiles per group (zero between calls;
+                             // the combine launch clears them)
   DevErrRecord* err;
   int T, d, E, k, I, Is;
   int imax;                  // max(I, Is): row length of hdense
@@ -568,16 +568,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     __syncwarp();
     ptx::tmem_dealloc(tmem_base, p.tmem_cols);
   }
-  if (tid == 0) {
-    // the last CTA clears the group counters for the next call
-    __threadfence();
-    if (atomicAdd(p.exit_ticket, 1) == nb - 1) {
-      for (int gi = 0; gi <= p.E; ++gi) p.h_ready[gi] = 0;
-      __threadfence();
-      *p.exit_ticket = 0;
-    }
-    ED_AT(9);
-  }
+  if (tid == 0) ED_AT(9);
   KLOG(DMOE_KERNEL_EXPERTS, 1);
 }
 
@@ -714,7 +705,6 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.yslot = a.yslot;
   p.yshared = a.yshared;
   p.h_ready = a.h_ready;
-  p.exit_ticket = a.tickets + kTicketDecodeExit;
   p.err = a.err;
   p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
   p.imax = imax;
@@ -746,7 +736,7 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
-  return launch_combine(a, s);
+  return launch_combine(a, s, a.h_ready, a.E + 1);
 }
 
 }  // namespace dmoe
