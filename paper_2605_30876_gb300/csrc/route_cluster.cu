@@ -3,7 +3,9 @@
 //
 // Cluster c owns 32 experts; CTA r of the cluster owns the r-th eighth of d:
 //   1. logits: TMA brings the W_r slice (d/8 rows x 32 experts, 128-B rows) and the x
-//      slice (T rows x d/8); fp32 FFMA gives partial logits [T x 32] in shared memory;
+//      slice (T rows x d/8); the W_r slice is split into three bf16 parts (hi + mid + lo
+//      = w to 2^-27, x * part exact in fp32) and tensor cores (mma.sync, fp32 accumulate)
+//      give the partial logits [T x 32] in shared memory;
 //      CTA r then adds, in rank order, the eight partials of the tokens t = r (mod 8) over
 //      distributed shared memory and writes those logits.
 //   2. one atomic ticket: the last cluster to finish continues; the others exit.
@@ -22,7 +24,8 @@
 // and 7: globaltimer, others: 1 = reached; + 32: clock64): 0 entry, 1 TMA landed, 8 x converted,
 // 2 partial logits done, 3 logits reduced, 4 ticket, 9 score loads issued, 10 softmax,
 // 11 top-k, 5 scores, 12 coreset, 13 MaskOutside, 6 Algorithm 1, 7 dispatch; 16-24: steps
-// inside the dispatch, the coreset and MaskOutside (DMOE_STAMP in the shared headers).
+// inside the dispatch, the coreset and MaskOutside (DMOE_STAMP in the shared headers);
+// 25 coreset of the block known, 26 coreset received, 27 token's restricted top-k known.
 #ifdef DMOE_TRACE
 #include <stdint.h>
 __device__ uint64_t g_ctrace[64 * 8 * 64];
@@ -220,15 +223,16 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   __syncthreads();
   CT_AT(8);
   // tensor cores (mma.sync m16n8k16): warp tile = 16 tokens x 8 experts over the whole
-  // slice; per 16-wide K step the hi, mid and lo parts in that order
+  // slice; one accumulator per part (hi, mid, lo), summed in that order at the end
   {
     const int g = lane >> 2, tq = lane & 3;
     const int ntile = (T16 / 16) * (kClExp / 8);
     for (int tile = warp; tile < ntile; tile += 8) {
       const int mt = tile / (kClExp / 8), nt = tile % (kClExp / 8);
       const int r0 = mt * 16 + g;                   // A rows r0, r0 + 8 (same swizzle phase)
-      float acc[4] = {0.f, 0.f, 0.f, 0.f};
+      float accp[3][4] = {};
       const uint8_t* brow = Wt + (nt * 8 + g) * kWtStride + tq * 4;
+#pragma unroll 2
       for (int k0 = 0; k0 < DC; k0 += 16) {
         const int bx = k0 >> 6, c = (k0 & 63) >> 3;   // box, 16-B chunk of k0
         const uint8_t* xb = Xs + bx * T16 * 128;
@@ -240,10 +244,13 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 #pragma unroll
         for (int part = 0; part < 3; ++part) {
           const uint8_t* bp = brow + part * kClExp * kWtStride + k0 * 2;
-          mma_bf16_16816(acc, af, *reinterpret_cast<const uint32_t*>(bp),
+          mma_bf16_16816(accp[part], af, *reinterpret_cast<const uint32_t*>(bp),
                          *reinterpret_cast<const uint32_t*>(bp + 16));
         }
       }
+      float acc[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) acc[i] = (accp[0][i] + accp[1][i]) + accp[2][i];
       // D rows r0, r0 + 8; columns 2tq, 2tq + 1 of the tile
       const int e = nt * 8 + 2 * tq;
       if (r0 < T) {
@@ -419,6 +426,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           E, k, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
+      CT_AT(25);
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order
       for (int i = tid; i < B * (size + 1); i += 256) {
@@ -430,6 +438,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     }
     CT_AT(12);
     cluster_sync();
+    CT_AT(26);
     {
       const int t = 8 * (int)rank + warp;
       if (t < T) {
@@ -465,6 +474,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           }
           warp_topk(cv, ce, valid, k, my_e, my_v);
         }
+        CT_AT(27);
         float g = 0.f;
         for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
         if (lane < k) {

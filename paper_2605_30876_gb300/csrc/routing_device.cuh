@@ -187,9 +187,10 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 //
 // Top-P accumulates the sorted values in order in fp32 and stops at the first running sum
 // >= p (p >= 1: at the last nonzero entry); the floor extends the coreset to k entries
-// (zero entries in id order). For p < 1 one warp takes the entries in sorted order by a
-// tournament until both rules are met; for p >= 1 every nonzero S~ counts the nonzero
-// entries that beat it (larger, or equal with a lower id), all in parallel.
+// (zero entries in id order). For p < 1 every warp sorts its 32 entries by rank, then one
+// warp merges the sorted lists by a tournament over their heads until both rules are met;
+// for p >= 1 every nonzero S~ counts the nonzero entries that beat it (larger, or equal
+// with a lower id), all in parallel. Needs blockDim.x == kMaxExperts.
 template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
@@ -220,48 +221,45 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
   DMOE_STAMP(19);
   const float st = live ? S / tot : 0.f;
   if (top_p < 1.f) {
-    // p < 1: the coreset is a short sorted prefix. Warp 0 takes the entries in sorted order
-    // by a tournament (lane l holds experts l + 32j and its best remaining one; each round
-    // the warp's best by two single-instruction reductions) and keeps the running sum.
-    if (live) st_s[tid] = st;
+    // p < 1: the coreset is a short sorted prefix. Each warp sorts its 32 entries by their
+    // ranks (larger key, then lower id); warp 0 then takes the entries in sorted order by a
+    // tournament over the heads of the eight lists (lane w holds list w's head; each round
+    // the best head by two single-instruction reductions, and its list advances) and keeps
+    // the running sum. Padding entries (id >= E) have key 0 and are never reached.
+    __shared__ uint32_t wkey[kMaxExperts];
+    __shared__ uint2 wl[kMaxExperts];   // list of warp w: wl[32 w .. 32 w + 31], best first
+    const uint32_t key = live ? order_key(st) : 0u;
+    wkey[tid] = key;
+    const uint32_t bnz = __ballot_sync(0xffffffffu, live && st > 0.f);
+    if (lane == 0) wcnt[0][warp] = __popc(bnz);
+    __syncwarp();
+    int r = 0;
+#pragma unroll 8
+    for (int j = 0; j < 32; ++j) {
+      const uint32_t kj = wkey[warp * 32 + j];
+      r += (kj > key || (kj == key && j < lane)) ? 1 : 0;
+    }
+    wl[warp * 32 + r] = make_uint2(key, (uint32_t)tid);
     __syncthreads();
     if (warp == 0) {
-      uint32_t key[8];
-      int nz = 0;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int e = lane + 32 * j;
-        const float x = e < E ? st_s[e] : 0.f;
-        key[j] = e < E ? order_key(x) : 0u;
-        nz += (e < E && x > 0.f) ? 1 : 0;
-      }
-      const int nnz = __reduce_add_sync(0xffffffffu, nz);
-      uint32_t bk = 0u;
-      int bj = 0;
-#pragma unroll
-      for (int j = 0; j < 8; ++j)
-        if (key[j] > bk) { bk = key[j]; bj = j; }   // ties: the lower id (lower j) stays
+      const int nw = (int)(blockDim.x >> 5);
+      const int nnz = __reduce_add_sync(0xffffffffu, lane < nw ? wcnt[0][lane] : 0);
+      int h = 0;
+      uint2 hd = lane < nw ? wl[lane * 32] : make_uint2(0u, 0xffffffffu);
       float cum = 0.f;
       int m = -1, cnt = 0;
       for (;;) {
         const int target = (m < 0) ? E : max(m, k);
         if (cnt >= target) break;
-        const uint32_t kmax = __reduce_max_sync(0xffffffffu, bk);
-        const uint32_t imin =
-            __reduce_min_sync(0xffffffffu, bk == kmax ? (uint32_t)(lane + 32 * bj) : 0xffffffffu);
+        const uint32_t kmax = __reduce_max_sync(0xffffffffu, hd.x);
+        const uint32_t imin = __reduce_min_sync(0xffffffffu, hd.x == kmax ? hd.y : 0xffffffffu);
         if (lane == 0) order[cnt] = (int)imin;
         cum += key_value(kmax);
         ++cnt;
         if (m < 0 && (cum >= top_p || cnt >= nnz)) m = min(cnt, nnz);
-        if (bk == kmax && (uint32_t)(lane + 32 * bj) == imin) {
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (j == bj) key[j] = 0u;
-          bk = 0u;
-          bj = 0;
-#pragma unroll
-          for (int j = 0; j < 8; ++j)
-            if (key[j] > bk) { bk = key[j]; bj = j; }
+        if (hd.y == imin) {   // ids are unique: only the winner's list advances
+          ++h;
+          hd = h < 32 ? wl[lane * 32 + h] : make_uint2(0u, 0xffffffffu);
         }
       }
       if (lane == 0) s_size = max(m, k);
