@@ -146,6 +146,18 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   const int e0 = blockIdx.y * kClExp;
   const int n_clusters = gridDim.y;
   pdl_launch_dependents();
+  if (tid == 0) {
+    // while the previous launch on the stream finishes: pull this CTA's W_r slice and the
+    // shared expert's weights into L2. Only L2 is touched, and L2 is where a write by that
+    // launch would land, so the loads below still see it.
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.wmap)) : "memory");
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.xmap)) : "memory");
+    asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(
+                     reinterpret_cast<uint64_t>(&f.wmap)),
+                 "r"(e0), "r"((int)rank * DC)
+                 : "memory");
+    issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
+  }
   pdl_wait();
   KLOG(DMOE_KERNEL_ROUTER, 0);
   CT_AT(0);
@@ -158,8 +170,6 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(s_addr(&s_bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.wmap)) : "memory");
-    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&f.xmap)) : "memory");
     const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)nxb * T16 * 128;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_addr(&s_bar)),
                  "r"(bytes)
@@ -177,7 +187,6 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           "l"(reinterpret_cast<uint64_t>(&f.xmap)), "r"(s_addr(&s_bar)),
           "r"((int)rank * DC + 64 * bx), "r"(0)
           : "memory");
-    issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
   }
   for (int e = tid; e < E; e += 256) s_bias[e] = a.bias != nullptr ? a.bias[e] : 0.f;
   __syncthreads();
