@@ -37,6 +37,8 @@ enum DevWhere : int32_t {
   kAtCombine = 6, kAtGather = 7,
 };
 constexpr int kRouteTickets = 256;
+constexpr int kTicketSpec = 64;   // tickets[64] (own 128-B line): coresets published
+constexpr int kRouteClusterCtas = 8;   // CTAs per cluster of the decode-size routing launch
 struct DevErrRecord {
   int32_t code;
   int32_t where;
@@ -76,6 +78,7 @@ struct Workspace {
   size_t yslot;        // fp32 [T*k, d]   expert outputs per (token, slot)
   size_t yshared;      // fp32 [T, d]
   size_t hdense;       // bf16 [(E+1) * n_pad, max(I, I_s)]: H per group over all tokens
+  size_t spec;         // int32 [n_blocks, k]: the coreset of every block (block top-k call)
                        // (decode-size forwards only)
   size_t total;
   int router_splits;
@@ -147,6 +150,11 @@ struct RouterArgs {
   DevErrRecord* err;
   L2Prefetch shared_pf;   // the shared expert's weights (one "expert")
   bool probs_requested;   // the caller wants the scores in `probs`
+  // block top-k (p <= 0) in the fused decode-size call: every block's coreset, which is
+  // then the block's routing, is published early here (k ids per block), and spec_cnt is
+  // raised once per block (release); nullptr otherwise
+  int32_t* spec_ids;
+  int32_t* spec_cnt;
 };
 
 struct DispatchArgs {
@@ -187,15 +195,20 @@ struct ExpertArgs {
   int32_t* tickets;       // kRouteTickets ints, zero between calls
   DevErrRecord* err;
   bool prefetch_shared;   // the shared expert's weights were not prefetched by the router
+  // decode-size path, block top-k: the unique experts are the union of the published
+  // coresets (RouterArgs::spec_ids), known before the routing launch ends; nullptr otherwise
+  const int32_t* spec_ids;
+  int32_t* spec_cnt;
+  int spec_blocks;
   // shape
   int T, d, E, k, I, Is, n_max;
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E);
 // gate-weighted combine of the expert rows into y (the last launch of both expert paths);
-// it also clears zero[0 .. n_zero) once the launch before it has ended
+// it also clears zero[0 .. n_zero) and *zero1 (when set) once the launch before it has ended
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = nullptr,
-                           int n_zero = 0);
+                           int n_zero = 0, int32_t* zero1 = nullptr);
 // Decode-sized forwards (T <= 64): one persistent launch over gate/up and down tiles of
 // every group, all tokens at once (no gather), then the combine.
 bool experts_decode_ok(int T, int d, int I, int Is);

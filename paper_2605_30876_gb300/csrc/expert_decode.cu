@@ -74,6 +74,9 @@ struct DParams {
   float* yshared;            // [T, d]
   int32_t* h_ready;          // [E+1]: published gate/up tiles per group (zero between calls;
                              // the combine launch clears them)
+  const int32_t* spec_ids;   // block top-k: published coresets [spec_blocks, k], or nullptr
+  const int32_t* spec_cnt;   // coresets published so far
+  int spec_blocks;
   DevErrRecord* err;
   int T, d, E, k, I, Is;
   int imax;                  // max(I, Is): row length of hdense
@@ -168,6 +171,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   int* s_u = const_cast<int*>(s_abort) + 1;
+  uint8_t* s_spec = reinterpret_cast<uint8_t*>(s_u + 1);   // [kMaxExperts]: unique ids
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nb = gridDim.x, b = blockIdx.x;
@@ -191,14 +195,58 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
-  pdl_wait();   // the dispatch is complete from here on
-  if (tid == 0) {
-    int u = __ldcg(p.n_unique);
-    if (u < 0 || u > p.E) {
-      record_error(p.err, kErrBadDispatch, kAtGateUp, u);
-      u = 0;
+  // Block top-k: the unique experts are the union of the blocks' coresets (every token of a
+  // block is routed to all k experts of its coreset), published by the routing launch
+  // before it ends; the weight stream starts on them, and only the down epilogue waits for
+  // the dispatch. Otherwise (or if the coresets do not come) everything waits for it.
+  bool spec = p.spec_ids != nullptr;
+  if (spec) {
+    if (warp == 0) {
+      int ok = 1;
+      if (lane == 0) {
+        const uint64_t t0 = ptx::globaltimer_ns();
+        while (ld_acquire(p.spec_cnt) < p.spec_blocks) {
+          if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {
+            ok = 0;
+            break;
+          }
+          __nanosleep(64);
+        }
+      }
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      uint32_t m[kMaxExperts / 32] = {};
+      bool bad = !ok;
+      if (ok)
+        for (int i = lane; i < p.spec_blocks * p.k; i += 32) {
+          const int e = __ldcg(p.spec_ids + i);
+          if (e < 0 || e >= p.E) bad = true;
+          else m[e >> 5] |= 1u << (e & 31);
+        }
+      bad = __any_sync(0xffffffffu, bad);
+#pragma unroll
+      for (int w = 0; w < kMaxExperts / 32; ++w) m[w] = __reduce_or_sync(0xffffffffu, m[w]);
+      if (lane == 0) {
+        int u = 0;
+        if (!bad)
+          for (int w = 0; w < kMaxExperts / 32; ++w)
+            for (uint32_t bits = m[w]; bits != 0u; bits &= bits - 1u)
+              s_spec[u++] = (uint8_t)(w * 32 + __ffs((int)bits) - 1);
+        *s_u = bad ? -1 : u;
+      }
     }
-    *s_u = u;
+    __syncthreads();
+    spec = *s_u >= 0;
+  }
+  if (!spec) {
+    pdl_wait();   // the dispatch is complete from here on
+    if (tid == 0) {
+      int u = __ldcg(p.n_unique);
+      if (u < 0 || u > p.E) {
+        record_error(p.err, kErrBadDispatch, kAtGateUp, u);
+        u = 0;
+      }
+      *s_u = u;
+    }
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -224,31 +272,45 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   const int v0 = ((b - NGU % nb) % nb + nb) % nb;
   if (tid == 0) ED_AT(1);
 
-  auto group = [&](int gi) -> Grp {
+  // the group's expert and size (all the weight stream needs)
+  auto group_w = [&](int gi) -> Grp {
     Grp g;
+    g.row0 = 0;
+    g.n = 0;
     if (gi < p.has_shared) {
       g.shared = true;
       g.e = 0;
-      g.row0 = 0;
-      g.n = p.T;
       g.Ig = p.Is;
+      return g;
+    }
+    const int u = gi - p.has_shared;
+    int e = spec ? (int)s_spec[u] : __ldcg(p.unique_ids + u);
+    if (e < 0 || e >= p.E) {
+      record_error(p.err, kErrBadDispatch, kAtGateUp, u);
+      e = 0;
+    }
+    g.shared = false;
+    g.e = e;
+    g.Ig = p.I;
+    return g;
+  };
+  // ... and its rows of the dispatch (once the dispatch is complete)
+  auto group = [&](int gi) -> Grp {
+    Grp g = group_w(gi);
+    if (g.shared) {
+      g.n = p.T;
       return g;
     }
     const int u = gi - p.has_shared;
     int row0 = __ldcg(p.offsets + u);
     int n = __ldcg(p.offsets + u + 1) - row0;
-    int e = __ldcg(p.unique_ids + u);
-    if (e < 0 || e >= p.E || n < 0 || n > p.T || row0 < 0 || row0 + n > p.T * p.k) {
-      record_error(p.err, kErrBadDispatch, kAtGateUp, u);
+    if (n < 0 || n > p.T || row0 < 0 || row0 + n > p.T * p.k) {
+      record_error(p.err, kErrBadDispatch, kAtDown, u);
       n = 0;
-      e = 0;
       row0 = 0;
     }
-    g.shared = false;
-    g.e = e;
     g.row0 = row0;
     g.n = n;
-    g.Ig = p.I;
     return g;
   };
   // gate/up unit -> (group, 64-row tile)
@@ -290,7 +352,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     for (int u = b; u < NGU && ok; u += nb) {
       int gi, m;
       gu_unit(u, gi, m);
-      const Grp g = group(gi);
+      const Grp g = group_w(gi);
       const CUtensorMap* mg =
           hg == 32 ? (g.shared ? &tm.sg32 : &tm.wg32) : (g.shared ? &tm.sg : &tm.wg);
       const CUtensorMap* mu =
@@ -316,7 +378,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     first = true;
     for (int v = v0; v < ND && ok; v += nb) {
       const int gi = v / ndn, i = v % ndn;
-      const Grp g = group(gi);
+      const Grp g = group_w(gi);
       const CUtensorMap* md = g.shared ? &tm.sd : &tm.wd;
       const int arow = (g.shared ? 0 : g.e * p.d) + i * kTileM;
       const int ndk = g.Ig / kStageK;
@@ -438,7 +500,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     }
     first = true;
     for (int v = v0; v < ND && ok; v += nb) {
-      const Grp g = group(v / ndn);
+      const Grp g = group_w(v / ndn);
       run(g.Ig / kStageK, kKB, kABox, (uint32_t)kTileM, v, false);
       if (first) ED_AT(7);
       first = false;
@@ -513,6 +575,17 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       first = false;
     }
     first = true;
+    if (spec && v0 < ND) {
+      // the rows of the dispatch from here on; the coresets must have given its unique list
+      pdl_wait();
+      if (warp == 2) {
+        bool bad = __ldcg(p.n_unique) != U;
+        for (int u = lane; u < U; u += 32)
+          if (__ldcg(p.unique_ids + u) != (int)s_spec[u]) bad = true;
+        if (__any_sync(0xffffffffu, bad) && lane == 0)
+          record_error(p.err, kErrBadDispatch, kAtDown, -1);
+      }
+    }
     for (int v = v0; v < ND; v += nb) {
       const int gi = v / ndn, i = v % ndn;
       const Grp g = group(gi);
@@ -630,7 +703,7 @@ uint32_t pow2_cols(uint32_t n) {
 // Shared memory besides the ring: staging tile, SwiGLU exchange, token list, barriers.
 size_t fixed_smem(int n_pad) {
   return 1024 /* alignment */ + (size_t)kTileM * (n_pad + 1) * 4 + kXchgBytes + kMaxTok * 4 +
-         (size_t)(2 * kMaxStagesD + 9) * 8 + 64;
+         (size_t)(2 * kMaxStagesD + 9) * 8 + 16 + kMaxExperts + 48;
 }
 
 // Pipeline ring: the shared memory left by the fixed part. A slot holds 32 KB of weights
@@ -705,6 +778,9 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.yslot = a.yslot;
   p.yshared = a.yshared;
   p.h_ready = a.h_ready;
+  p.spec_ids = a.spec_ids;
+  p.spec_cnt = a.spec_cnt;
+  p.spec_blocks = a.spec_blocks;
   p.err = a.err;
   p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
   p.imax = imax;
@@ -730,13 +806,16 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
       if (dev < 31) attr_dev_mask |= 1 << dev;
     }
   }
+  // one CTA per SM; when the stream starts on the published coresets, the last routing
+  // cluster still holds its SMs, and a CTA placed there would start only when it ends
   int grid = device_sm_count();
+  if (a.spec_ids != nullptr && grid > 2 * kRouteClusterCtas) grid -= kRouteClusterCtas;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
   cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
-  return launch_combine(a, s, a.h_ready, a.E + 1);
+  return launch_combine(a, s, a.h_ready, a.E + 1, a.spec_cnt);
 }
 
 }  // namespace dmoe

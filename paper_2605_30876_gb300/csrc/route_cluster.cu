@@ -56,7 +56,7 @@ __device__ uint64_t g_ctrace[64 * 8 * 64];
 namespace dmoe {
 namespace {
 
-constexpr int kCl = 8;                 // CTAs per cluster (split of d)
+constexpr int kCl = kRouteClusterCtas;   // CTAs per cluster (split of d)
 constexpr int kClExp = 32;             // experts per cluster
 constexpr int kClMaxTok = 64;          // tokens of a decode-sized forward
 constexpr int kClMaxDChunk = 256;      // d / kCl at most (one TMA box of rows)
@@ -145,7 +145,6 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   const int DC = a.d / kCl;                          // rows of d in this CTA's slice
   const int e0 = blockIdx.y * kClExp;
   const int n_clusters = gridDim.y;
-  pdl_launch_dependents();
   if (tid == 0) {
     // while the previous launch on the stream finishes: pull this CTA's W_r slice and the
     // shared expert's weights into L2. Only L2 is touched, and L2 is where a write by that
@@ -159,6 +158,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
   }
   pdl_wait();
+  // the expert launch may start now (not earlier: it reads the early coreset counter, which
+  // the launch before this one clears)
+  pdl_launch_dependents();
   KLOG(DMOE_KERNEL_ROUTER, 0);
   CT_AT(0);
 
@@ -436,6 +438,16 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
       CT_AT(25);
+      if (a.spec_ids != nullptr) {
+        // block top-k: the coreset (k experts) is the routing of every token of the block;
+        // publish it for the expert launch
+        if (tid < k) a.spec_ids[(size_t)b * k + tid] = order[tid];
+        __syncthreads();
+        if (tid == 0) {
+          __threadfence();
+          asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.spec_cnt) : "memory");
+        }
+      }
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order
       for (int i = tid; i < B * (size + 1); i += 256) {

@@ -26,6 +26,9 @@ LAYER_CASES = {
     "E8_k3_d128": TINY.with_(n_experts=8, top_k=3, top_p=0.7, d_model=128, d_ff=256),
     "T300_multi_ntile": LAYER.with_(block_size=60, n_blocks=5, top_p=0.0),
     "wide_ff_I1024": TINY.with_(d_model=512, d_ff=1024, d_ff_shared=384, n_blocks=3, top_p=0.6),
+    # block top-k at decode sizes: the expert launch starts on the published coresets
+    "decode_B16x4_p0": LAYER.with_(block_size=16, n_blocks=4),
+    "decode_B1x40_p0": LAYER.with_(block_size=1, n_blocks=40, bias_scale=0.0),
 }
 SAMPLED = {"T300_multi_ntile"}
 
