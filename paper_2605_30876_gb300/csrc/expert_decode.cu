@@ -190,6 +190,11 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     ptx::mbar_init(drain, 1);
     ptx::fence_mbarrier_init();
     *s_abort = 0;
+  } else if (tid == 32) {
+    // the descriptors of the first copies
+    const CUtensorMap* maps[7] = {&tm.wg32, &tm.wu32, &tm.wg, &tm.wu, &tm.x, &tm.sg32, &tm.su32};
+#pragma unroll
+    for (int i = 0; i < 7; ++i) ptx::prefetch_tensormap(maps[i]);
   }
   if (warp == 1) {
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
