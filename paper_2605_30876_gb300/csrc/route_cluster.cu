@@ -5,9 +5,9 @@
 //   1. logits: TMA brings the W_r slice (d/8 rows x 32 experts, 128-B rows) and the x
 //      slice (T rows x d/8); the W_r slice is split into three bf16 parts (hi + mid + lo
 //      = w to 2^-27, x * part exact in fp32) and tensor cores (mma.sync, fp32 accumulate)
-//      give the partial logits [T x 32] in shared memory;
-//      CTA r then adds, in rank order, the eight partials of the tokens t = r (mod 8) over
-//      distributed shared memory and writes those logits.
+//      give the partial logits [T x 32], pushed over distributed shared memory to the CTA
+//      that owns each token (t mod 8); CTA r then adds, in rank order, the eight partials of
+//      its tokens and writes those logits.
 //   2. one atomic ticket: the last cluster to finish continues; the others exit.
 //   3. scores: one warp per token (8 CTAs x 8 warps = 64 tokens): softmax, top-k (token
 //      mode: the routing; block mode: TopKMask, whose k nonzeros are stored straight into
@@ -90,16 +90,15 @@ __device__ __forceinline__ uint32_t peer_addr(const void* p, uint32_t rank) {
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(s_addr(p)), "r"(rank));
   return r;
 }
-__device__ __forceinline__ float ld_peer_f32(uint32_t addr) {
-  float v;
-  asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(addr) : "memory");
-  return v;
-}
 __device__ __forceinline__ void st_peer_u32(uint32_t addr, uint32_t v) {
   asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
 __device__ __forceinline__ void st_peer_f32(uint32_t addr, float v) {
   asm volatile("st.shared::cluster.f32 [%0], %1;" ::"r"(addr), "f"(v) : "memory");
+}
+__device__ __forceinline__ void st_peer_f32x2(uint32_t addr, float v0, float v1) {
+  asm volatile("st.shared::cluster.v2.f32 [%0], {%1, %2};" ::"r"(addr), "f"(v0), "f"(v1)
+               : "memory");
 }
 
 // Shared-memory layout after the logits (the W_r / x slices are dead by then), in bytes
@@ -134,7 +133,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   uint8_t* dsm = dsm_raw + ((1024u - (s_addr(dsm_raw) & 1023u)) & 1023u);
   __shared__ __align__(8) uint64_t s_bar;
   __shared__ uint32_t s_last;
-  __shared__ float s_part[kClMaxTok * kClExp];                     // partial logits [T][32]
+  // partial logits pushed by every CTA of the cluster to the owner of each token (token t:
+  // CTA t mod 8): [source rank][t / 8][32 experts]
+  __shared__ __align__(16) float s_part[kCl][kClMaxTok / kCl][kClExp];
   __shared__ float s_bias[kMaxExperts];
   __shared__ uint32_t s_loc[8][32];                  // one token's keys per warp
   __shared__ uint2 s_cand[8][kClMaxCand];            // merge: one token's candidates per warp
@@ -262,16 +263,13 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       float acc[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) acc[i] = (accp[0][i] + accp[1][i]) + accp[2][i];
-      // D rows r0, r0 + 8; columns 2tq, 2tq + 1 of the tile
+      // D rows r0, r0 + 8; columns 2tq, 2tq + 1 of the tile: to the owners of the tokens
       const int e = nt * 8 + 2 * tq;
-      if (r0 < T) {
-        s_part[r0 * kClExp + e] = acc[0];
-        s_part[r0 * kClExp + e + 1] = acc[1];
-      }
-      if (r0 + 8 < T) {
-        s_part[(r0 + 8) * kClExp + e] = acc[2];
-        s_part[(r0 + 8) * kClExp + e + 1] = acc[3];
-      }
+      if (r0 < T)
+        st_peer_f32x2(peer_addr(&s_part[rank][r0 >> 3][e], (uint32_t)(r0 & 7)), acc[0], acc[1]);
+      if (r0 + 8 < T)
+        st_peer_f32x2(peer_addr(&s_part[rank][(r0 + 8) >> 3][e], (uint32_t)((r0 + 8) & 7)),
+                      acc[2], acc[3]);
     }
   }
   __syncthreads();
@@ -280,7 +278,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     for (int i = tid; i < T * (kMaxExperts / 4); i += 256) hz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   CT_AT(2);
-  cluster_sync();
+  cluster_sync();   // every partial has reached its owner
   // CTA r adds the partials of tokens t = r (mod 8), in rank order, adds the bias, and keeps
   // the cluster's k best experts of the token (candidates for the top-k over all experts:
   // any expert of the top-k is among the k best of its own cluster)
@@ -288,32 +286,29 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   {
     const int t = (int)rank + 8 * warp;
     if (t < T) {
-      float p[kCl];
-#pragma unroll
-      for (uint32_t q = 0; q < (uint32_t)kCl; ++q)
-        p[q] = ld_peer_f32(peer_addr(&s_part[t * kClExp + lane], q));
       float v = 0.f;
 #pragma unroll
-      for (int q = 0; q < kCl; ++q) v += p[q];
+      for (int q = 0; q < kCl; ++q) v += s_part[q][warp][lane];
       const bool ok = e0 + lane < E;
       v += ok ? s_bias[e0 + lane] : 0.f;
       if (ok) a.logits_part[(size_t)t * E + e0 + lane] = v;
       const uint32_t key = ok ? order_key(v) : 0u;
       s_loc[warp][lane] = key;
       __syncwarp();
+      // rank among the cluster's 32 experts: larger key, ties to the lower lane (one 64-bit
+      // comparison of key and inverted lane)
+      const uint64_t mine = ((uint64_t)key << 32) | (uint32_t)(31 - lane);
       int r = 0;
 #pragma unroll 8
-      for (int j = 0; j < 32; ++j) {
-        const uint32_t kj = s_loc[warp][j];
-        r += (kj > key || (kj == key && j < lane)) ? 1 : 0;
-      }
+      for (int j = 0; j < 32; ++j)
+        r += ((((uint64_t)s_loc[warp][j]) << 32) | (uint32_t)(31 - j)) > mine ? 1 : 0;
       if (r < k)
         cand[((size_t)t * n_clusters + blockIdx.y) * k + r] =
             make_uint2(key, ok ? (uint32_t)(e0 + lane) : 0xffffffffu);
     }
   }
-  // every CTA of the cluster has written its logits and finished reading its peers' s_part
-  // (cluster scope); rank 0 then publishes the cluster at GPU scope
+  // every CTA of the cluster has written its logits and candidates (cluster scope); rank 0
+  // then publishes the cluster at GPU scope
   cluster_sync();
   CT_AT(3);
 
