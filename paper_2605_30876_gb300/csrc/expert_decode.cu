@@ -54,7 +54,8 @@ constexpr int kMaxTok = 64;                     // tokens of a decode-sized forw
 // g_dtrace[cta * 32 + slot] (globaltimer ns): 0 entry, 1 unit list known, 2 gate/up first
 // stage landed, 3 gate/up MMAs committed, 4 gate/up tile published, 5 down weights issued,
 // 6 H ready seen, 7 down MMAs committed, 8 down rows stored, 9 exit, 10 gate/up unit id,
-// 11 down unit id.
+// 11 down unit id, 12/13 first/last down stage landed, 14 down accumulator ready, 15 down
+// accumulator staged, 16 staging complete, 17 row copies issued.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_dtrace[kMaxPersistentCtas * 32];
 #define ED_AT(slot) (g_dtrace[blockIdx.x * 32 + (slot)] = ptx::globaltimer_ns())
@@ -96,6 +97,7 @@ struct DMaps {
   CUtensorMap x;             // x [T, d], n_pad-row boxes (rows >= T read as zeros)
   CUtensorMap h;             // hdense, n_pad-row boxes, 128-B swizzle (down B operand)
   CUtensorMap hst;           // hdense, 32 columns x n_pad rows, no swizzle (tile stores)
+  CUtensorMap ys, ysh;       // yslot [T*k, d], yshared [T, d] fp32: 128 columns x 8 rows
 };
 
 // One group of the forward.
@@ -135,6 +137,17 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, const void*
 __device__ __forceinline__ void bulk_commit_wait_all() {
   asm volatile("cp.async.bulk.commit_group;\n\tcp.async.bulk.wait_group 0;" ::: "memory");
 }
+// 1-D bulk copy of `bytes` (multiple of 16, both addresses 16-B aligned) from shared to
+// global memory, tracked by a bulk group
+__device__ __forceinline__ void bulk_store(void* gdst, const void* ssrc, uint32_t bytes) {
+  asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(gdst),
+               "r"(ptx::smem_addr(ssrc)), "r"(bytes)
+               : "memory");
+}
+// waits until the committed bulk copies have read their shared-memory sources
+__device__ __forceinline__ void bulk_commit_wait_read() {
+  asm volatile("cp.async.bulk.commit_group;\n\tcp.async.bulk.wait_group.read 0;" ::: "memory");
+}
 
 // AND of `v` over the 128 epilogue threads (named barrier 1), so that warp-collective TMEM
 // loads are taken by all of them or by none.
@@ -160,7 +173,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   const int SP = p.n_pad + 1;                     // floats per row of the down staging tile
   // ring of S slots [32 KB of weights | token boxes]; S and the slot size follow hg below
   uint8_t* ring = smem;
-  float* stage_t = reinterpret_cast<float*>(ring + p.ring_bytes);  // [128][SP]
+  // staging: a gate/up tile's H box, or a down tile as [token][128 rows] fp32 (128 x SP floats)
+  float* stage_t = reinterpret_cast<float*>(ring + p.ring_bytes);
   float* xchg = stage_t + kTileM * SP;
   int* tok = reinterpret_cast<int*>(xchg + 2 * 64 * kXStride);      // [kMaxTok]
   uint64_t* full = reinterpret_cast<uint64_t*>(tok + kMaxTok);
@@ -480,6 +494,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       for (int c = 0; c < nstages; ++c) {
         if (!wait(&full[stage], phase, value)) { ok = false; return; }
         if (gu && first && c == 0) ED_AT(2);
+        if (!gu && first && c == 0) ED_AT(12);
+        if (!gu && first && c == nstages - 1) ED_AT(13);
         ptx::tc_fence_after();
         const uint32_t a0 = ptx::smem_addr(slot_a(stage));
         const uint32_t b0 = ptx::smem_addr(slot_b(stage));
@@ -597,40 +613,55 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (!g.shared && et < g.n) tok[et] = __ldcg(p.rows + g.row0 + et) / p.k;
       const bool ok = epi_all(wait(&acc_full[acc], acc_phase, v));   // also orders tok[]
       if (!ok) break;
+      if (first && et == 0) ED_AT(14);
       ptx::tc_fence_after();
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
-      const int drow = i * kTileM + row;
-      if (g.shared) {
-        for (int c0 = 0; c0 < n_mma; c0 += 16) {
-          float vv[16];
-          ptx::tmem_ld16(tbase + c0, vv);
-          ptx::tmem_ld_wait();
+      // the accumulator column of token t is the group's output for t: the tile goes through
+      // shared memory as [token][128 rows] fp32, then one 512-B bulk copy per kept row (every
+      // token for the shared expert, the routed ones in dispatch order otherwise)
+      float* stg = stage_t;
+      for (int c0 = 0; c0 < n_mma; c0 += 16) {
+        float vv[16];
+        ptx::tmem_ld16(tbase + c0, vv);
+        ptx::tmem_ld_wait();
 #pragma unroll
-          for (int c = 0; c < 16; ++c)
-            if (c0 + c < p.T) p.yshared[(size_t)(c0 + c) * p.d + drow] = vv[c];
-        }
-      } else {
-        // the accumulator column of token t is the group's output for t: keep the routed
-        // ones, in dispatch order, through this thread's own staging row
-        float* srow = stage_t + row * SP;
-        for (int c0 = 0; c0 < n_mma; c0 += 16) {
-          float vv[16];
-          ptx::tmem_ld16(tbase + c0, vv);
-          ptx::tmem_ld_wait();
-#pragma unroll
-          for (int c = 0; c < 16; ++c) srow[c0 + c] = vv[c];
-        }
-        float* out = p.yslot + (size_t)g.row0 * p.d + drow;
-#pragma unroll 8
-        for (int r = 0; r < g.n; ++r) {
-          const int t = tok[r];
-          if (t >= 0 && t < p.T) out[(size_t)r * p.d] = srow[t];
-        }
+        for (int c = 0; c < 16; ++c)
+          if (c0 + c < p.T) stg[(c0 + c) * kTileM + row] = vv[c];
       }
       ptx::tc_fence_before();
       ptx::mbar_arrive(&acc_empty[acc]);
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
-      named_bar_sync(2, 128);   // tok[] is rewritten by the next unit
+      if (first && et == 0) ED_AT(15);
+      ptx::fence_proxy_async_smem();
+      named_bar_sync(2, 128);
+      if (et < 32) {
+        if (first && et == 0) ED_AT(16);
+        const int nrows = g.shared ? p.T : g.n;
+        // every token kept (the shared expert; a routed group that all T tokens use, whose
+        // dispatch rows are then tokens 0..T-1 in order): the staging tile is the rows' image,
+        // stored 8 rows per tensor copy; otherwise one 512-B row copy per lane
+        bool dense = nrows == p.T && (p.T & 7) == 0;
+        if (dense && !g.shared)
+          for (int r = et; r < nrows; r += 32) dense = dense && tok[r] == r;
+        dense = __all_sync(0xffffffffu, dense);
+        if (dense) {
+          if (et == 0)
+            for (int r8 = 0; r8 < nrows; r8 += 8)
+              tma_store_2d(g.shared ? &tm.ysh : &tm.ys, stg + r8 * kTileM, i * kTileM,
+                           (g.shared ? 0 : g.row0) + r8);
+        } else {
+          const size_t col = (size_t)i * kTileM;
+          for (int r = et; r < nrows; r += 32) {
+            const int t = g.shared ? r : tok[r];
+            float* dst = g.shared ? p.yshared + (size_t)r * p.d + col
+                                  : p.yslot + (size_t)(g.row0 + r) * p.d + col;
+            if (t >= 0 && t < p.T) bulk_store(dst, stg + t * kTileM, kTileM * 4);
+          }
+        }
+        if (first && et == 0) ED_AT(17);
+        bulk_commit_wait_read();   // the staging tile is rewritten by the next unit
+      }
+      named_bar_sync(2, 128);   // tok[] and the staging tile are rewritten by the next unit
       if (first && et == 0) ED_AT(8);
       first = false;
     }
@@ -684,6 +715,19 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
              estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
              plain ? CU_TENSOR_MAP_SWIZZLE_NONE : CU_TENSOR_MAP_SWIZZLE_128B,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// fp32 matrix [rows, cols] row-major, box = 128 columns x 8 rows, no swizzle.
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  const cuuint64_t dims[2] = {cols, rows};
+  const cuuint64_t strides[1] = {cols * 4};
+  const cuuint32_t box[2] = {(cuuint32_t)kTileM, 8};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // Opt-in shared memory per CTA; without a device (host-side planning) the sm_100-family
@@ -764,7 +808,9 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
             make_map(&m.h, a.hdense, (uint64_t)(a.E + 1) * n_pad, (uint64_t)imax,
                      (uint32_t)n_pad) &&
             make_map(&m.hst, a.hdense, (uint64_t)(a.E + 1) * n_pad, (uint64_t)imax,
-                     (uint32_t)n_pad, true, 32);
+                     (uint32_t)n_pad, true, 32) &&
+            make_map_f32(&m.ys, a.yslot, (uint64_t)a.T * a.k, a.d) &&
+            make_map_f32(&m.ysh, a.yshared, (uint64_t)a.T, a.d);
   if (ok && has_shared)
     ok = make_map(&m.sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
          make_map(&m.su, a.ws_up, (uint64_t)a.Is, a.d, 64) &&
