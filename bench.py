@@ -11,7 +11,9 @@ L2 honesty: the steps rotate over --sets independently seeded copies of the laye
 router and input), so consecutive steps never find their ~60 MB of expert weights in the
 129 MB L2. Steps are replayed from CUDA graphs (launch-bound otherwise).
 
-Prints one JSON line (rank 0). --impl reference times the CPU oracle instead.
+Prints one JSON line (rank 0). --impl reference times the CPU oracle instead. --suite
+measures the other workloads instead (one JSON line each): 8 sequences x 32 tokens, the
+block-size x batch x bias-scale grid, and the 20-layer stack of 64 x 32 tokens.
 """
 from __future__ import annotations
 
@@ -397,6 +399,118 @@ def run_reference(args, shape, rank):
     print(json.dumps(line), flush=True)
 
 
+# ----------------------------------------------------------------------------- suite
+def graph_time(torch, calls, target_s: float = 0.25) -> float:
+    """Device seconds per call of the `calls` (zero-argument functions), replayed from one
+    CUDA graph that runs them once each in order, after warm-up, over about target_s."""
+    for _ in range(2):
+        for f in calls:
+            f()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        for f in calls:
+            f()
+    st, en = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    g.replay()
+    st.record()
+    g.replay()
+    en.record()
+    torch.cuda.synchronize()
+    reps = int(max(3, min(5000, target_s / max(st.elapsed_time(en) * 1e-3, 1e-7))))
+    for _ in range(2):
+        g.replay()
+    st.record()
+    for _ in range(reps):
+        g.replay()
+    en.record()
+    torch.cuda.synchronize()
+    return st.elapsed_time(en) * 1e-3 / reps / len(calls)
+
+
+def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
+    """The other workloads, one JSON line per point: 8 sequences x 32 tokens (block p = 0,
+    block p = 0.6, token routing), the block-size x batch x bias-scale grid (block p = 0 and
+    token routing), and the 20-layer residual stack of 64 x 32 tokens (block p = 0 and token
+    routing; x_{l+1} = bf16(x_l + y_l), the add by torch). The single-layer points rotate over
+    --sets seeded copies of the layer's weights, as the headline does."""
+    from dmoe_synth import (LAYER, LAYER_B8, ROUTE_BLOCK, ROUTE_TOKEN, STACK20, STACK20_LAYERS,
+                            layer_inputs, router_bias, sweep_shapes)
+
+    def emit(line):
+        print(json.dumps(line), flush=True)
+
+    def stats(shape, sec, U):
+        lb = layer_bytes(shape, U)
+        fl = layer_flops(shape)
+        return {"us_per_forward": sec * 1e6, "tokens_per_s": shape.T / sec,
+                "unique_experts_mean": U, "bytes_per_forward": lb,
+                "achieved_gbs": lb / sec / 1e9, "hbm_roofline_frac": lb / sec / 1e9 / hbm,
+                "flops_per_forward": fl, "tensor_frac": fl / sec / 1e12 / bf16_peak}
+
+    def label(shape):
+        return ("token" if shape.mode == ROUTE_TOKEN else f"block_p{shape.top_p:g}")
+
+    sets = [layer_inputs(LAYER, seed=args.seed + s, device="cuda") for s in range(args.sets)]
+
+    def point(suite, shape):
+        layers, xs = [], []
+        for s, w0 in enumerate(sets):
+            w = dict(w0)
+            w["bias"] = torch.from_numpy(router_bias(shape.n_experts, shape.bias_scale,
+                                                     args.seed + s)).to("cuda")
+            layers.append(MoELayer.from_shape(shape, w))
+            xs.append(layer_inputs(shape, seed=args.seed + s, device="cuda",
+                                   with_weights=False)["x"])
+        sec = graph_time(torch, [lambda L=L, x=x: L.forward(x) for L, x in zip(layers, xs)])
+        for L in layers:
+            st, info = dm.dmoe_get_device_error(L.ws)
+            if st != 0:
+                raise RuntimeError(f"device fault {info}")
+        U = float(np.mean([int(L.n_unique.item()) for L in layers]))
+        emit({"suite": suite, "workload": workload_name(shape), "routing": label(shape),
+              "block_size": shape.block_size, "batch": shape.n_blocks,
+              "bias_scale": shape.bias_scale, "T": shape.T, **stats(shape, sec, U)})
+
+    for mode, p in ((ROUTE_BLOCK, 0.0), (ROUTE_BLOCK, 0.6), (ROUTE_TOKEN, 0.0)):
+        point("8x32", LAYER_B8.with_(mode=mode, top_p=p))
+    for mode in (ROUTE_BLOCK, ROUTE_TOKEN):
+        for shape in sweep_shapes(mode=mode):
+            point("grid", shape)
+    del sets
+    torch.cuda.empty_cache()
+
+    # the stack: separate seeded weights per layer, shared by the two routings
+    weights = [layer_inputs(STACK20, seed=args.seed + 1000 + l, device="cuda", layer=l)
+               for l in range(STACK20_LAYERS)]
+    x0 = layer_inputs(STACK20, seed=args.seed + 999, device="cuda", with_weights=False)["x"]
+    for mode in (ROUTE_BLOCK, ROUTE_TOKEN):
+        shape = STACK20.with_(mode=mode, top_p=0.0)
+        layers = [MoELayer.from_shape(shape, w) for w in weights]
+        xs = [x0] + [torch.empty_like(x0) for _ in range(STACK20_LAYERS)]
+
+        def step():
+            for l, L in enumerate(layers):
+                y = L.forward(xs[l])
+                torch.add(xs[l], y, out=xs[l + 1])
+
+        sec = graph_time(torch, [step]) / STACK20_LAYERS
+        for L in layers:
+            st, info = dm.dmoe_get_device_error(L.ws)
+            if st != 0:
+                raise RuntimeError(f"device fault {info}")
+        per_layer = [int(L.n_unique.item()) for L in layers]
+        U = float(np.mean(per_layer))
+        line = {"suite": "stack20", "workload": workload_name(shape), "routing": label(shape),
+                "layers": STACK20_LAYERS, "T": shape.T, "us_per_step": sec * STACK20_LAYERS * 1e6,
+                "step_tokens_per_s": shape.T / (sec * STACK20_LAYERS), **stats(shape, sec, U),
+                "unique_experts_per_layer": per_layer,
+                "note": "per-layer figures include the residual add"}
+        emit(line)
+        del layers
+    del weights
+
+
 # ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -413,6 +527,9 @@ def main():
     ap.add_argument("--ref-budget", type=float, default=90.0)
     ap.add_argument("--only-headline", action="store_true",
                     help="skip the e2e and side-by-side arms (small profiling runs)")
+    ap.add_argument("--suite", action="store_true",
+                    help="measure the other workloads instead of the headline (one JSON line "
+                         "per point; one GPU)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -438,6 +555,10 @@ def main():
 
     peaks, peak_src = measured_peaks()
     hbm = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    if args.suite:
+        run_suite(args, torch, dm, MoELayer, hbm,
+                  float(peaks.get("bf16_tflops_sustained", 1700.0)))
+        return
     sampler = ClockSampler(gpu_uuid(torch)) if rank == 0 else None
 
     # headline: block routing, p = 0
