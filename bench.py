@@ -432,8 +432,9 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
     """The other workloads, one JSON line per point: 8 sequences x 32 tokens (block p = 0,
     block p = 0.6, token routing), the block-size x batch x bias-scale grid (block p = 0 and
     token routing), and the 20-layer residual stack of 64 x 32 tokens (block p = 0 and token
-    routing; x_{l+1} = bf16(x_l + y_l), the add by torch). The single-layer points rotate over
-    --sets seeded copies of the layer's weights, as the headline does."""
+    routing; each layer fed the RMS-normalised stream, u_l = bf16(x_l / rms(x_l)), and
+    x_{l+1} = bf16(x_l + y_l), both by torch). The single-layer points rotate over --sets
+    seeded copies of the layer's weights, as the headline does."""
     from dmoe_synth import (LAYER, LAYER_B8, ROUTE_BLOCK, ROUTE_TOKEN, STACK20, STACK20_LAYERS,
                             layer_inputs, router_bias, sweep_shapes)
 
@@ -488,10 +489,13 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
         shape = STACK20.with_(mode=mode, top_p=0.0)
         layers = [MoELayer.from_shape(shape, w) for w in weights]
         xs = [x0] + [torch.empty_like(x0) for _ in range(STACK20_LAYERS)]
+        us = [torch.empty_like(x0) for _ in range(STACK20_LAYERS)]
 
         def step():
             for l, L in enumerate(layers):
-                y = L.forward(xs[l])
+                xf = xs[l].float()
+                us[l].copy_(xf * torch.rsqrt(xf.pow(2).mean(-1, keepdim=True)))
+                y = L.forward(us[l])
                 torch.add(xs[l], y, out=xs[l + 1])
 
         sec = graph_time(torch, [step]) / STACK20_LAYERS
@@ -505,7 +509,7 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
                 "layers": STACK20_LAYERS, "T": shape.T, "us_per_step": sec * STACK20_LAYERS * 1e6,
                 "step_tokens_per_s": shape.T / (sec * STACK20_LAYERS), **stats(shape, sec, U),
                 "unique_experts_per_layer": per_layer,
-                "note": "per-layer figures include the residual add"}
+                "note": "per-layer figures include the torch RMS norm and residual add"}
         emit(line)
         del layers
     del weights
