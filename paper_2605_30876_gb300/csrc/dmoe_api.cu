@@ -17,6 +17,7 @@ size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 // (about 128 tiles), a divisor of d/32, at most 32 partial sums.
 int router_splits(const dmoe_layer_desc& d) {
   if (route_cluster_ok(d.n_blocks * d.block_size, d.d_model, d.n_experts)) return 0;
+  if (route_cluster_logits_ok(d.d_model, d.n_experts)) return 1;   // one [T, E] logits array
   const int tiles = ((d.n_experts + 63) / 64) * ((d.n_blocks * d.block_size + 31) / 32);
   int target = 128 / tiles;
   if (target < 1) target = 1;

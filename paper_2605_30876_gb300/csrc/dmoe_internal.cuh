@@ -175,6 +175,10 @@ cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s);
 cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                           cudaStream_t s);
 bool route_cluster_ok(int T, int d, int E);
+// The logits stage of that launch alone, over tiles of 64 tokens (any T): logits + bias
+// into a.logits_part [T, E] (no split).
+bool route_cluster_logits_ok(int d, int E);
+cudaError_t launch_logits_cluster(const RouterArgs& a, cudaStream_t s);
 cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                                  cudaStream_t s);
 

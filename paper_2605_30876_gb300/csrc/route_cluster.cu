@@ -70,6 +70,8 @@ struct ClusterArgs {
   RouterArgs r;
   DispatchArgs dsp;   // dsp.n_unique == nullptr: no dispatch
   int32_t* ticket;    // zero between calls
+  int box_rows;       // token rows of an x box (a multiple of 16, at most kClMaxTok)
+  int logits_only;    // tile z of kClMaxTok tokens: stop once the logits are written
 };
 
 __device__ __forceinline__ uint32_t s_addr(const void* p) {
@@ -141,7 +143,12 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   __shared__ uint2 s_cand[8][kClMaxCand];            // merge: one token's candidates per warp
   const RouterArgs& a = f.r;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int T = a.T, E = a.E, k = a.k, B = a.B;
+  // logits-only launches take the tokens in tiles of kClMaxTok (blockIdx.z); otherwise
+  // z = 0 and the tile is the whole forward
+  const int tz = blockIdx.z * kClMaxTok;
+  const int T = a.T - tz < kClMaxTok ? a.T - tz : kClMaxTok;
+  const int E = a.E, k = a.k, B = a.B;
+  const int TB = f.box_rows;
   const uint32_t rank = cluster_rank();
   const int DC = a.d / kCl;                          // rows of d in this CTA's slice
   const int e0 = blockIdx.y * kClExp;
@@ -156,7 +163,8 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
                      reinterpret_cast<uint64_t>(&f.wmap)),
                  "r"(e0), "r"((int)rank * DC)
                  : "memory");
-    issue_shared_prefetch(a.shared_pf, blockIdx.y * kCl + (int)rank, gridDim.x * gridDim.y);
+    issue_shared_prefetch(a.shared_pf, (blockIdx.z * gridDim.y + blockIdx.y) * kCl + (int)rank,
+                          gridDim.x * gridDim.y * gridDim.z);
   }
   pdl_wait();
   // the expert launch may start now (not earlier: it reads the early coreset counter, which
@@ -167,13 +175,13 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 
   // ---- 1. partial logits over this CTA's slice of d
   float* Ws = reinterpret_cast<float*>(dsm);                                   // [DC][32]
-  // x slice: boxes of 64 columns x T16 rows with the 128-byte swizzle
+  // x slice: boxes of 64 columns x TB rows with the 128-byte swizzle
   uint8_t* Xs = dsm + kClMaxDChunk * kClExp * 4;
   const int T16 = (T + 15) & ~15, nxb = (DC + 63) / 64;
   if (tid == 0) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(s_addr(&s_bar)) : "memory");
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)nxb * T16 * 128;
+    const uint32_t bytes = (uint32_t)DC * kClExp * 4 + (uint32_t)nxb * TB * 128;
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(s_addr(&s_bar)),
                  "r"(bytes)
                  : "memory");
@@ -186,9 +194,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     for (int bx = 0; bx < nxb; ++bx)
       asm volatile(
           "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
-          " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Xs) + (uint32_t)(bx * T16 * 128)),
+          " [%0], [%1, {%3, %4}], [%2];" ::"r"(s_addr(Xs) + (uint32_t)(bx * TB * 128)),
           "l"(reinterpret_cast<uint64_t>(&f.xmap)), "r"(s_addr(&s_bar)),
-          "r"((int)rank * DC + 64 * bx), "r"(0)
+          "r"((int)rank * DC + 64 * bx), "r"(tz)
           : "memory");
   }
   for (int e = tid; e < E; e += 256) s_bias[e] = a.bias != nullptr ? a.bias[e] : 0.f;
@@ -247,7 +255,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 #pragma unroll 2
       for (int k0 = 0; k0 < DC; k0 += 16) {
         const int bx = k0 >> 6, c = (k0 & 63) >> 3;   // box, 16-B chunk of k0
-        const uint8_t* xb = Xs + bx * T16 * 128;
+        const uint8_t* xb = Xs + bx * TB * 128;
         uint32_t af[4];
         af[0] = *reinterpret_cast<const uint32_t*>(xb + r0 * 128 + ((c ^ (r0 & 7)) << 4) + tq * 4);
         af[1] = *reinterpret_cast<const uint32_t*>(xb + (r0 + 8) * 128 + ((c ^ (r0 & 7)) << 4) + tq * 4);
@@ -275,7 +283,8 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   __syncthreads();
   {  // TopKMask rows start as zeros (scoring warps anywhere in the cluster add the winners)
     float4* hz = reinterpret_cast<float4*>(dsm + kOffHat);
-    for (int i = tid; i < T * (kMaxExperts / 4); i += 256) hz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (!f.logits_only)
+      for (int i = tid; i < T * (kMaxExperts / 4); i += 256) hz[i] = make_float4(0.f, 0.f, 0.f, 0.f);
   }
   CT_AT(2);
   cluster_sync();   // every partial has reached its owner
@@ -291,26 +300,29 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       for (int q = 0; q < kCl; ++q) v += s_part[q][warp][lane];
       const bool ok = e0 + lane < E;
       v += ok ? s_bias[e0 + lane] : 0.f;
-      if (ok) a.logits_part[(size_t)t * E + e0 + lane] = v;
-      const uint32_t key = ok ? order_key(v) : 0u;
-      s_loc[warp][lane] = key;
-      __syncwarp();
-      // rank among the cluster's 32 experts: larger key, ties to the lower lane (one 64-bit
-      // comparison of key and inverted lane)
-      const uint64_t mine = ((uint64_t)key << 32) | (uint32_t)(31 - lane);
-      int r = 0;
+      if (ok) a.logits_part[(size_t)(tz + t) * E + e0 + lane] = v;
+      if (!f.logits_only) {
+        const uint32_t key = ok ? order_key(v) : 0u;
+        s_loc[warp][lane] = key;
+        __syncwarp();
+        // rank among the cluster's 32 experts: larger key, ties to the lower lane (one
+        // 64-bit comparison of key and inverted lane)
+        const uint64_t mine = ((uint64_t)key << 32) | (uint32_t)(31 - lane);
+        int r = 0;
 #pragma unroll 8
-      for (int j = 0; j < 32; ++j)
-        r += ((((uint64_t)s_loc[warp][j]) << 32) | (uint32_t)(31 - j)) > mine ? 1 : 0;
-      if (r < k)
-        cand[((size_t)t * n_clusters + blockIdx.y) * k + r] =
-            make_uint2(key, ok ? (uint32_t)(e0 + lane) : 0xffffffffu);
+        for (int j = 0; j < 32; ++j)
+          r += ((((uint64_t)s_loc[warp][j]) << 32) | (uint32_t)(31 - j)) > mine ? 1 : 0;
+        if (r < k)
+          cand[((size_t)t * n_clusters + blockIdx.y) * k + r] =
+              make_uint2(key, ok ? (uint32_t)(e0 + lane) : 0xffffffffu);
+      }
     }
   }
   // every CTA of the cluster has written its logits and candidates (cluster scope); rank 0
   // then publishes the cluster at GPU scope
   cluster_sync();
   CT_AT(3);
+  if (f.logits_only) return;
 
   // ---- 2. the last cluster to finish routes the forward
   if (rank == 0 && tid == 0) {
@@ -558,13 +570,32 @@ extern "C" int dmoe_debug_ctrace_clear() {
 }
 #endif
 
-bool route_cluster_ok(int T, int d, int E) {
+bool route_cluster_logits_ok(int d, int E) {
   // d % 256: each CTA's slice splits into eight runs of whole float4 groups
-  return T <= kClMaxTok && d % (kCl * 32) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
+  return d % (kCl * 32) == 0 && d / kCl <= kClMaxDChunk && E % 8 == 0;
+}
+
+bool route_cluster_ok(int T, int d, int E) {
+  return T <= kClMaxTok && route_cluster_logits_ok(d, E);
+}
+
+namespace {
+cudaError_t launch_cluster_common(const RouterArgs& a, const DispatchArgs* dsp,
+                                  int32_t* tickets, cudaStream_t s, bool logits_only);
 }
 
 cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                                  cudaStream_t s) {
+  return launch_cluster_common(a, dsp, tickets, s, false);
+}
+
+cudaError_t launch_logits_cluster(const RouterArgs& a, cudaStream_t s) {
+  return launch_cluster_common(a, nullptr, nullptr, s, true);
+}
+
+namespace {
+cudaError_t launch_cluster_common(const RouterArgs& a, const DispatchArgs* dsp,
+                                  int32_t* tickets, cudaStream_t s, bool logits_only) {
   EncodeTiledFnC enc = encoder();
   if (enc == nullptr) return cudaErrorInvalidValue;
   ClusterArgs f{};
@@ -582,7 +613,8 @@ cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, i
   {
     const cuuint64_t dims[2] = {(cuuint64_t)a.d, (cuuint64_t)a.T};
     const cuuint64_t strides[1] = {(cuuint64_t)a.d * 2};
-    const cuuint32_t box[2] = {64u, (cuuint32_t)((a.T + 15) & ~15)};
+    f.box_rows = logits_only ? kClMaxTok : (a.T + 15) & ~15;
+    const cuuint32_t box[2] = {64u, (cuuint32_t)f.box_rows};
     const cuuint32_t estr[2] = {1, 1};
     if (enc(&f.xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<__nv_bfloat16*>(a.x), dims,
             strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -592,6 +624,7 @@ cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, i
   f.r = a;
   if (dsp != nullptr) f.dsp = *dsp;
   f.ticket = tickets;
+  f.logits_only = logits_only ? 1 : 0;
   const size_t smem = route_cluster_smem();
   static int mask = 0;
   int dev = 0;
@@ -602,10 +635,12 @@ cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, i
     if (e != cudaSuccess) return e;
     if (dev < 31) mask |= 1 << dev;
   }
-  dim3 grid(kCl, (a.E + kClExp - 1) / kClExp);
+  dim3 grid(kCl, (a.E + kClExp - 1) / kClExp,
+            logits_only ? (a.T + kClMaxTok - 1) / kClMaxTok : 1);
   // programmatic dependent launch: the set-up overlaps the previous kernel on the stream;
   // the kernel waits for it (griddepcontrol.wait) before it reads anything
   return launch_cluster(route_cluster_kernel, grid, dim3(256), smem, s, kCl, true, f);
 }
+}  // namespace
 
 }  // namespace dmoe

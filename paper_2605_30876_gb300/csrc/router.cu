@@ -2,7 +2,10 @@
 //
 // Decode-sized batches take the single cluster launch of route_cluster.cu. Larger batches
 // use one kernel per step:
-//   router_logits_kernel   logits = x W_r, fp32 FFMA, 32 x 64 tiles, optional split over d
+//   logits                 the logits stage of the cluster launch over 64-token tiles
+//                          (tensor cores, exact bf16 split of W_r), or where its shape rules
+//                          do not hold, router_logits_kernel: fp32 FFMA, 32 x 64 tiles,
+//                          optional split over d
 //   router_softmax_kernel  one warp per token: sum the partials in split order, + b,
 //                          softmax, top-k
 //   block_route_kernel     one CTA per diffusion block: Algorithm 1 (routing_device.cuh)
@@ -117,13 +120,21 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
     e = launch_route_cluster(a, dsp, tickets, s);
     if (e != cudaSuccess) return e;
   } else {
-    const int dchunk = a.d / a.splits;
-    dim3 g1((a.E + kRtExp - 1) / kRtExp, (a.T + kRtTok - 1) / kRtTok, a.splits);
-    router_logits_kernel<<<g1, 256, 0, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E, dchunk,
-                                            a.shared_pf);
+    // logits (+ bias) on tensor cores in the cluster launch when the shape allows it, else
+    // the FFMA tiles with partial sums over a split of d
+    const bool cl = route_cluster_logits_ok(a.d, a.E);
+    if (cl) {
+      e = launch_logits_cluster(a, s);
+      if (e != cudaSuccess) return e;
+    } else {
+      const int dchunk = a.d / a.splits;
+      dim3 g1((a.E + kRtExp - 1) / kRtExp, (a.T + kRtTok - 1) / kRtTok, a.splits);
+      router_logits_kernel<<<g1, 256, 0, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E, dchunk,
+                                              a.shared_pf);
+    }
     e = launch_ex(router_softmax_kernel, dim3((a.T + 7) / 8), dim3(256), 0, s, true,
-                  a.logits_part, a.splits, a.bias, a.probs, a.probs_hat, a.topk_idx,
-                  a.topk_gate, a.T, a.E, a.k, a.mode);
+                  a.logits_part, cl ? 1 : a.splits, cl ? nullptr : a.bias, a.probs, a.probs_hat,
+                  a.topk_idx, a.topk_gate, a.T, a.E, a.k, a.mode);
     if (e != cudaSuccess) return e;
     if (a.mode == DMOE_ROUTE_BLOCK) {
       e = launch_ex(block_route_kernel, dim3(a.n_blocks), dim3(256), 0, s, true, a.probs,
