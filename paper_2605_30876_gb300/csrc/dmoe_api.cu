@@ -39,13 +39,21 @@ struct ProfSlot {
 thread_local ProfSlot g_prof[DMOE_KERNEL_COUNT];
 }  // namespace
 
+// Inside a stream capture the event becomes an external record node of the graph (recorded
+// at every replay); outside, a plain record.
+void prof_record(cudaEvent_t ev, cudaStream_t s) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(s, &cs) != cudaSuccess) cudaGetLastError();
+  if (cs == cudaStreamCaptureStatusActive)
+    cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal);
+  else
+    cudaEventRecord(ev, s);
+}
 void prof_begin(int kernel, cudaStream_t s) {
-  if (g_prof[kernel].begin != nullptr)
-    cudaEventRecordWithFlags(g_prof[kernel].begin, s, cudaEventRecordExternal);
+  if (g_prof[kernel].begin != nullptr) prof_record(g_prof[kernel].begin, s);
 }
 void prof_end(int kernel, cudaStream_t s) {
-  if (g_prof[kernel].end != nullptr)
-    cudaEventRecordWithFlags(g_prof[kernel].end, s, cudaEventRecordExternal);
+  if (g_prof[kernel].end != nullptr) prof_record(g_prof[kernel].end, s);
 }
 
 void set_last_error(cudaError_t e) {

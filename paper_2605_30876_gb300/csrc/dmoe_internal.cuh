@@ -85,10 +85,13 @@ struct Workspace {
   int n_max;           // token tile (MMA N) of the expert GEMMs
 };
 
-// Token tile of the expert GEMMs: every group's rows are covered by tiles of n_max.
+// Token tile (MMA N) of the general expert kernel: every group's rows are covered by tiles
+// of n_max; 64 rows up to 256 tokens per forward, 128 above (measured: wider tiles leave two
+// pipeline stages in shared memory, narrower ones re-stream the weights for more tiles).
 inline int expert_n_max(int T) {
+  const int cap = T <= 256 ? 64 : 128;
   int n = ((T + 15) / 16) * 16;
-  return n > 256 ? 256 : (n < 16 ? 16 : n);
+  return n > cap ? cap : (n < 16 ? 16 : n);
 }
 
 Workspace plan_workspace(const dmoe_layer_desc& d);
