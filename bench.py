@@ -282,7 +282,8 @@ def traffic_from_profile(kernel: str, source: str):
         for ln in open(path):
             if ":" in ln:
                 k, v = ln.split(":", 1)
-                vals[k.strip()] = v.strip()
+                v = v.split()
+                vals[k.strip()] = v[0] if v else ""   # the value's first word
         if vals.get("source_sha256_16") != h:
             return None
         return float(vals["dram_bytes_per_launch"])
