@@ -49,6 +49,8 @@ def workload_shape(mode: str, top_p: float):
 def workload_name(shape) -> str:
     mode = "block" if shape.mode == 1 else "token"
     tail = f"_p{shape.top_p:g}" if shape.mode == 1 else ""
+    if shape.mode == 1 and getattr(shape, "block_top_k", 0):
+        tail += f"_mask{shape.block_top_k}"
     return (f"moe_layer_d{shape.d_model}_E{shape.n_experts}_k{shape.top_k}_I{shape.d_ff}"
             f"_shared{shape.d_ff_shared}_B{shape.block_size}x{shape.n_blocks}_{mode}{tail}")
 
@@ -431,7 +433,9 @@ def graph_time(torch, calls, target_s: float = 0.25) -> float:
 
 def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
     """The other workloads, one JSON line per point: 8 sequences x 32 tokens (block p = 0,
-    block p = 0.6, token routing), the block-size x batch x bias-scale grid (block p = 0 and
+    block p = 0.6, token routing), a sweep of the coreset threshold p with a line fitted to
+    latency against unique experts, fewer experts per token inside the coreset and the Top-4
+    token baseline, the block-size x batch x bias-scale grid (block p = 0 and
     token routing), and the 20-layer residual stack of 64 x 32 tokens (block p = 0 and token
     routing; each layer fed the RMS-normalised stream, u_l = bf16(x_l / rms(x_l)), and
     x_{l+1} = bf16(x_l + y_l), both by torch). The single-layer points rotate over --sets
@@ -451,7 +455,12 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
                 "flops_per_forward": fl, "tensor_frac": fl / sec / 1e12 / bf16_peak}
 
     def label(shape):
-        return ("token" if shape.mode == ROUTE_TOKEN else f"block_p{shape.top_p:g}")
+        base = "token" if shape.mode == ROUTE_TOKEN else f"block_p{shape.top_p:g}"
+        if shape.top_k != LAYER.top_k:
+            base += f"_k{shape.top_k}"
+        if shape.mode == ROUTE_BLOCK and shape.block_top_k:
+            base += f"_of{shape.block_top_k}"
+        return base
 
     sets = [layer_inputs(LAYER, seed=args.seed + s, device="cuda") for s in range(args.sets)]
 
@@ -473,9 +482,32 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
         emit({"suite": suite, "workload": workload_name(shape), "routing": label(shape),
               "block_size": shape.block_size, "batch": shape.n_blocks,
               "bias_scale": shape.bias_scale, "T": shape.T, **stats(shape, sec, U)})
+        return sec, U
 
     for mode, p in ((ROUTE_BLOCK, 0.0), (ROUTE_BLOCK, 0.6), (ROUTE_TOKEN, 0.0)):
         point("8x32", LAYER_B8.with_(mode=mode, top_p=p))
+    # the coreset threshold as a performance axis: p over the paper's sweep values at block
+    # size 32 and four batch sizes, with block top-k and token routing as the two ends; per
+    # batch, a least-squares line of latency against the unique-expert count
+    for nb in (1, 4, 16, 32):
+        pts = []
+        shapes = ([LAYER.with_(n_blocks=nb, top_p=p) for p in (0.0, 0.4, 0.5, 0.6, 0.7, 0.8)]
+                  + [LAYER.with_(n_blocks=nb, mode=ROUTE_TOKEN)])
+        for shape in shapes:
+            pts.append(point("top_p_sweep", shape))
+        sec_, U_ = np.array([q[0] for q in pts]) * 1e6, np.array([q[1] for q in pts])
+        slope, icpt = np.polyfit(U_, sec_, 1)
+        fit = slope * U_ + icpt
+        r2 = 1.0 - float(np.sum((sec_ - fit) ** 2) / max(np.sum((sec_ - sec_.mean()) ** 2), 1e-30))
+        emit({"suite": "top_p_sweep_fit", "batch": nb, "T": 32 * nb, "points": len(pts),
+              "us_per_unique_expert": float(slope), "us_at_zero_experts": float(icpt),
+              "r2": r2, "hbm_us_per_expert": LAYER.expert_bytes() / hbm / 1e3})
+    # fewer experts per token inside the block's coreset (App. A) and the Top-4 token
+    # baseline, at 1 and 8 sequences of 32 tokens
+    for nb in (1, 8):
+        for kw in (dict(top_k=4, block_top_k=8), dict(top_k=2, block_top_k=8),
+                   dict(top_k=4, block_top_k=8, top_p=0.6), dict(top_k=4, mode=ROUTE_TOKEN)):
+            point("fewer_experts", LAYER.with_(n_blocks=nb, **kw))
     for mode in (ROUTE_BLOCK, ROUTE_TOKEN):
         for shape in sweep_shapes(mode=mode):
             point("grid", shape)

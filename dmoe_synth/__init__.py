@@ -51,7 +51,9 @@ class MoEShape:
     block_size: diffusion block size B; n_blocks: blocks per forward (one per sequence);
     mode: ROUTE_BLOCK or ROUTE_TOKEN; top_p: coreset threshold p (0 => coreset of size k,
     i.e. block top-k; >= 1 => every expert with a nonzero block score);
-    bias_scale: s in b_e = s * ln(1/rank_e).
+    bias_scale: s in b_e = s * ln(1/rank_e); block_top_k: block mode, the k of TopKMask and
+    of the coreset floor when every token keeps only top_k < block_top_k members of its
+    coreset (0 = top_k).
     """
     d_model: int
     n_experts: int
@@ -63,6 +65,7 @@ class MoEShape:
     mode: int = ROUTE_BLOCK
     top_p: float = 0.0
     bias_scale: float = 0.0
+    block_top_k: int = 0
 
     @property
     def T(self) -> int:

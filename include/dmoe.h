@@ -38,7 +38,7 @@
 extern "C" {
 #endif
 
-#define DMOE_ABI_VERSION 1
+#define DMOE_ABI_VERSION 2
 
 typedef enum {
   DMOE_OK = 0,
@@ -57,6 +57,7 @@ typedef enum {
 
 /* Shape and routing parameters of one MoE-layer forward (plain data, host memory).
  * Limits of this build: 1 <= k <= 16, k <= E <= 256, E % 8 == 0; d % 128 == 0,
+ * block_top_k = 0 or k <= block_top_k <= min(E, 16);
  * 128 <= d <= 16384; I % 128 == 0 and I_s % 128 == 0 (I_s may be 0), I, I_s <= 8192;
  * 1 <= T <= 4096; block_size >= 1. */
 typedef struct {
@@ -70,9 +71,17 @@ typedef struct {
   int32_t mode;           /* dmoe_route_mode                                         */
   float top_p;            /* block mode: coreset threshold p. The coreset is the
                              shortest prefix of the experts sorted by normalised block
-                             score whose running sum reaches p, extended to at least k
-                             entries; p <= 0 gives exactly k (block top-k), p >= 1 every
+                             score whose running sum reaches p, extended to at least
+                             block_top_k entries; p <= 0 gives exactly block_top_k (block
+                             top-k), p >= 1 every
                              expert with a nonzero block score. Ignored in token mode. */
+  int32_t block_top_k;    /* block mode: the k of Algorithm 1's TopKMask (the per-token
+                             contribution to the block score) and of the coreset floor;
+                             0 means top_k. A value above top_k keeps Algorithm 1's
+                             coreset but lets every token use only the top_k best members
+                             of it by its own score (the "fewer experts for each token"
+                             direction of App. A); then top_k <= block_top_k <= min(E, 16).
+                             Ignored in token mode. */
 } dmoe_layer_desc;
 
 /* Bytes of device workspace needed by every call below for this shape (host only; no

@@ -32,6 +32,10 @@ Readings (the paper is silent or ambiguous here):
   R10 expert:   SwiGLU, y_e(x) = W_down (silu(W_gate x) * (W_up x)), fp64 throughout, with
                 the intermediate kept unrounded. Token-level routing (the "Original"
                 baseline of §5.1) is R_i = TopK(s_i, k) with the same gates.
+  R11 fewer experts per token (the direction App. A names, not evaluated in the paper):
+                Algorithm 1 runs with k_mask in TopKMask and in the floor, and the final
+                TopK inside the coreset keeps k < k_mask experts per token, gates R8 over
+                those k. k_mask = k is Algorithm 1 itself.
 
 Decisions (a top-k, the coreset boundary) are taken on fp32 values, as the router's
 fp32 output is the input of Algorithm 1. Each decision also reports a *margin*: how far
@@ -234,11 +238,19 @@ def route_token(s: np.ndarray, k: int) -> Routing:
     return Routing(idx, gate, [], sm, om, np.zeros(0), s)
 
 
-def route_block(s: np.ndarray, k: int, block_size: int, p: float) -> Routing:
+def route_block(s: np.ndarray, k: int, block_size: int, p: float,
+                k_mask: Optional[int] = None) -> Routing:
     """Algorithm 1 applied to every block of ``block_size`` consecutive tokens; blocks are
-    routed independently. Returns R_i for every token with the R8 gates."""
+    routed independently. Returns R_i for every token with the R8 gates.
+
+    ``k_mask`` (default k) is the k of TopKMask and of the floor (R6); the final TopK keeps
+    k <= k_mask members of the coreset per token (R11: App. A's "fewer experts for each
+    token"). The block's margin also covers every TopKMask decision of its tokens: a near
+    tie at a token's k_mask-th score can move that score to another expert of S_block."""
     T, E = s.shape
     assert T % block_size == 0
+    km = k if k_mask is None or k_mask <= 0 else int(k_mask)
+    assert 1 <= k <= km <= E
     nb = T // block_size
     idx = np.zeros((T, k), np.int32)
     gate = np.zeros((T, k), F64)
@@ -248,11 +260,12 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float) -> Routing:
     coresets = []
     for b in range(nb):
         rows = slice(b * block_size, (b + 1) * block_size)
-        S = aggregate(s[rows], k)                     # Algorithm 1: S_block
+        S = aggregate(s[rows], km)                    # Algorithm 1: S_block
         S_tilde = normalize(S)                        # Algorithm 1: Normalize
-        C = top_p(S_tilde, p, k)                      # Algorithm 1: TopP (+ floor)
+        C = top_p(S_tilde, p, km)                     # Algorithm 1: TopP (+ floor)
         coresets.append(C.ids)
-        cm[b] = C.margin
+        mask_margin = min(topk_margins(s[i], km)[0] for i in range(b * block_size, (b + 1) * block_size))
+        cm[b] = min(C.margin, mask_margin)
         for i in range(b * block_size, (b + 1) * block_size):
             sC = mask_outside(s[i], C.ids)            # Algorithm 1: MaskOutside
             R = topk_desc(sC, k)                      # Algorithm 1: TopK
@@ -262,12 +275,14 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float) -> Routing:
     return Routing(idx, gate, coresets, sm, om, cm, s)
 
 
-def route(x_bits, w_r, bias, k: int, mode: int, block_size: int, p: float) -> Routing:
-    """Router (R1) followed by token-level or block-level routing."""
+def route(x_bits, w_r, bias, k: int, mode: int, block_size: int, p: float,
+          k_mask: Optional[int] = None) -> Routing:
+    """Router (R1) followed by token-level or block-level routing (k_mask: see route_block;
+    ignored in token mode)."""
     s = router_scores(router_logits(x_bits, w_r, bias))
     if mode == ROUTE_TOKEN:
         return route_token(s, k)
-    return route_block(s, k, block_size, p)
+    return route_block(s, k, block_size, p, k_mask)
 
 
 # ----------------------------------------------------------------------------------------

@@ -39,7 +39,7 @@ class LayerDesc(ctypes.Structure):
                 ("top_k", ctypes.c_int32), ("d_ff", ctypes.c_int32),
                 ("d_ff_shared", ctypes.c_int32), ("block_size", ctypes.c_int32),
                 ("n_blocks", ctypes.c_int32), ("mode", ctypes.c_int32),
-                ("top_p", ctypes.c_float)]
+                ("top_p", ctypes.c_float), ("block_top_k", ctypes.c_int32)]
 
     @property
     def T(self) -> int:
@@ -47,9 +47,9 @@ class LayerDesc(ctypes.Structure):
 
 
 def make_desc(d_model, n_experts, top_k, d_ff, d_ff_shared, block_size, n_blocks,
-              mode=DMOE_ROUTE_BLOCK, top_p=0.0) -> LayerDesc:
+              mode=DMOE_ROUTE_BLOCK, top_p=0.0, block_top_k=0) -> LayerDesc:
     return LayerDesc(d_model, n_experts, top_k, d_ff, d_ff_shared, block_size, n_blocks,
-                     mode, float(top_p))
+                     mode, float(top_p), int(block_top_k))
 
 
 class DmoeError(RuntimeError):

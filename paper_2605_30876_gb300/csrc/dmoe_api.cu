@@ -94,7 +94,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.logits_part = take(sizeof(float) * (w.router_splits == 0 ? 1 : w.router_splits) * T * E);
   w.probs = take(sizeof(float) * T * E);
   w.probs_hat = take(sizeof(float) * T * E);
-  w.cand = take(sizeof(uint2) * T * ((E + 31) / 32) * k);
+  w.cand = take(sizeof(uint2) * T * ((E + 31) / 32) * (size_t)mask_top_k(d));
   w.tk_idx = take(sizeof(int32_t) * T * k);
   w.tk_gate = take(sizeof(float) * T * k);
   w.unique_ids = take(sizeof(int32_t) * E);
@@ -129,6 +129,10 @@ dmoe_status check_desc(const dmoe_layer_desc* d) {
   if (d->mode != DMOE_ROUTE_TOKEN && d->mode != DMOE_ROUTE_BLOCK) return DMOE_ERR_INVALID_ARG;
   if (!(d->top_p == d->top_p) || d->top_p < 0.f) return DMOE_ERR_INVALID_ARG;  // NaN or < 0
   if (d->top_k > d->n_experts) return DMOE_ERR_INVALID_ARG;
+  if (d->block_top_k < 0 || (d->block_top_k > 0 && d->block_top_k < d->top_k) ||
+      d->block_top_k > d->n_experts)
+    return DMOE_ERR_INVALID_ARG;
+  if (d->block_top_k > kMaxTopK) return DMOE_ERR_UNSUPPORTED;
   if (d->top_k > kMaxTopK || d->n_experts > kMaxExperts || d->n_experts % 8 != 0)
     return DMOE_ERR_UNSUPPORTED;
   if (d->d_model % 128 != 0 || d->d_model > kMaxDModel) return DMOE_ERR_UNSUPPORTED;
@@ -187,6 +191,7 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.d = desc->d_model;
   a.E = desc->n_experts;
   a.k = desc->top_k;
+  a.kb = mask_top_k(*desc);
   a.B = desc->block_size;
   a.n_blocks = desc->n_blocks;
   a.mode = desc->mode;
@@ -372,11 +377,12 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   dsp.k = desc->top_k;
   dsp.err = at<DevErrRecord>(workspace, plan.err);
   // block top-k through the decode-size launches: the expert launch starts streaming on the
-  // early-published coresets, before the routing launch ends
+  // early-published coresets, before the routing launch ends (only when every token keeps
+  // the whole coreset, so that the coresets' union is the unique set)
   const int T = desc->n_blocks * desc->block_size;
   int32_t* spec_ids = nullptr;
   int32_t* spec_cnt = nullptr;
-  if (desc->mode == DMOE_ROUTE_BLOCK && desc->top_p <= 0.f &&
+  if (desc->mode == DMOE_ROUTE_BLOCK && desc->top_p <= 0.f && mask_top_k(*desc) == desc->top_k &&
       route_cluster_ok(T, desc->d_model, desc->n_experts) &&
       experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared)) {
     spec_ids = at<int32_t>(workspace, plan.spec);

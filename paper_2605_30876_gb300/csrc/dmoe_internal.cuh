@@ -96,6 +96,12 @@ inline int expert_n_max(int T) {
 
 Workspace plan_workspace(const dmoe_layer_desc& d);
 
+// The k of Algorithm 1's TopKMask and coreset floor: block_top_k in block mode when set,
+// else the per-token k.
+inline int mask_top_k(const dmoe_layer_desc& d) {
+  return (d.mode == DMOE_ROUTE_BLOCK && d.block_top_k > 0) ? d.block_top_k : d.top_k;
+}
+
 // ---------------------------------------------------------------------------------------
 // launchers (each defined in its own translation unit)
 // ---------------------------------------------------------------------------------------
@@ -143,12 +149,13 @@ struct RouterArgs {
   float* logits_part;
   float* probs;        // [T, E]
   float* probs_hat;    // [T, E] (block mode)
-  uint2* cand;         // [T, ceil(E/32), k] (decode-size routing)
+  uint2* cand;         // [T, ceil(E/32), kb] (decode-size routing)
   int32_t* topk_idx;   // [T, k] final routing
   float* topk_gate;    // [T, k]
   int32_t* coreset;    // [n_blocks, E] or null
   int32_t* coreset_size;
   int T, d, E, k, B, n_blocks, mode, splits;
+  int kb;              // k of TopKMask and of the coreset floor (block mode; k >= this k)
   float top_p;
   DevErrRecord* err;
   L2Prefetch shared_pf;   // the shared expert's weights (one "expert")

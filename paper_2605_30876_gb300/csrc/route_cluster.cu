@@ -147,7 +147,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   // z = 0 and the tile is the whole forward
   const int tz = blockIdx.z * kClMaxTok;
   const int T = a.T - tz < kClMaxTok ? a.T - tz : kClMaxTok;
-  const int E = a.E, k = a.k, B = a.B;
+  // k: experts per token; kc: candidates per cluster and token = the TopKMask width
+  // (block mode; kc >= k) or k (token mode)
+  const int E = a.E, k = a.k, kc = a.kb, B = a.B;
   const int TB = f.box_rows;
   const uint32_t rank = cluster_rank();
   const int DC = a.d / kCl;                          // rows of d in this CTA's slice
@@ -289,9 +291,9 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   CT_AT(2);
   cluster_sync();   // every partial has reached its owner
   // CTA r adds the partials of tokens t = r (mod 8), in rank order, adds the bias, and keeps
-  // the cluster's k best experts of the token (candidates for the top-k over all experts:
-  // any expert of the top-k is among the k best of its own cluster)
-  uint2* cand = a.cand;   // [T][clusters][k]: (order key, id)
+  // the cluster's kc best experts of the token (candidates for the top-kc over all experts:
+  // any expert of the top-kc is among the kc best of its own cluster)
+  uint2* cand = a.cand;   // [T][clusters][kc]: (order key, id)
   {
     const int t = (int)rank + 8 * warp;
     if (t < T) {
@@ -312,8 +314,8 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
 #pragma unroll 8
         for (int j = 0; j < 32; ++j)
           r += ((((uint64_t)s_loc[warp][j]) << 32) | (uint32_t)(31 - j)) > mine ? 1 : 0;
-        if (r < k)
-          cand[((size_t)t * n_clusters + blockIdx.y) * k + r] =
+        if (r < kc)
+          cand[((size_t)t * n_clusters + blockIdx.y) * kc + r] =
               make_uint2(key, ok ? (uint32_t)(e0 + lane) : 0xffffffffu);
       }
     }
@@ -348,7 +350,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   {
     const int t = 8 * (int)rank + warp;
     if (t < T) {
-      const int nc = n_clusters * k;                       // candidates of the token
+      const int nc = n_clusters * kc;                      // candidates of the token
       const uint2* tc = cand + (size_t)t * nc;
       uint2 cd[kClMaxCand / 32];
 #pragma unroll
@@ -397,10 +399,10 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       for (int q = 0; q < kClMaxCand / 32; ++q) s_cand[warp][lane + 32 * q] = cd[q];
       __syncwarp();
       int head = 0;
-      uint2 hc = lane < n_clusters ? s_cand[warp][lane * k] : make_uint2(0u, 0xffffffffu);
+      uint2 hc = lane < n_clusters ? s_cand[warp][lane * kc] : make_uint2(0u, 0xffffffffu);
       int my_idx = -1;
       float my_val = 0.f;
-      for (int r = 0; r < k; ++r) {
+      for (int r = 0; r < kc; ++r) {
         const uint32_t kmax = __reduce_max_sync(0xffffffffu, hc.x);
         const uint32_t imin = __reduce_min_sync(0xffffffffu, hc.x == kmax ? hc.y : 0xffffffffu);
         if (lane == r) {
@@ -409,14 +411,14 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         }
         if (hc.x == kmax && hc.y == imin) {
           ++head;
-          hc = head < k ? s_cand[warp][lane * k + head] : make_uint2(0u, 0xffffffffu);
+          hc = head < kc ? s_cand[warp][lane * kc + head] : make_uint2(0u, 0xffffffffu);
         }
       }
       CT_AT(11);
       if (a.mode == DMOE_ROUTE_BLOCK) {
-        // TopKMask: the k winners into the zeroed row of token t in the CTA that routes
+        // TopKMask: the kc winners into the zeroed row of token t in the CTA that routes
         // its block (block b: CTA b mod 8)
-        if (lane < k)
+        if (lane < kc)
           st_peer_f32(peer_addr(sHat + t * kMaxExperts + my_idx, (uint32_t)((t / B) % kCl)),
                       my_val);
       } else {
@@ -441,7 +443,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     for (int b = (int)rank; b < a.n_blocks; b += kCl) {
       const int t0 = b * B;
       const int size = block_coreset_steps(
-          E, k, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
+          E, kc, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
       CT_AT(25);

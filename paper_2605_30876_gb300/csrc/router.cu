@@ -84,7 +84,8 @@ router_logits_kernel(const __nv_bfloat16* __restrict__ x, const float* __restric
   }
 }
 
-// Eight tokens per CTA, one warp each.
+// Eight tokens per CTA, one warp each. k is the TopKMask width in block mode and the
+// routed k in token mode.
 __global__ void __launch_bounds__(256)
 router_softmax_kernel(const float* __restrict__ part, int splits, const float* __restrict__ bias,
                       float* __restrict__ probs, float* __restrict__ probs_hat,
@@ -101,12 +102,12 @@ router_softmax_kernel(const float* __restrict__ part, int splits, const float* _
 
 __global__ void __launch_bounds__(256)
 block_route_kernel(const float* __restrict__ probs, const float* __restrict__ probs_hat,
-                   int E, int k, int B, float top_p,
+                   int E, int kb, int k, int B, float top_p,
                    int32_t* __restrict__ topk_idx, float* __restrict__ topk_gate,
                    int32_t* __restrict__ coreset, int32_t* __restrict__ coreset_size) {
   pdl_launch_dependents();
   pdl_wait();
-  block_route_cta(blockIdx.x, probs, probs_hat, E, k, B, top_p, topk_idx, topk_gate, coreset,
+  block_route_cta(blockIdx.x, probs, probs_hat, E, kb, k, B, top_p, topk_idx, topk_gate, coreset,
                   coreset_size);
 }
 
@@ -134,11 +135,11 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
     }
     e = launch_ex(router_softmax_kernel, dim3((a.T + 7) / 8), dim3(256), 0, s, true,
                   a.logits_part, cl ? 1 : a.splits, cl ? nullptr : a.bias, a.probs, a.probs_hat,
-                  a.topk_idx, a.topk_gate, a.T, a.E, a.k, a.mode);
+                  a.topk_idx, a.topk_gate, a.T, a.E, a.kb, a.mode);
     if (e != cudaSuccess) return e;
     if (a.mode == DMOE_ROUTE_BLOCK) {
       e = launch_ex(block_route_kernel, dim3(a.n_blocks), dim3(256), 0, s, true, a.probs,
-                    a.probs_hat, a.E, a.k, a.B, a.top_p, a.topk_idx, a.topk_gate, a.coreset,
+                    a.probs_hat, a.E, a.kb, a.k, a.B, a.top_p, a.topk_idx, a.topk_gate, a.coreset,
                     a.coreset_size);
       if (e != cudaSuccess) return e;
     } else {

@@ -108,6 +108,7 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
   a.d = desc->d_model;
   a.E = desc->n_experts;
   a.k = desc->top_k;
+  a.kb = mask_top_k(*desc);
   a.B = desc->block_size;
   a.n_blocks = desc->n_blocks;
   a.mode = desc->mode;

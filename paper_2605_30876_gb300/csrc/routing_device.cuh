@@ -412,24 +412,26 @@ __device__ inline void mask_topk_small(int k, int B, int size, const int* order,
 }
 
 template <class HatFn, class ProbFn, class OutFn>
-__device__ inline void block_route_steps(int E, int k, int B, float top_p, HatFn hat, ProbFn prob,
-                                         OutFn out, int32_t* __restrict__ coreset,
+__device__ inline void block_route_steps(int E, int kb, int k, int B, float top_p, HatFn hat,
+                                         ProbFn prob, OutFn out, int32_t* __restrict__ coreset,
                                          int32_t* __restrict__ coreset_size) {
   __shared__ int order[kMaxExperts];
-  const int size = block_coreset_steps(E, k, B, top_p, hat, order, coreset, coreset_size);
+  const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size);
   mask_topk_warps(k, B, size, order, prob, out);
   __syncthreads();
 }
 
-// Algorithm 1 for block b with the block's rows in global memory ([T, E] row-major).
+// Algorithm 1 for block b with the block's rows in global memory ([T, E] row-major). The
+// hat rows hold TopKMask(s_i, kb); every token keeps its k <= kb best coreset members.
 __device__ inline void block_route_cta(int b, const float* probs, const float* probs_hat, int E,
-                                       int k, int B, float top_p, int32_t* __restrict__ topk_idx,
+                                       int kb, int k, int B, float top_p,
+                                       int32_t* __restrict__ topk_idx,
                                        float* __restrict__ topk_gate,
                                        int32_t* __restrict__ coreset,
                                        int32_t* __restrict__ coreset_size) {
   const size_t r0 = (size_t)b * B;
   block_route_steps(
-      E, k, B, top_p,
+      E, kb, k, B, top_p,
       [&](int i, int e) { return probs_hat[(r0 + i) * E + e]; },
       [&](int i, int e) { return probs[(r0 + i) * E + e]; },
       [&](int i, int r, int e, float g) {

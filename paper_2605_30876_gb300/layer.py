@@ -36,7 +36,8 @@ class MoELayer:
     def from_shape(cls, shape, weights, device="cuda", workspace=None) -> "MoELayer":
         desc = make_desc(shape.d_model, shape.n_experts, shape.top_k, shape.d_ff,
                          shape.d_ff_shared, shape.block_size, shape.n_blocks,
-                         getattr(shape, "mode", DMOE_ROUTE_BLOCK), getattr(shape, "top_p", 0.0))
+                         getattr(shape, "mode", DMOE_ROUTE_BLOCK), getattr(shape, "top_p", 0.0),
+                         getattr(shape, "block_top_k", 0))
         return cls(desc, weights, device, workspace)
 
     def forward(self, x: torch.Tensor, y: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:

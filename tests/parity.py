@@ -28,7 +28,7 @@ def dm():
 def desc_of(shape):
     return dm().make_desc(shape.d_model, shape.n_experts, shape.top_k, shape.d_ff,
                           shape.d_ff_shared, shape.block_size, shape.n_blocks, shape.mode,
-                          shape.top_p)
+                          shape.top_p, shape.block_top_k)
 
 
 def make(shape, seed=0, layer=0, device="cuda"):
@@ -74,7 +74,7 @@ def gpu_dispatch(shape, idx_t, ws=None):
 
 def oracle_routing(shape, host):
     return O.route(host["x"], host["w_r"], host["bias"], shape.top_k, shape.mode,
-                   shape.block_size, shape.top_p)
+                   shape.block_size, shape.top_p, shape.block_top_k)
 
 
 def check_routing(shape, g, orc: O.Routing, report=None):
@@ -96,7 +96,7 @@ def check_routing(shape, g, orc: O.Routing, report=None):
             gc = g["coreset"][b]
             assert np.all(gc[size:] == -1)
             gset = set(gc[:size].tolist())
-            assert len(gset) == size >= k
+            assert len(gset) == size >= max(k, shape.block_top_k)
             oset = set(orc.coresets[b].tolist())
             if orc.coreset_margin[b] >= DELTA:
                 assert gset == oset, (b, sorted(gset ^ oset))

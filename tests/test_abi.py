@@ -31,7 +31,7 @@ def test_every_declared_symbol_is_exported(dm):
 
 
 def test_abi_version_and_status_strings(dm):
-    assert dm.dmoe_abi_version() == 1
+    assert dm.dmoe_abi_version() == 2
     for s in range(7):
         assert dm.dmoe_status_string(s).startswith("DMOE_")
 
@@ -56,12 +56,23 @@ def test_workspace_size_grows_with_tokens(dm):
     (dict(top_k=17, n_experts=64), 2), (dict(d_model=200), 2), (dict(d_ff=100), 2),
     (dict(d_ff_shared=-1), 1), (dict(d_ff_shared=96), 2), (dict(block_size=0), 1),
     (dict(n_blocks=200), 2), (dict(mode=7), 1), (dict(top_p=-0.5), 1),
-    (dict(top_p=float("nan")), 1),
+    (dict(top_p=float("nan")), 1), (dict(block_top_k=-1), 1), (dict(block_top_k=4), 1),
+    (dict(block_top_k=17), 2), (dict(n_experts=16, top_k=2, block_top_k=24), 1),
 ])
 def test_invalid_desc_is_rejected(dm, kw, status):
     with pytest.raises(dm.DmoeError) as ei:
         dm.dmoe_workspace_size(_desc(dm, **kw))
     assert ei.value.status == status
+
+
+def test_block_top_k_accepted_and_struct_layout(dm):
+    # block_top_k = 0 (= top_k), = top_k, and above top_k are valid
+    for kw in (dict(), dict(block_top_k=8), dict(top_k=4, block_top_k=8),
+               dict(top_k=1, block_top_k=16), dict(mode=dm.DMOE_ROUTE_TOKEN, top_k=4)):
+        assert dm.dmoe_workspace_size(_desc(dm, **kw)) > 0
+    # the C struct: nine 4-byte fields, block_top_k last
+    assert ctypes.sizeof(dm.LayerDesc) == 40
+    assert dm.LayerDesc.block_top_k.offset == 36
 
 
 def test_null_and_misaligned_pointers_are_rejected_before_launch(dm):

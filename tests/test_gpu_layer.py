@@ -29,6 +29,12 @@ LAYER_CASES = {
     # block top-k at decode sizes: the expert launch starts on the published coresets
     "decode_B16x4_p0": LAYER.with_(block_size=16, n_blocks=4),
     "decode_B1x40_p0": LAYER.with_(block_size=1, n_blocks=40, bias_scale=0.0),
+    # fewer experts per token inside the coreset; the Top-4 token baseline
+    "layer_fewer_k4_of8_p0": LAYER.with_(top_k=4, block_top_k=8),
+    "layer_fewer_k2_of8_p06": LAYER.with_(top_k=2, block_top_k=8, top_p=0.6),
+    "layer_b8_fewer_k4_of8": LAYER_B8.with_(top_k=4, block_top_k=8),
+    "tiny_fewer_k1_of2_shared": TINY.with_(top_k=1, block_top_k=2, d_ff_shared=128),
+    "layer_token_top4": LAYER.with_(mode=ROUTE_TOKEN, top_k=4),
 }
 SAMPLED = {"T300_multi_ntile"}
 

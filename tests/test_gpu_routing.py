@@ -32,6 +32,15 @@ ROUTING_CASES = {
     "k_equals_E": TINY.with_(top_k=16, top_p=0.3),
     "E8_k3": TINY.with_(n_experts=8, top_k=3, top_p=0.7, d_model=128),
     "max_tokens_4096": LAYER.with_(block_size=64, n_blocks=64, top_p=0.6),
+    # fewer experts per token inside the coreset (TopKMask and floor at block_top_k)
+    "layer_fewer_k4_of8_p0": LAYER.with_(top_k=4, block_top_k=8),
+    "layer_fewer_k2_of8_p06": LAYER.with_(top_k=2, block_top_k=8, top_p=0.6),
+    "layer_b8_fewer_k4_of8": LAYER_B8.with_(top_k=4, block_top_k=8),
+    "tiny_fewer_k1_of2": TINY.with_(top_k=1, block_top_k=2),
+    "tiny_fewer_k3_of16_p03": TINY.with_(top_k=3, block_top_k=16, top_p=0.3),
+    "stack_fewer_k4_of8": STACK20.with_(top_k=4, block_top_k=8),
+    # the Top-4 token-level baseline
+    "layer_token_top4": LAYER.with_(mode=ROUTE_TOKEN, top_k=4),
 }
 
 

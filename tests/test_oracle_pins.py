@@ -89,6 +89,68 @@ def test_hand_case_through_router():
 
 
 # ------------------------------------------------------------------------------------
+# Fewer experts per token (App. A): TopKMask and the floor at k_mask, final TopK at k.
+# Hand case, S_HAND with k_mask = 3, k = 2, p = 0:
+#   TopKMask(s_1, 3) = [.5, .3, .15, 0], TopKMask(s_2, 3) = [0, .4, .2, .3]
+#   S = [.5, .7, .35, .3] -> sorted order 1, 0, 2, 3 -> floor 3: C = {1, 0, 2}
+#   R_1 = (0, 1), g = (.625, .375); R_2 inside {1, 0, 2} = (1, 2), g = (2/3, 1/3)
+#   (with TopKMask at k = 2 the coreset would be {1, 0} and R_2 = (1, 0); token routing
+#   gives R_2 = (1, 3): the case separates all three)
+# k_mask = 2, k = 1: p = 0 -> C = {1, 0}, R_1 = (0,), R_2 = (1,), gates 1;
+#                    p = .9 -> C = {1, 0, 3}, the same R (the coreset only grows)
+# ------------------------------------------------------------------------------------
+def test_hand_case_fewer_experts_k_mask3_k2():
+    r = O.route_block(S_HAND, k=2, block_size=2, p=0.0, k_mask=3)
+    assert list(r.coresets[0]) == [1, 0, 2]
+    assert r.idx.tolist() == [[0, 1], [1, 2]]
+    np.testing.assert_allclose(r.gate, [[0.625, 0.375], [2 / 3, 1 / 3]], rtol=1e-6)
+
+
+@pytest.mark.parametrize("p,core", [(0.0, [1, 0]), (0.9, [1, 0, 3])])
+def test_hand_case_fewer_experts_k1(p, core):
+    r = O.route_block(S_HAND, k=1, block_size=2, p=p, k_mask=2)
+    assert list(r.coresets[0]) == core
+    assert r.idx.tolist() == [[0], [1]]
+    np.testing.assert_allclose(r.gate, [[1.0], [1.0]], rtol=0)
+
+
+@pytest.mark.parametrize("E,km,k,p", [(8, 3, 2, 0.0), (8, 4, 1, 0.5), (10, 4, 3, 0.8),
+                                      (6, 5, 2, 1.0)])
+def test_fewer_experts_brute_force(E, km, k, p):
+    """R_i is the k-subset of the coreset with the largest score sum (brute force over
+    all subsets), listed by descending score; the coreset is the k_mask one."""
+    rng = np.random.default_rng(100 + E + km)
+    B, nb = 4, 3
+    s = f32(rng.dirichlet(np.ones(E), size=B * nb))
+    r = O.route_block(s, k, B, p, k_mask=km)
+    full = O.route_block(s, km, B, p)
+    for b in range(nb):
+        assert np.array_equal(r.coresets[b], full.coresets[b])   # the coreset uses k_mask
+        C = r.coresets[b].tolist()
+        assert len(C) >= km
+        for i in range(b * B, (b + 1) * B):
+            best = max(itertools.combinations(C, k), key=lambda c: s[i, list(c)].astype(float).sum())
+            assert set(r.idx[i].tolist()) == set(best)
+            v = s[i, r.idx[i]]
+            assert all(v[j] > v[j + 1] for j in range(k - 1))
+            assert abs(r.gate[i].sum() - 1.0) <= 1e-12
+
+
+@pytest.mark.parametrize("p", [0.0, 0.6])
+def test_fewer_experts_is_prefix_of_full_routing(p):
+    """Inside one coreset TopK(., k) is the first k of TopK(., k_mask): the same ids in
+    the same order, gates renormalised over the k."""
+    shape = TINY.with_(top_k=4, n_blocks=4, bias_scale=0.5)
+    s = _scores(shape, 21)
+    full = O.route_block(s, 4, shape.block_size, p)
+    for k in (1, 2, 3):
+        r = O.route_block(s, k, shape.block_size, p, k_mask=4)
+        assert np.array_equal(r.idx, full.idx[:, :k])
+        w = s[np.arange(shape.T)[:, None], full.idx[:, :k]].astype(np.float64)
+        np.testing.assert_allclose(r.gate, w / w.sum(1, keepdims=True), rtol=1e-12)
+
+
+# ------------------------------------------------------------------------------------
 # Router closed forms
 # ------------------------------------------------------------------------------------
 def test_softmax_closed_form():
