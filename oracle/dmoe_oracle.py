@@ -245,8 +245,9 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
 
     ``k_mask`` (default k) is the k of TopKMask and of the floor (R6); the final TopK keeps
     k <= k_mask members of the coreset per token (R11: App. A's "fewer experts for each
-    token"). The block's margin also covers every TopKMask decision of its tokens: a near
-    tie at a token's k_mask-th score can move that score to another expert of S_block."""
+    token"). The block's margin also covers the TopKMask decisions of its tokens that
+    matter: where swapping a token's k_mask-th and (k_mask+1)-th experts in its mask would
+    change the coreset, that token's set margin bounds the block's margin."""
     T, E = s.shape
     assert T % block_size == 0
     km = k if k_mask is None or k_mask <= 0 else int(k_mask)
@@ -264,8 +265,7 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
         S_tilde = normalize(S)                        # Algorithm 1: Normalize
         C = top_p(S_tilde, p, km)                     # Algorithm 1: TopP (+ floor)
         coresets.append(C.ids)
-        mask_margin = min(topk_margins(s[i], km)[0] for i in range(b * block_size, (b + 1) * block_size))
-        cm[b] = min(C.margin, mask_margin)
+        cm[b] = min(C.margin, mask_flip_margin(s[rows], S, km, p, C, C.margin))
         for i in range(b * block_size, (b + 1) * block_size):
             sC = mask_outside(s[i], C.ids)            # Algorithm 1: MaskOutside
             R = topk_desc(sC, k)                      # Algorithm 1: TopK
@@ -273,6 +273,29 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
             gate[i] = renormalize(s[i], R)
             sm[i], om[i] = topk_margins(sC, k)
     return Routing(idx, gate, coresets, sm, om, cm, s)
+
+
+def mask_flip_margin(s_block: np.ndarray, S: np.ndarray, k: int, p: float, C: Coreset,
+                     bound: float) -> float:
+    """Smallest TopKMask set margin (gap between a token's k-th and (k+1)-th score) among
+    the block's tokens whose flip at that boundary changes the coreset as a set; only
+    margins below ``bound`` are examined (larger ones cannot lower the block's margin)."""
+    out = float("inf")
+    core = set(C.ids.tolist())
+    for i in range(s_block.shape[0]):
+        sm, _ = topk_margins(s_block[i], k)
+        if not sm < min(bound, out):
+            continue
+        order = sort_desc(np.asarray(s_block[i], F64))
+        a, c = int(order[k - 1]), int(order[k])      # the k-th and the first left out
+        v = np.asarray(s_block[i], F32).astype(F64)
+        S_alt = np.array(S, F64)
+        S_alt[a] -= v[a]
+        S_alt[c] += v[c]
+        alt = top_p(normalize(S_alt), p, k)
+        if set(alt.ids.tolist()) != core:
+            out = sm
+    return out
 
 
 def route(x_bits, w_r, bias, k: int, mode: int, block_size: int, p: float,
