@@ -40,7 +40,9 @@ Readings (the paper is silent or ambiguous here):
 Decisions (a top-k, the coreset boundary) are taken on fp32 values, as the router's
 fp32 output is the input of Algorithm 1. Each decision also reports a *margin*: how far
 the decision is from flipping, in the units of the compared quantity. A decision with a
-margin below 1e-5 may legitimately come out either way on the GPU.
+margin below NEAR_TIE = 1e-5 may legitimately come out either way on the GPU; for a block
+whose coreset decision is that close, the coresets that one such flip reaches are listed
+too (Routing.coreset_alts), so that a GPU result can be checked against them.
 """
 from __future__ import annotations
 
@@ -54,6 +56,7 @@ F64 = np.float64
 
 ROUTE_TOKEN = 0
 ROUTE_BLOCK = 1
+NEAR_TIE = 1e-5        # decisions closer than this may come out either way on the GPU
 
 
 # ----------------------------------------------------------------------------------------
@@ -157,6 +160,8 @@ class Coreset:
     ids: np.ndarray       # int32, sorted by S~ descending (ties: lower index first)
     m_p: int              # length of the prefix the p rule alone selects
     margin: float         # distance of the decision from flipping (see coreset_margin)
+    alts: List[np.ndarray] = dataclasses.field(default_factory=list)
+    # the coresets one flip of a decision closer than NEAR_TIE reaches (see coreset_margin)
 
 
 def top_p(S_tilde: np.ndarray, p: float, k: int) -> Coreset:
@@ -178,7 +183,19 @@ def top_p(S_tilde: np.ndarray, p: float, k: int) -> Coreset:
         m = min(m, nnz)
     size = max(m, k)
     ids = order[:size].astype(np.int32)
-    return Coreset(ids=ids, m_p=m, margin=coreset_margin(vals, cum, p, m, k, size))
+    C = Coreset(ids=ids, m_p=m, margin=coreset_margin(vals, cum, p, m, k, size))
+    # one flip of a near decision: the boundary pair swapped, one expert more (the sum
+    # falls just short of p) or one fewer (the sum reaches p one step earlier)
+    v = np.asarray(vals, F64)
+    if size < v.size and v[size - 1] - v[size] < NEAR_TIE:
+        C.alts.append(np.concatenate([order[:size - 1], order[size:size + 1]]).astype(np.int32))
+    if cum is not None and p > 0.0 and m >= k:
+        pp = float(F32(p))
+        if float(cum[m - 1]) - pp < NEAR_TIE and size < v.size and v[size] > 0:
+            C.alts.append(order[:size + 1].astype(np.int32))
+        if m > k and m >= 2 and pp - float(cum[m - 2]) < NEAR_TIE:
+            C.alts.append(order[:size - 1].astype(np.int32))
+    return C
 
 
 def coreset_margin(vals: np.ndarray, cum: Optional[np.ndarray], p: float, m: int, k: int,
@@ -221,6 +238,15 @@ class Routing:
     order_margin: np.ndarray        # float64 [T]: margin of the slot order of token i
     coreset_margin: np.ndarray      # float64 [n_blocks] (inf in token mode)
     scores: np.ndarray              # fp32 [T,E] router scores s_i
+    coreset_alts: List[List[np.ndarray]] = dataclasses.field(default_factory=list)
+    # per block: the coresets one near-tie flip reaches ([] per block in token mode)
+
+
+def topk_in_coreset(s_i: np.ndarray, C: np.ndarray, k: int):
+    """MaskOutside then TopK for one token (R7): (R_i, set margin, order margin)."""
+    sC = mask_outside(s_i, C)
+    sm, om = topk_margins(sC, k)
+    return topk_desc(sC, k), sm, om
 
 
 def route_token(s: np.ndarray, k: int) -> Routing:
@@ -258,7 +284,7 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
     sm = np.zeros(T, F64)
     om = np.zeros(T, F64)
     cm = np.zeros(nb, F64)
-    coresets = []
+    coresets, alts = [], []
     for b in range(nb):
         rows = slice(b * block_size, (b + 1) * block_size)
         S = aggregate(s[rows], km)                    # Algorithm 1: S_block
@@ -266,25 +292,25 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
         C = top_p(S_tilde, p, km)                     # Algorithm 1: TopP (+ floor)
         coresets.append(C.ids)
         cm[b] = min(C.margin, mask_flip_margin(s[rows], S, km, p, C, C.margin))
+        alts.append(C.alts)
         for i in range(b * block_size, (b + 1) * block_size):
-            sC = mask_outside(s[i], C.ids)            # Algorithm 1: MaskOutside
-            R = topk_desc(sC, k)                      # Algorithm 1: TopK
+            R, sm[i], om[i] = topk_in_coreset(s[i], C.ids, k)   # MaskOutside, TopK
             idx[i] = R
             gate[i] = renormalize(s[i], R)
-            sm[i], om[i] = topk_margins(sC, k)
-    return Routing(idx, gate, coresets, sm, om, cm, s)
+    return Routing(idx, gate, coresets, sm, om, cm, s, alts)
 
 
 def mask_flip_margin(s_block: np.ndarray, S: np.ndarray, k: int, p: float, C: Coreset,
                      bound: float) -> float:
     """Smallest TopKMask set margin (gap between a token's k-th and (k+1)-th score) among
     the block's tokens whose flip at that boundary changes the coreset as a set; only
-    margins below ``bound`` are examined (larger ones cannot lower the block's margin)."""
+    margins below ``bound`` or NEAR_TIE are examined (larger ones cannot lower the block's
+    margin). The coreset such a flip closer than NEAR_TIE reaches joins C.alts."""
     out = float("inf")
     core = set(C.ids.tolist())
     for i in range(s_block.shape[0]):
         sm, _ = topk_margins(s_block[i], k)
-        if not sm < min(bound, out):
+        if not (sm < min(bound, out) or sm < NEAR_TIE):
             continue
         order = sort_desc(np.asarray(s_block[i], F64))
         a, c = int(order[k - 1]), int(order[k])      # the k-th and the first left out
@@ -294,7 +320,9 @@ def mask_flip_margin(s_block: np.ndarray, S: np.ndarray, k: int, p: float, C: Co
         S_alt[c] += v[c]
         alt = top_p(normalize(S_alt), p, k)
         if set(alt.ids.tolist()) != core:
-            out = sm
+            out = min(out, sm)
+            if sm < NEAR_TIE:
+                C.alts.append(alt.ids)
     return out
 
 

@@ -2,7 +2,9 @@
 the CPU oracle under the rules stated for this layer:
 
 * routing (expert ids, coreset, dispatch) bit-exact, except at decisions whose oracle
-  margin is below DELTA = 1e-5, where either choice is accepted if it is a valid one;
+  margin is below DELTA = 1e-5, where either choice is accepted if it is a valid one (a
+  block's coreset: the oracle's or one that a single near-tie flip reaches, its tokens then
+  checked exactly against the oracle's routing inside the GPU's coreset);
 * outputs (bf16 y vs the oracle's float64 y on the GPU's selection):
   relative L2 <= 1e-2 and max-abs <= 3e-2.
 """
@@ -90,7 +92,9 @@ def check_routing(shape, g, orc: O.Routing, report=None):
     for t in range(T):
         assert len(set(idx[t].tolist())) == k, (t, idx[t])
     block_ok = np.ones(shape.n_blocks, bool)
+    ref_idx, ref_sm, ref_om = orc.idx, orc.set_margin, orc.order_margin
     if shape.mode == ROUTE_BLOCK:
+        ref_idx, ref_sm, ref_om = ref_idx.copy(), ref_sm.copy(), ref_om.copy()
         for b in range(shape.n_blocks):
             size = int(g["coreset_size"][b])
             gc = g["coreset"][b]
@@ -101,18 +105,27 @@ def check_routing(shape, g, orc: O.Routing, report=None):
             if orc.coreset_margin[b] >= DELTA:
                 assert gset == oset, (b, sorted(gset ^ oset))
             else:
-                block_ok[b] = False
                 stats["blocks_ambiguous"] += 1
+                # a near tie in the block: the GPU's coreset must be the oracle's or one that
+                # a single near-tie flip reaches; its tokens are then checked exactly against
+                # the oracle's routing inside that coreset
+                alts = [set(a.tolist()) for a in orc.coreset_alts[b]]
+                assert gset == oset or gset in alts, (b, sorted(gset ^ oset))
+                if gset != oset:
+                    stats["blocks_alternative"] = stats.get("blocks_alternative", 0) + 1
+                    C = gc[:size].astype(np.int32)
+                    for t in range(b * B, (b + 1) * B):
+                        ref_idx[t], ref_sm[t], ref_om[t] = O.topk_in_coreset(orc.scores[t], C, k)
             for t in range(b * B, (b + 1) * B):
                 assert set(idx[t].tolist()) <= gset, t
     else:
         assert np.all(g["coreset"] == -1) and np.all(g["coreset_size"] == 0)
     for t in range(T):
         b = t // B
-        if block_ok[b] and orc.set_margin[t] >= DELTA:
-            assert set(idx[t].tolist()) == set(orc.idx[t].tolist()), (t, idx[t], orc.idx[t])
-            if orc.order_margin[t] >= DELTA:
-                assert np.array_equal(idx[t], orc.idx[t]), (t, idx[t], orc.idx[t])
+        if block_ok[b] and ref_sm[t] >= DELTA:
+            assert set(idx[t].tolist()) == set(ref_idx[t].tolist()), (t, idx[t], ref_idx[t])
+            if ref_om[t] >= DELTA:
+                assert np.array_equal(idx[t], ref_idx[t]), (t, idx[t], ref_idx[t])
             stats["exact"] += 1
         else:
             stats["ambiguous"] += 1

@@ -114,6 +114,34 @@ def test_hand_case_fewer_experts_k1(p, core):
     np.testing.assert_allclose(r.gate, [[1.0], [1.0]], rtol=0)
 
 
+def test_near_tie_mask_flip_lists_the_other_coreset():
+    """k = 1, p = 0, B = 2: token 1 ties experts 0 and 1 exactly; TopKMask keeps 0 (lower
+    index), S = [.4, 0, .35, 0], C = {0}. Keeping 1 instead gives S = [0, .4, .35, 0] and
+    C = {1}: the block's margin is 0 and {1} is listed as the alternative. A third token
+    pattern with no tie leaves the margin at the boundary gap and lists nothing."""
+    s = f32([[0.4, 0.4, 0.1, 0.1], [0.1, 0.3, 0.35, 0.25]])
+    r = O.route_block(s, k=1, block_size=2, p=0.0)
+    assert list(r.coresets[0]) == [0]
+    assert r.coreset_margin[0] == 0.0
+    assert [a.tolist() for a in r.coreset_alts[0]] == [[1]]
+    s2 = f32([[0.5, 0.3, 0.1, 0.1], [0.1, 0.3, 0.35, 0.25]])
+    r2 = O.route_block(s2, k=1, block_size=2, p=0.0)
+    assert r2.coreset_alts[0] == []
+    np.testing.assert_allclose(r2.coreset_margin[0], (0.5 - 0.35) / 0.85, rtol=1e-6)
+
+
+def test_near_tie_boundary_and_p_crossing_alternatives():
+    """S~ with an exact tie at the floor boundary lists the swapped coreset; p set exactly on
+    a running sum lists the coreset with one expert more."""
+    C = O.top_p(f32([0.4, 0.3, 0.3, 0.0]), 0.0, 2)
+    assert C.ids.tolist() == [0, 1] and C.margin == 0.0
+    assert [a.tolist() for a in C.alts] == [[0, 2]]
+    St = f32([0.5, 0.25, 0.25, 0.0])               # running sums .5, .75, 1 exact in fp32
+    C = O.top_p(St, 0.75, 1)
+    assert C.ids.tolist() == [0, 1] and C.margin == 0.0
+    assert [a.tolist() for a in C.alts] == [[0, 2], [0, 1, 2]]
+
+
 @pytest.mark.parametrize("E,km,k,p", [(8, 3, 2, 0.0), (8, 4, 1, 0.5), (10, 4, 3, 0.8),
                                       (6, 5, 2, 1.0)])
 def test_fewer_experts_brute_force(E, km, k, p):
