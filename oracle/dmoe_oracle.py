@@ -32,7 +32,7 @@ Readings (the paper is silent or ambiguous here):
   R10 expert:   SwiGLU, y_e(x) = W_down (silu(W_gate x) * (W_up x)), fp64 throughout, with
                 the intermediate kept unrounded. Token-level routing (the "Original"
                 baseline of §5.1) is R_i = TopK(s_i, k) with the same gates.
-  R11 fewer experts per token (the direction App. A names, not evaluated in the paper):
+  R17 fewer experts per token (the direction App. A names, not evaluated in the paper):
                 Algorithm 1 runs with k_mask in TopKMask and in the floor, and the final
                 TopK inside the coreset keeps k < k_mask experts per token, gates R8 over
                 those k. k_mask = k is Algorithm 1 itself.
@@ -270,7 +270,7 @@ def route_block(s: np.ndarray, k: int, block_size: int, p: float,
     routed independently. Returns R_i for every token with the R8 gates.
 
     ``k_mask`` (default k) is the k of TopKMask and of the floor (R6); the final TopK keeps
-    k <= k_mask members of the coreset per token (R11: App. A's "fewer experts for each
+    k <= k_mask members of the coreset per token (R17: App. A's "fewer experts for each
     token"). The block's margin also covers the TopKMask decisions of its tokens that
     matter: where swapping a token's k_mask-th and (k_mask+1)-th experts in its mask would
     change the coreset, that token's set margin bounds the block's margin."""
