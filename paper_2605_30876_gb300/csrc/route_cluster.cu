@@ -111,12 +111,8 @@ constexpr int kOffP = 0;                                      // f32 [8][kMaxExp
 constexpr int kOffIdx = kOffP + 8 * kMaxExperts * 4;          // i32 [kClMaxTok * kMaxTopK]
 constexpr int kOffCore = kOffIdx + kClMaxTok * kMaxTopK * 4;  // i32 [8][1 + kMaxExperts]
 constexpr int kOffHat = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;  // f32 [kClMaxTok][kMaxExperts]
-// logits phase: the three bf16 parts of the W_r slice, [3][32 experts][kWtStride bytes]
-constexpr int kOffWt = kClMaxDChunk * kClExp * 4 + kClMaxTok * kClMaxDChunk * 2;
 static_assert(kOffCore + 8 * (1 + kMaxExperts) * 4 <= kClMaxDChunk * kClExp * 4,
               "the routing scratch must fit where the W_r slice was");
-
-constexpr int kWtStride = kClMaxDChunk * 2 + 16;   // bytes per expert row of a W_r part
 
 // bf16 tensor-core product D[16 x 8] += A[16 x 16] B[16 x 8] (fp32 accumulators)
 __device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
@@ -224,36 +220,22 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     }
   }
   CT_AT(1);
-  // W_r slice -> three bf16 parts (hi + mid + lo = w to 2^-27), transposed to
-  // [expert][d] rows of kWtStride bytes (the column-major B operand, padded against bank
-  // conflicts); x * part is exact in fp32, so the three products summed in fp32 give the
-  // fp32 logit
-  uint8_t* Wt = dsm + kOffWt;
-  for (int q = tid; q < kClExp * (DC / 2); q += 256) {
-    const int n = q % kClExp, kp = q / kClExp;
-    const float w0 = Ws[(2 * kp) * kClExp + n], w1 = Ws[(2 * kp + 1) * kClExp + n];
-    const __nv_bfloat16 h0 = __float2bfloat16_rn(w0), h1 = __float2bfloat16_rn(w1);
-    const float r0 = w0 - __bfloat162float(h0), r1 = w1 - __bfloat162float(h1);
-    const __nv_bfloat16 m0 = __float2bfloat16_rn(r0), m1 = __float2bfloat16_rn(r1);
-    const __nv_bfloat16 l0 = __float2bfloat16_rn(r0 - __bfloat162float(m0));
-    const __nv_bfloat16 l1 = __float2bfloat16_rn(r1 - __bfloat162float(m1));
-    uint8_t* row = Wt + n * kWtStride + kp * 4;
-    *reinterpret_cast<__nv_bfloat162*>(row) = __halves2bfloat162(h0, h1);
-    *reinterpret_cast<__nv_bfloat162*>(row + kClExp * kWtStride) = __halves2bfloat162(m0, m1);
-    *reinterpret_cast<__nv_bfloat162*>(row + 2 * kClExp * kWtStride) = __halves2bfloat162(l0, l1);
-  }
-  __syncthreads();
   CT_AT(8);
   // tensor cores (mma.sync m16n8k16): warp tile = 16 tokens x 8 experts over the whole
-  // slice; one accumulator per part (hi, mid, lo), summed in that order at the end
+  // slice. The B fragments come straight from the fp32 W_r slice (rows of 32 experts, 128
+  // bytes, 128-byte swizzle: expert n of row k sits in 16-byte chunk (n / 4) xor (k mod 8),
+  // so a warp's fragment loads hit 32 distinct banks) and are split there into three bf16
+  // parts (hi + mid + lo = w to 2^-27; x * part is exact in fp32), one accumulator per part,
+  // summed in that order at the end
   {
     const int g = lane >> 2, tq = lane & 3;
     const int ntile = (T16 / 16) * (kClExp / 8);
+    const uint8_t* wsb = reinterpret_cast<const uint8_t*>(Ws);
     for (int tile = warp; tile < ntile; tile += 8) {
       const int mt = tile / (kClExp / 8), nt = tile % (kClExp / 8);
       const int r0 = mt * 16 + g;                   // A rows r0, r0 + 8 (same swizzle phase)
+      const int n = nt * 8 + g;                     // B column (expert) of this thread
       float accp[3][4] = {};
-      const uint8_t* brow = Wt + (nt * 8 + g) * kWtStride + tq * 4;
 #pragma unroll 2
       for (int k0 = 0; k0 < DC; k0 += 16) {
         const int bx = k0 >> 6, c = (k0 & 63) >> 3;   // box, 16-B chunk of k0
@@ -263,12 +245,29 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         af[1] = *reinterpret_cast<const uint32_t*>(xb + (r0 + 8) * 128 + ((c ^ (r0 & 7)) << 4) + tq * 4);
         af[2] = *reinterpret_cast<const uint32_t*>(xb + r0 * 128 + (((c + 1) ^ (r0 & 7)) << 4) + tq * 4);
         af[3] = *reinterpret_cast<const uint32_t*>(xb + (r0 + 8) * 128 + (((c + 1) ^ (r0 & 7)) << 4) + tq * 4);
+        // W_r[k][n] for k = k0 + 2tq, +1 (register 0) and +8, +9 (register 1)
+        float w[4];
 #pragma unroll
-        for (int part = 0; part < 3; ++part) {
-          const uint8_t* bp = brow + part * kClExp * kWtStride + k0 * 2;
-          mma_bf16_16816(accp[part], af, *reinterpret_cast<const uint32_t*>(bp),
-                         *reinterpret_cast<const uint32_t*>(bp + 16));
+        for (int j = 0; j < 4; ++j) {
+          const int k = k0 + 2 * tq + (j & 1) + 8 * (j >> 1);
+          w[j] = *reinterpret_cast<const float*>(
+              wsb + k * 128 + ((((n >> 2) ^ (k & 7)) << 4) | ((n & 3) << 2)));
         }
+        uint32_t bp[3][2];
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const __nv_bfloat162 hi = __floats2bfloat162_rn(w[2 * h], w[2 * h + 1]);
+          const float2 hf = __bfloat1622float2(hi);
+          const float q0 = w[2 * h] - hf.x, q1 = w[2 * h + 1] - hf.y;
+          const __nv_bfloat162 mid = __floats2bfloat162_rn(q0, q1);
+          const float2 mf = __bfloat1622float2(mid);
+          const __nv_bfloat162 lo = __floats2bfloat162_rn(q0 - mf.x, q1 - mf.y);
+          bp[0][h] = *reinterpret_cast<const uint32_t*>(&hi);
+          bp[1][h] = *reinterpret_cast<const uint32_t*>(&mid);
+          bp[2][h] = *reinterpret_cast<const uint32_t*>(&lo);
+        }
+#pragma unroll
+        for (int part = 0; part < 3; ++part) mma_bf16_16816(accp[part], af, bp[part][0], bp[part][1]);
       }
       float acc[4];
 #pragma unroll
@@ -554,7 +553,7 @@ EncodeTiledFnC encoder() {
 }
 
 size_t route_cluster_smem() {
-  const size_t stage1 = (size_t)kOffWt + 3 * (size_t)kClExp * (kClMaxDChunk * 2 + 16);
+  const size_t stage1 = (size_t)kOffHat;   // the W_r and x slices
   const size_t stage4 = (size_t)kOffHat + (size_t)kClMaxTok * kMaxExperts * 4;
   return (stage1 > stage4 ? stage1 : stage4) + 1024;
 }
@@ -608,7 +607,7 @@ cudaError_t launch_cluster_common(const RouterArgs& a, const DispatchArgs* dsp,
     const cuuint32_t box[2] = {(cuuint32_t)kClExp, (cuuint32_t)DC};
     const cuuint32_t estr[2] = {1, 1};
     if (enc(&f.wmap, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, const_cast<float*>(a.w_r), dims, strides,
-            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+            box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
       return cudaErrorInvalidValue;
   }
