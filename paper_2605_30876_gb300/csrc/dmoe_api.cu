@@ -109,7 +109,7 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.yshared = take(sizeof(float) * T * dm);
   const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
   w.hdense = take(dec ? 2 * (E + 1) * (size_t)((T + 15) / 16 * 16) * (I > Is ? I : Is) : 0);
-  w.spec = take(dec ? sizeof(int32_t) * d.n_blocks * k : 0);
+  w.spec = take(dec ? sizeof(uint32_t) * d.n_blocks * spec_words((int)k) : 0);
   w.total = off;
   return w;
 }
@@ -170,11 +170,9 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
                        const float* bias, int32_t* topk_idx, float* topk_gate, int32_t* coreset,
                        int32_t* coreset_size, float* probs, void* ws, const Workspace& plan,
                        cudaStream_t s, const L2Prefetch& shared_pf = L2Prefetch(),
-                       const DispatchArgs* dsp = nullptr, int32_t* spec_ids = nullptr,
-                       int32_t* spec_cnt = nullptr) {
+                       const DispatchArgs* dsp = nullptr, uint32_t* spec_words = nullptr) {
   RouterArgs a{};
-  a.spec_ids = spec_ids;
-  a.spec_cnt = spec_cnt;
+  a.spec_words = spec_words;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.w_r = w_r;
   a.bias = bias;
@@ -225,12 +223,10 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
                         const int32_t* n_unique, const int32_t* unique_ids,
                         const int32_t* offsets, const int32_t* rows, const int32_t* pos,
                         void* y, void* ws, const Workspace& plan, cudaStream_t s,
-                        bool shared_prefetched = false, const int32_t* spec_ids = nullptr,
-                        int32_t* spec_cnt = nullptr) {
+                        bool shared_prefetched = false, uint32_t* spec_words = nullptr) {
   ExpertArgs a{};
   a.prefetch_shared = !shared_prefetched;
-  a.spec_ids = spec_ids;
-  a.spec_cnt = spec_cnt;
+  a.spec_words = spec_words;
   a.spec_blocks = desc->n_blocks;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.w_gate = w_gate;
@@ -380,20 +376,17 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   // early-published coresets, before the routing launch ends (only when every token keeps
   // the whole coreset, so that the coresets' union is the unique set)
   const int T = desc->n_blocks * desc->block_size;
-  int32_t* spec_ids = nullptr;
-  int32_t* spec_cnt = nullptr;
+  uint32_t* spec_w = nullptr;
   if (desc->mode == DMOE_ROUTE_BLOCK && desc->top_p <= 0.f && mask_top_k(*desc) == desc->top_k &&
       route_cluster_ok(T, desc->d_model, desc->n_experts) &&
       experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared)) {
-    spec_ids = at<int32_t>(workspace, plan.spec);
-    spec_cnt = at<int32_t>(workspace, plan.tickets) + kTicketSpec;
+    spec_w = at<uint32_t>(workspace, plan.spec);
   }
   st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
-                  shared_pf, &dsp, spec_ids, spec_cnt);
+                  shared_pf, &dsp, spec_w);
   if (st != DMOE_OK) return st;
   return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid, offs,
-                     rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_ids,
-                     spec_cnt);
+                     rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w);
 }
 
 dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) {

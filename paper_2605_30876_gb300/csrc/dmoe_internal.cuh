@@ -37,7 +37,6 @@ enum DevWhere : int32_t {
   kAtCombine = 6, kAtGather = 7,
 };
 constexpr int kRouteTickets = 256;
-constexpr int kTicketSpec = 64;   // tickets[64] (own 128-B line): coresets published
 constexpr int kRouteClusterCtas = 8;   // CTAs per cluster of the decode-size routing launch
 struct DevErrRecord {
   int32_t code;
@@ -161,10 +160,10 @@ struct RouterArgs {
   L2Prefetch shared_pf;   // the shared expert's weights (one "expert")
   bool probs_requested;   // the caller wants the scores in `probs`
   // block top-k (p <= 0) in the fused decode-size call: every block's coreset, which is
-  // then the block's routing, is published early here (k ids per block), and spec_cnt is
-  // raised once per block (release); nullptr otherwise
-  int32_t* spec_ids;
-  int32_t* spec_cnt;
+  // then the block's routing, is published early here: spec_words(k) words per block, three
+  // ids and a marker byte each, one 32-bit store per word (a word reads as zero until it is
+  // complete; zero between calls); nullptr otherwise
+  uint32_t* spec_words;
 };
 
 struct DispatchArgs {
@@ -210,9 +209,9 @@ struct ExpertArgs {
   DevErrRecord* err;
   bool prefetch_shared;   // the shared expert's weights were not prefetched by the router
   // decode-size path, block top-k: the unique experts are the union of the published
-  // coresets (RouterArgs::spec_ids), known before the routing launch ends; nullptr otherwise
-  const int32_t* spec_ids;
-  int32_t* spec_cnt;
+  // coresets (RouterArgs::spec_words), known before the routing launch ends; nullptr
+  // otherwise
+  uint32_t* spec_words;
   int spec_blocks;
   // shape
   int T, d, E, k, I, Is, n_max;
@@ -220,9 +219,13 @@ struct ExpertArgs {
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E);
 // gate-weighted combine of the expert rows into y (the last launch of both expert paths);
-// it also clears zero[0 .. n_zero) and *zero1 (when set) once the launch before it has ended
+// it also clears zero[0 .. n_zero) and zero2[0 .. n_zero2) once the launch before it has
+// ended
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = nullptr,
-                           int n_zero = 0, int32_t* zero1 = nullptr);
+                           int n_zero = 0, uint32_t* zero2 = nullptr, int n_zero2 = 0);
+
+// Words of one block's published coreset (three 8-bit ids and a marker byte per word).
+__host__ __device__ inline int spec_words(int k) { return (k + 2) / 3; }
 // Decode-sized forwards (T <= 64): one persistent launch over gate/up and down tiles of
 // every group, all tokens at once (no gather), then the combine.
 bool experts_decode_ok(int T, int d, int I, int Is);

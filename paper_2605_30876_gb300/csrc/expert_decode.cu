@@ -75,8 +75,8 @@ struct DParams {
   float* yshared;            // [T, d]
   int32_t* h_ready;          // [E+1]: published gate/up tiles per group (zero between calls;
                              // the combine launch clears them)
-  const int32_t* spec_ids;   // block top-k: published coresets [spec_blocks, k], or nullptr
-  const int32_t* spec_cnt;   // coresets published so far
+  const uint32_t* spec_words;   // block top-k: published coresets (spec_words(k) words per
+                                // block, three ids and a marker byte each), or nullptr
   int spec_blocks;
   DevErrRecord* err;
   int T, d, E, k, I, Is;
@@ -115,6 +115,7 @@ using ptx::bulk_store;
 using ptx::epi_all;
 using ptx::fence_proxy_async_global;
 using ptx::ld_acquire;
+using ptx::ld_relaxed_u32;
 using ptx::named_bar_sync;
 using ptx::red_release_add;
 using ptx::tma_store_2d;
@@ -175,29 +176,38 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   // block is routed to all k experts of its coreset), published by the routing launch
   // before it ends; the weight stream starts on them, and only the down epilogue waits for
   // the dispatch. Otherwise (or if the coresets do not come) everything waits for it.
-  bool spec = p.spec_ids != nullptr;
+  bool spec = p.spec_words != nullptr;
   if (spec) {
     if (warp == 0) {
-      int ok = 1;
-      if (lane == 0) {
-        const uint64_t t0 = ptx::globaltimer_ns();
-        while (ld_acquire(p.spec_cnt) < p.spec_blocks) {
-          if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {
-            ok = 0;
-            break;
+      // poll every block's words until all are nonzero; a nonzero word is complete (one
+      // 32-bit store), so its ids go into the mask as it is seen (or-ing twice is harmless)
+      const int nw = spec_words(p.k), total = p.spec_blocks * nw;
+      uint32_t m[kMaxExperts / 32] = {};
+      bool bad = false;
+      const uint64_t t0 = ptx::globaltimer_ns();
+      for (;;) {
+        bool all = true;
+        for (int i = lane; i < total; i += 32) {
+          const uint32_t w = ld_relaxed_u32(p.spec_words + i);
+          if (w == 0u) {
+            all = false;
+            continue;
           }
-          __nanosleep(64);
+          const int r0 = 3 * (i % nw);
+#pragma unroll
+          for (int j = 0; j < 3; ++j) {
+            if (r0 + j >= p.k) break;
+            const int e = (int)((w >> (8 * j)) & 0xffu);
+            if (e >= p.E) bad = true;
+            else m[e >> 5] |= 1u << (e & 31);
+          }
+        }
+        if (__all_sync(0xffffffffu, all)) break;
+        if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {   // the coresets did not come
+          bad = true;
+          break;
         }
       }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      uint32_t m[kMaxExperts / 32] = {};
-      bool bad = !ok;
-      if (ok)
-        for (int i = lane; i < p.spec_blocks * p.k; i += 32) {
-          const int e = __ldcg(p.spec_ids + i);
-          if (e < 0 || e >= p.E) bad = true;
-          else m[e >> 5] |= 1u << (e & 31);
-        }
       bad = __any_sync(0xffffffffu, bad);
 #pragma unroll
       for (int w = 0; w < kMaxExperts / 32; ++w) m[w] = __reduce_or_sync(0xffffffffu, m[w]);
@@ -786,8 +796,7 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.yslot = a.yslot;
   p.yshared = a.yshared;
   p.h_ready = a.h_ready;
-  p.spec_ids = a.spec_ids;
-  p.spec_cnt = a.spec_cnt;
+  p.spec_words = a.spec_words;
   p.spec_blocks = a.spec_blocks;
   p.err = a.err;
   p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
@@ -817,13 +826,14 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   // one CTA per SM; when the stream starts on the published coresets, the last routing
   // cluster still holds its SMs, and a CTA placed there would start only when it ends
   int grid = device_sm_count();
-  if (a.spec_ids != nullptr && grid > 2 * kRouteClusterCtas) grid -= kRouteClusterCtas;
+  if (a.spec_words != nullptr && grid > 2 * kRouteClusterCtas) grid -= kRouteClusterCtas;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
   cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
-  return launch_combine(a, s, a.h_ready, a.E + 1, a.spec_cnt);
+  return launch_combine(a, s, a.h_ready, a.E + 1, a.spec_words,
+                        a.spec_words != nullptr ? a.spec_blocks * spec_words(a.k) : 0);
 }
 
 }  // namespace dmoe

@@ -564,19 +564,19 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
 }
 
 // y[t, :] = bf16( sum_j g[t,j] * yslot[pos[t*k + j], :] (slot order) + yshared[t, :] );
-// block (0, 0) also clears `zero[0 .. n_zero)` and `*zero1` (counters of the launches
-// before, now done)
+// block (0, 0) also clears `zero[0 .. n_zero)` and `zero2[0 .. n_zero2)` (counters and
+// flags of the launches before, now done)
 __global__ void __launch_bounds__(256)
 combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshared,
                const int32_t* __restrict__ pos, const float* __restrict__ gate,
                __nv_bfloat16* __restrict__ y, int k, int d, int has_shared, int32_t* zero,
-               int n_zero, int32_t* zero1) {
+               int n_zero, uint32_t* zero2, int n_zero2) {
   pdl_launch_dependents();
   pdl_wait();
   KLOG(DMOE_KERNEL_COMBINE, 0);
   if (blockIdx.x == 0 && blockIdx.y == 0) {
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
-    if (zero1 != nullptr && threadIdx.x == 0) *zero1 = 0;
+    for (int i = threadIdx.x; i < n_zero2; i += blockDim.x) zero2[i] = 0u;
   }
   const int t = blockIdx.y;
   const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
@@ -757,12 +757,12 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero, int n_zero,
-                           int32_t* zero1) {
+                           uint32_t* zero2, int n_zero2) {
   dim3 cgrid((a.d / 4 + 255) / 256, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
   cudaError_t e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared,
                             a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero,
-                            zero1);
+                            zero2, n_zero2);
   prof_end(DMOE_KERNEL_COMBINE, s);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

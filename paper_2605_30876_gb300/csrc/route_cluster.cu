@@ -446,14 +446,15 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
       CT_AT(25);
-      if (a.spec_ids != nullptr) {
+      if (a.spec_words != nullptr) {
         // block top-k: the coreset (k experts) is the routing of every token of the block;
-        // publish it for the expert launch
-        if (tid < k) a.spec_ids[(size_t)b * k + tid] = order[tid];
-        __syncthreads();
-        if (tid == 0) {
-          __threadfence();
-          asm volatile("red.release.gpu.global.add.s32 [%0], 1;" ::"l"(a.spec_cnt) : "memory");
+        // publish it for the expert launch, three ids and a marker byte per word
+        const int nw = spec_words(k);
+        if (tid < nw) {
+          uint32_t w = 1u << 24;
+          for (int j = 0; j < 3 && 3 * tid + j < k; ++j) w |= (uint32_t)order[3 * tid + j] << (8 * j);
+          asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(a.spec_words + (size_t)b * nw + tid),
+                       "r"(w) : "memory");
         }
       }
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
