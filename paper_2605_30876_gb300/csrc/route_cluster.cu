@@ -236,7 +236,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       const int r0 = mt * 16 + g;                   // A rows r0, r0 + 8 (same swizzle phase)
       const int n = nt * 8 + g;                     // B column (expert) of this thread
       float accp[3][4] = {};
-#pragma unroll 2
+#pragma unroll 8
       for (int k0 = 0; k0 < DC; k0 += 16) {
         const int bx = k0 >> 6, c = (k0 & 63) >> 3;   // box, 16-B chunk of k0
         const uint8_t* xb = Xs + bx * TB * 128;
