@@ -520,6 +520,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       gu_unit(u, gi, m);
       const bool ok = epi_all(wait(&acc_full[acc], acc_phase, u));
       if (!ok) break;
+      if (first && et == 0) ED_AT(20);
       ptx::tc_fence_after();
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)(acc * p.n_pad);
       // the H tile (n_pad token rows x hg columns, bf16) is laid out in the staging tile as
@@ -529,21 +530,32 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
         float v[16];
         ptx::tmem_ld16(tbase + c0, v);
         ptx::tmem_ld_wait();
+        if (first && et == 0 && c0 == 0) ED_AT(23);
         float* buf = xchg + xb * (64 * kXStride);
         if (!is_gate && g_act) {
 #pragma unroll
           for (int c = 0; c < 16; ++c) buf[rr * kXStride + c] = v[c];
         }
         named_bar_sync(2, 128);
+        if (first && et == 0 && c0 == 0) ED_AT(24);
         if (is_gate && g_act) {
+          // all loads first, then all stores: interleaved, each load would wait for the store
+          // before it (the compiler cannot tell the two shared arrays apart), serialising
+          // the sixteen elements (~1300 cycles against ~300)
+          float uv[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) uv[c] = buf[rr * kXStride + c];
+          __nv_bfloat16 hv[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c) hv[c] = __float2bfloat16(silu_f(v[c]) * uv[c]);
           uint8_t* hcol = hbox + (rr >> 5) * p.n_pad * 64 + (rr & 31) * 2;
 #pragma unroll
           for (int c = 0; c < 16; ++c)
-            *reinterpret_cast<__nv_bfloat16*>(hcol + (c0 + c) * 64) =
-                __float2bfloat16(silu_f(v[c]) * buf[rr * kXStride + c]);
+            *reinterpret_cast<__nv_bfloat16*>(hcol + (c0 + c) * 64) = hv[c];
         }
         xb ^= 1;
       }
+      if (first && et == 0) ED_AT(25);
       ptx::tc_fence_before();
       ptx::mbar_arrive(&acc_empty[acc]);
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
@@ -552,9 +564,11 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       ptx::fence_proxy_async_smem();
       named_bar_sync(2, 128);
       if (et == 0) {
+        if (first) ED_AT(21);
         for (int j = 0; j < hg / 32; ++j)
           tma_store_2d(&tm.hst, hbox + j * p.n_pad * 64, m * hg + 32 * j, gi * p.n_pad);
         bulk_commit_wait_all();
+        if (first) ED_AT(22);
         fence_proxy_async_global();
         red_release_add(p.h_ready + gi, 1);
         if (first) ED_AT(4);
