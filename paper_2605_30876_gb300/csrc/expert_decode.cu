@@ -512,7 +512,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     const bool g_act = lane < rq;
     const int rr = (q & 1) * rq + lane;           // row within the hg-row slice
     const int n_mma = (p.T + 15) & ~15;
-    int acc = 0, xb = 0;
+    int acc = 0;
     uint32_t acc_phase = 0;
     bool first = true;
     for (int u = b; u < NGU; u += nb) {
@@ -526,34 +526,44 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       // the H tile (n_pad token rows x hg columns, bf16) is laid out in the staging tile as
       // hg / 32 row-major boxes of 32 columns, then stored by TMA
       uint8_t* hbox = reinterpret_cast<uint8_t*>(stage_t);
+      // per 16-token slice: every row's 16 values go to the exchange tile (gate rows
+      // 0..hg-1, up rows hg..2hg-1), then all 128 threads take hg / 8 adjacent columns of one
+      // token each (loads first, then the SwiGLU, then one 8- or 16-byte store)
+      const int cpt = hg >> 3, xc = et >> 3, col0 = (et & 7) * cpt;
+      uint8_t* hdst = hbox + (col0 >> 5) * p.n_pad * 64 + (col0 & 31) * 2;
       for (int c0 = 0; c0 < n_mma; c0 += 16) {
         float v[16];
         ptx::tmem_ld16(tbase + c0, v);
         ptx::tmem_ld_wait();
         if (first && et == 0 && c0 == 0) ED_AT(23);
-        float* buf = xchg + xb * (64 * kXStride);
-        if (!is_gate && g_act) {
+        if (g_act) {
+          float* xr = xchg + ((is_gate ? 0 : hg) + rr) * kXStride;
 #pragma unroll
-          for (int c = 0; c < 16; ++c) buf[rr * kXStride + c] = v[c];
+          for (int c = 0; c < 16; ++c) xr[c] = v[c];
         }
         named_bar_sync(2, 128);
         if (first && et == 0 && c0 == 0) ED_AT(24);
-        if (is_gate && g_act) {
-          // all loads first, then all stores: interleaved, each load would wait for the store
-          // before it (the compiler cannot tell the two shared arrays apart), serialising
-          // the sixteen elements (~1300 cycles against ~300)
-          float uv[16];
+        float gv[8], uv[8];
 #pragma unroll
-          for (int c = 0; c < 16; ++c) uv[c] = buf[rr * kXStride + c];
-          __nv_bfloat16 hv[16];
+        for (int j = 0; j < 8; ++j)
+          if (j < cpt) {
+            gv[j] = xchg[(col0 + j) * kXStride + xc];
+            uv[j] = xchg[(hg + col0 + j) * kXStride + xc];
+          }
+        uint32_t hp[4];
 #pragma unroll
-          for (int c = 0; c < 16; ++c) hv[c] = __float2bfloat16(silu_f(v[c]) * uv[c]);
-          uint8_t* hcol = hbox + (rr >> 5) * p.n_pad * 64 + (rr & 31) * 2;
-#pragma unroll
-          for (int c = 0; c < 16; ++c)
-            *reinterpret_cast<__nv_bfloat16*>(hcol + (c0 + c) * 64) = hv[c];
-        }
-        xb ^= 1;
+        for (int j = 0; j < 4; ++j)
+          if (2 * j < cpt) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(silu_f(gv[2 * j]) * uv[2 * j],
+                                                            silu_f(gv[2 * j + 1]) * uv[2 * j + 1]);
+            hp[j] = *reinterpret_cast<const uint32_t*>(&h2);
+          }
+        uint8_t* hrow = hdst + (c0 + xc) * 64;
+        if (cpt == 4)
+          *reinterpret_cast<uint2*>(hrow) = make_uint2(hp[0], hp[1]);
+        else
+          *reinterpret_cast<uint4*>(hrow) = make_uint4(hp[0], hp[1], hp[2], hp[3]);
+        named_bar_sync(2, 128);   // the exchange tile is rewritten by the next slice
       }
       if (first && et == 0) ED_AT(25);
       ptx::tc_fence_before();
