@@ -39,6 +39,8 @@ ROUTING_CASES = {
     "tiny_fewer_k1_of2": TINY.with_(top_k=1, block_top_k=2),
     "tiny_fewer_k3_of16_p03": TINY.with_(top_k=3, block_top_k=16, top_p=0.3),
     "stack_fewer_k4_of8": STACK20.with_(top_k=4, block_top_k=8),
+    # blocks whose score rows do not fit one CTA's shared memory (two-launch block routing)
+    "block_size_128": LAYER.with_(block_size=128, n_blocks=2, top_p=0.6),
     # the Top-4 token-level baseline
     "layer_token_top4": LAYER.with_(mode=ROUTE_TOKEN, top_k=4),
 }
