@@ -548,6 +548,189 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
     del weights
 
 
+# ----------------------------------------------------------------------------- decode sim
+def run_decode_sim(args, torch, dm, MoELayer):
+    """A synthetic block-diffusion decoding loop around the MoE stack, one JSON line per
+    routing: how much of a denoising step the MoE layers take, and how the unique-expert
+    count U varies across steps (its coefficient of variation, the statistic of the paper's
+    Table 1).
+
+    Model stand-in (random weights; only the costs and the data flow are real): one
+    sequence, a block of 32 positions decoded at a time; per step every position of the
+    block passes 20 layers, each an attention stand-in (RMS norm, q/k/v/o projections,
+    16 heads of 128 over a 1024-token cached context plus the block, by torch SDPA) and the
+    MoE layer of the benchmark shape (this library; RMS-normalised input, residual add),
+    then a tied embedding / LM head of a 128k vocabulary; the block's positions carry
+    position embeddings. The stand-ins are plain torch, not tuned: their share is an upper
+    bound of what a tuned attention would take. Unmasking: every masked position
+    whose top softmax probability reaches 0.95 takes its argmax token, at least the most
+    confident one per step; the logit scale is fixed once so that about two of the 32
+    masked positions of the first step pass. A block ends when all its positions are
+    unmasked; the next block starts fully masked over the same context.
+
+    Each step is one CUDA graph replay (its device time is the step latency); the MoE and
+    attention shares come from graphs of the 20 MoE layers alone and the 20 attention
+    stand-ins alone, replayed on the same step's inputs."""
+    from dmoe_synth import LAYER, ROUTE_BLOCK, ROUTE_TOKEN, STACK20_LAYERS, layer_inputs
+    NL, B, V, H, HD, CTX = STACK20_LAYERS, 32, 128000, 16, 128, 1024
+    d = LAYER.d_model
+    g = torch.Generator(device="cuda")
+    g.manual_seed(args.seed + 77)
+
+    def rnd(*shape, std=1.0):
+        return (torch.randn(*shape, generator=g, device="cuda") * std).to(torch.bfloat16)
+
+    w_head = rnd(V, d, std=0.02)              # tied embedding and LM head
+    e_mask = rnd(d, std=0.02)
+    pos = rnd(B, d, std=0.02)                 # position embeddings of the block
+    # per layer: q|k|v projection [d, 3d], o projection [d, d]; K and V of the cached context
+    # followed by the block's own rows (written in place every step)
+    attn_w = [(rnd(d, 3 * d, std=d ** -0.5), rnd(d, d, std=d ** -0.5)) for _ in range(NL)]
+    kv = [(rnd(1, H, CTX + B, HD), rnd(1, H, CTX + B, HD)) for _ in range(NL)]
+    moe_w = [layer_inputs(LAYER, seed=args.seed + 2000 + l, device="cuda", layer=l)
+             for l in range(NL)]
+    x_in = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
+    xs = [torch.empty(B, d, dtype=torch.bfloat16, device="cuda") for _ in range(2 * NL + 1)]
+    us = [torch.empty(B, d, dtype=torch.bfloat16, device="cuda") for _ in range(NL)]
+    conf = torch.empty(B, dtype=torch.float32, device="cuda")
+    arg = torch.empty(B, dtype=torch.int64, device="cuda")
+    scale = torch.ones(1, dtype=torch.float32, device="cuda")
+
+    def rms(x):
+        return torch.nn.functional.rms_norm(x, (d,), eps=1e-6)
+
+    def attn(l, x, out):
+        wqkv, wo = attn_w[l]
+        qkv = (rms(x) @ wqkv).view(B, 3, H, HD)
+        k, v = kv[l]
+        k[0, :, CTX:].copy_(qkv[:, 1].transpose(0, 1))
+        v[0, :, CTX:].copy_(qkv[:, 2].transpose(0, 1))
+        o = torch.nn.functional.scaled_dot_product_attention(qkv[:, 0].transpose(0, 1)[None], k, v)
+        torch.add(x, o[0].transpose(0, 1).reshape(B, d) @ wo, out=out)
+
+    def moe(l, L, x, out):
+        us[l].copy_(rms(x))
+        torch.add(x, L.forward(us[l]), out=out)
+
+    def head(x):
+        logits = (rms(x) @ w_head.t()).float() * scale
+        p = torch.softmax(logits, dim=-1)
+        c, a = p.max(dim=-1)
+        conf.copy_(c)
+        arg.copy_(a)
+
+    def capture(fn):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr):
+            fn()
+        return gr
+
+    def timed(gr, reps=3):
+        st, en = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        best = None
+        for _ in range(reps):
+            st.record()
+            gr.replay()
+            en.record()
+            torch.cuda.synchronize()
+            t = st.elapsed_time(en) * 1e-3
+            best = t if best is None else min(best, t)
+        return best
+
+    modes = [("block_p0", LAYER), ("block_p0.6", LAYER.with_(top_p=0.6)),
+             ("token", LAYER.with_(mode=ROUTE_TOKEN))]
+    n_blocks = args.sim_blocks
+    for name, shape in modes:
+        layers = [MoELayer.from_shape(shape, moe_w[l]) for l in range(NL)]
+
+        def step_fn():
+            x = x_in
+            for l in range(NL):
+                attn(l, x, xs[2 * l])
+                moe(l, layers[l], xs[2 * l], xs[2 * l + 1])
+                x = xs[2 * l + 1]
+            head(x)
+
+        def moe_fn():
+            for l in range(NL):
+                moe(l, layers[l], xs[2 * l], xs[2 * l + 1])
+
+        def attn_fn():
+            x = x_in
+            for l in range(NL):
+                attn(l, x, xs[2 * l])
+                x = xs[2 * l + 1]
+
+        tokens = torch.zeros(B, dtype=torch.int64, device="cuda")
+        masked = torch.ones(B, dtype=torch.bool, device="cuda")
+
+        def embed():
+            x_in.copy_(torch.where(masked[:, None], e_mask[None, :], w_head[tokens]) + pos)
+
+        embed()
+        g_step, g_moe, g_attn = capture(step_fn), capture(moe_fn), capture(attn_fn)
+        # logit scale: about two of the first step's 32 masked positions reach 0.95
+        g_step.replay()
+        torch.cuda.synchronize()
+        lo, hi = 1.0, 1e4
+        for _ in range(40):
+            mid = (lo * hi) ** 0.5
+            scale.fill_(mid)
+            head(xs[2 * NL - 1])
+            n_pass = int((conf >= 0.95).sum().item())
+            lo, hi = (mid, hi) if n_pass < 2 else (lo, mid)
+        scale.fill_(hi)
+        t_step, t_moe, t_attn, U, per_step = [], [], [], [], []
+        blocks_done = 0
+        while blocks_done < n_blocks:
+            embed()
+            t_step.append(timed(g_step, 1))
+            U.append([int(L.n_unique.item()) for L in layers])
+            if len(t_step) % 4 == 1:      # component graphs on this step's inputs
+                t_moe.append(timed(g_moe))
+                t_attn.append(timed(g_attn))
+                g_step.replay()           # the state the unmasking below reads
+                torch.cuda.synchronize()
+            c = torch.where(masked, conf, torch.full_like(conf, -1.0))
+            take = masked & (c >= 0.95)
+            if not bool(take.any()):
+                take = torch.zeros_like(masked)
+                take[int(c.argmax().item())] = True
+            tokens = torch.where(take, arg, tokens)
+            masked = masked & ~take
+            per_step.append(int(take.sum().item()))
+            if not bool(masked.any()):
+                blocks_done += 1
+                masked = torch.ones_like(masked)
+        for L in layers:
+            st_, info = dm.dmoe_get_device_error(L.ws)
+            if st_ != 0:
+                raise RuntimeError(f"device fault {info}")
+        Ua = np.array(U, dtype=np.float64)
+        mid = NL // 2
+        step_us = float(np.mean(t_step)) * 1e6
+        moe_us, attn_us = float(np.mean(t_moe)) * 1e6, float(np.mean(t_attn)) * 1e6
+        print(json.dumps({
+            "suite": "decode_sim", "routing": name, "layers": NL, "block_size": B,
+            "vocab": V, "context": CTX, "blocks": n_blocks, "steps": len(t_step),
+            "tokens_per_step_mean": float(np.mean(per_step)),
+            "step_us_mean": step_us, "moe_us": moe_us, "attention_us": attn_us,
+            "other_us": max(step_us - moe_us - attn_us, 0.0), "moe_share": moe_us / step_us,
+            "attention_share": attn_us / step_us,
+            f"U_layer{mid}_mean": float(Ua[:, mid].mean()),
+            f"U_layer{mid}_cv": float(Ua[:, mid].std() / max(Ua[:, mid].mean(), 1e-9)),
+            "U_mean_all_layers": float(Ua.mean()),
+            "U_cv_per_layer_mean": float(np.mean(Ua.std(0) / np.maximum(Ua.mean(0), 1e-9))),
+            "note": "synthetic stand-ins for attention, embeddings and LM head; MoE by this "
+                    "library; shares from graphs of each component replayed on the step's "
+                    "inputs"}), flush=True)
+        del layers, g_step, g_moe, g_attn
+        torch.cuda.empty_cache()
+
+
 # ----------------------------------------------------------------------------- main
 def main():
     ap = argparse.ArgumentParser()
@@ -567,6 +750,10 @@ def main():
     ap.add_argument("--suite", action="store_true",
                     help="measure the other workloads instead of the headline (one JSON line "
                          "per point; one GPU)")
+    ap.add_argument("--decode-sim", action="store_true",
+                    help="the synthetic block-diffusion decoding loop around the MoE stack "
+                         "(MoE share of a step, CV of U across steps; one GPU)")
+    ap.add_argument("--sim-blocks", type=int, default=4)
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -595,6 +782,9 @@ def main():
     if args.suite:
         run_suite(args, torch, dm, MoELayer, hbm,
                   float(peaks.get("bf16_tflops_sustained", 1700.0)))
+        return
+    if args.decode_sim:
+        run_decode_sim(args, torch, dm, MoELayer)
         return
     sampler = ClockSampler(gpu_uuid(torch)) if rank == 0 else None
 
