@@ -2,6 +2,7 @@
 // expert -> (token, slot) lists (see dispatch_impl.cuh for the method).
 #include "dispatch_impl.cuh"
 #include "dmoe_internal.cuh"
+#include "trace_log.cuh"
 
 namespace dmoe {
 namespace {
@@ -19,7 +20,9 @@ dispatch_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
   uint16_t* base = reinterpret_cast<uint16_t*>(bits + (size_t)nchunks * E);  // [nchunks][E]
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(DMOE_KERNEL_DISPATCH, 0);
   dispatch_cta(topk_idx, T, E, k, n_unique, unique_ids, offsets, rows, pos, err, bits, base);
+  KLOG(DMOE_KERNEL_DISPATCH, 1);
 }
 
 }  // namespace
@@ -51,3 +54,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s) {
 }
 
 }  // namespace dmoe
+
+#ifdef DMOE_TRACE
+DMOE_KLOG_EXPORT(dmoe_debug_klog_dispatch)
+#endif

@@ -323,7 +323,10 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
   // then publishes the cluster at GPU scope
   cluster_sync();
   CT_AT(3);
-  if (f.logits_only) return;
+  if (f.logits_only) {
+    KLOG(DMOE_KERNEL_ROUTER, 1);
+    return;
+  }
 
   // ---- 2. the last cluster to finish routes the forward
   if (rank == 0 && tid == 0) {
@@ -553,10 +556,14 @@ EncodeTiledFnC encoder() {
   return fn;
 }
 
-size_t route_cluster_smem() {
-  const size_t stage1 = (size_t)kOffHat;   // the W_r and x slices
+// Dynamic shared memory of a launch: the W_r and x slices, and for a routing launch the
+// TopKMask rows after them (a logits-only launch stops before it needs them, and its
+// smaller footprint lets two CTAs share an SM, so that the 64-token tiles of a large
+// forward run in one wave)
+size_t route_cluster_smem(bool logits_only) {
+  const size_t stage1 = (size_t)kOffHat;
   const size_t stage4 = (size_t)kOffHat + (size_t)kClMaxTok * kMaxExperts * 4;
-  return (stage1 > stage4 ? stage1 : stage4) + 1024;
+  return (logits_only || stage1 > stage4 ? stage1 : stage4) + 1024;
 }
 
 }  // namespace
@@ -627,13 +634,15 @@ cudaError_t launch_cluster_common(const RouterArgs& a, const DispatchArgs* dsp,
   if (dsp != nullptr) f.dsp = *dsp;
   f.ticket = tickets;
   f.logits_only = logits_only ? 1 : 0;
-  const size_t smem = route_cluster_smem();
+  const size_t smem = route_cluster_smem(logits_only);
+  const size_t smem_max = route_cluster_smem(false);
   static int mask = 0;
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 31 || !(mask & (1 << dev))) {
     cudaError_t e = cudaFuncSetAttribute(route_cluster_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)smem_max);
     if (e != cudaSuccess) return e;
     if (dev < 31) mask |= 1 << dev;
   }

@@ -16,6 +16,7 @@
 #include "block_reduce.cuh"
 #include "dmoe_internal.cuh"
 #include "routing_device.cuh"
+#include "trace_log.cuh"
 
 namespace dmoe {
 namespace {
@@ -93,11 +94,13 @@ router_softmax_kernel(const float* __restrict__ part, int splits, const float* _
                       int T, int E, int k, int mode) {
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(5, 0);
   const int t = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (t >= T) return;
   token_route_warp(part + (size_t)t * E, splits, (size_t)T * E, bias, E, k, mode,
                    probs + (size_t)t * E, probs_hat + (size_t)t * E, topk_idx + (size_t)t * k,
                    topk_gate + (size_t)t * k);
+  KLOG(5, 1);
 }
 
 __global__ void __launch_bounds__(256)
@@ -107,8 +110,10 @@ block_route_kernel(const float* __restrict__ probs, const float* __restrict__ pr
                    int32_t* __restrict__ coreset, int32_t* __restrict__ coreset_size) {
   pdl_launch_dependents();
   pdl_wait();
+  KLOG(6, 0);
   block_route_cta(blockIdx.x, probs, probs_hat, E, kb, k, B, top_p, topk_idx, topk_gate, coreset,
                   coreset_size);
+  KLOG(6, 1);
 }
 
 }  // namespace
@@ -159,3 +164,7 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
 }
 
 }  // namespace dmoe
+
+#ifdef DMOE_TRACE
+DMOE_KLOG_EXPORT(dmoe_debug_klog_routerg)
+#endif

@@ -338,6 +338,29 @@ template <class ProbFn, class OutFn>
 __device__ inline void mask_topk_warps(int k, int B, int size, const int* order, ProbFn prob,
                                        OutFn out) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (size <= 32) {
+    // one member per lane: k rounds of a tournament (larger score, ties to the lower id)
+    const int e = lane < size ? order[lane] : -1;
+    for (int i = warp; i < B; i += (int)(blockDim.x >> 5)) {
+      uint32_t key = e >= 0 ? order_key(prob(i, e)) : 0u;
+      int my_e = -1;
+      float my_v = 0.f;
+      for (int r = 0; r < k; ++r) {
+        const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+        const uint32_t imin =
+            __reduce_min_sync(0xffffffffu, key == kmax ? (uint32_t)e : 0xffffffffu);
+        if (lane == r) {
+          my_e = (int)imin;
+          my_v = key_value(kmax);
+        }
+        if (key == kmax && (uint32_t)e == imin) key = 0u;
+      }
+      float g = 0.f;
+      for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
+      if (lane < k) out(i, lane, my_e, my_v / g);
+    }
+    return;
+  }
   for (int i = warp; i < B; i += (int)(blockDim.x >> 5)) {
     float cv[8];
     int ce[8];
