@@ -13,6 +13,19 @@
 // Every reduction runs in a fixed order, so the routing is identical from run to run.
 #include <math.h>
 
+#ifdef DMOE_TRACE
+#include <stdint.h>
+// Debug builds: per-CTA phase stamps of the block routing kernel (%globaltimer, ns)
+__device__ uint64_t g_brtrace[64 * 32];
+#define DMOE_STAMP(st)                                                               \
+  do {                                                                               \
+    if (threadIdx.x == 0 && blockIdx.x < 64) {                                       \
+      uint64_t t_;                                                                   \
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                         \
+      g_brtrace[blockIdx.x * 32 + (st)] = t_;                                        \
+    }                                                                                \
+  } while (0)
+#endif
 #include "block_reduce.cuh"
 #include "dmoe_internal.cuh"
 #include "routing_device.cuh"
@@ -111,6 +124,7 @@ block_route_kernel(const float* __restrict__ probs, const float* __restrict__ pr
   pdl_launch_dependents();
   pdl_wait();
   KLOG(6, 0);
+  DMOE_STAMP(0);
   block_route_cta(blockIdx.x, probs, probs_hat, E, kb, k, B, top_p, topk_idx, topk_gate, coreset,
                   coreset_size);
   KLOG(6, 1);
@@ -167,4 +181,7 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
 
 #ifdef DMOE_TRACE
 DMOE_KLOG_EXPORT(dmoe_debug_klog_routerg)
+extern "C" int dmoe_debug_brtrace(void* host) {
+  return (int)cudaMemcpyFromSymbol(host, g_brtrace, sizeof(g_brtrace));
+}
 #endif

@@ -440,8 +440,10 @@ __device__ inline void block_route_steps(int E, int kb, int k, int B, float top_
                                          int32_t* __restrict__ coreset_size) {
   __shared__ int order[kMaxExperts];
   const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size);
+  DMOE_STAMP(25);
   mask_topk_warps(k, B, size, order, prob, out);
   __syncthreads();
+  DMOE_STAMP(26);
 }
 
 // Algorithm 1 for block b with the block's rows in global memory ([T, E] row-major). The
