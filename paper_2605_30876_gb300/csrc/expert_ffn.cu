@@ -115,7 +115,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   const uint32_t off_a = 0;
   const uint32_t off_b = off_a + (uint32_t)stages * kAStageBytes;
   const uint32_t off_x = off_b + (uint32_t)stages * b_stage;
-  const uint32_t x_bytes = 2u * 64u * kXchgStride * 4u;        // 2 buffers [64][17] fp32
+  const uint32_t x_bytes = 2u * 64u * kXchgStride * 4u;        // [128][17] fp32
   const uint32_t off_bar = (off_x + x_bytes + 7u) & ~7u;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + off_bar);
   uint64_t* empty = full + stages;
@@ -465,7 +465,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     // ================= epilogue: warps 2..5, TMEM lanes 32*(warp%4) ..
     const int q = warp & 3;
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
-    int acc = 0, xb = 0, li = 0;
+    int acc = 0, li = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++li) {
       const Unit un = decode(u);
@@ -484,25 +484,39 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         const int Ig = shared ? p.Is : p.I;
         __nv_bfloat16* hout = shared ? p.hs : p.h;
         const int hrow0 = (shared ? 0 : g_row0[un.g]) + col0;
-        const int icol = un.m * 64 + r64;
+        // per 16-token slice: every accumulator row's 16 values go to the exchange tile
+        // (gate rows 0-63, up rows 64-127), then each of the 128 threads takes 8 adjacent
+        // H columns of one token (loads, SwiGLU, one 16-byte store). Interleaving the
+        // exchange loads with the H stores instead serialises them: the compiler cannot
+        // tell the two memories apart.
+        const int et = tid - 64, xc = et >> 3, hc = (et & 7) * 8;
         for (int c0 = 0; c0 < n_mma; c0 += 16) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
           ptx::tmem_ld_wait();
-          float* buf = xchg + xb * (64 * kXchgStride);
-          if (!is_gate) {
+          {
+            float* xr = xchg + ((is_gate ? 0 : 64) + r64) * kXchgStride;
 #pragma unroll
-            for (int c = 0; c < 16; ++c) buf[r64 * kXchgStride + c] = v[c];
+            for (int c = 0; c < 16; ++c) xr[c] = v[c];
           }
           named_bar_sync(2, 128);
-          if (is_gate) {
+          float gv[8], uv[8];
 #pragma unroll
-            for (int c = 0; c < 16; ++c)
-              if (c0 + c < nvalid)
-                hout[(size_t)(hrow0 + c0 + c) * Ig + icol] =
-                    __float2bfloat16(silu_f(v[c]) * buf[r64 * kXchgStride + c]);
+          for (int j = 0; j < 8; ++j) {
+            gv[j] = xchg[(hc + j) * kXchgStride + xc];
+            uv[j] = xchg[(64 + hc + j) * kXchgStride + xc];
           }
-          xb ^= 1;
+          uint32_t hp[4];
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(silu_f(gv[2 * j]) * uv[2 * j],
+                                                            silu_f(gv[2 * j + 1]) * uv[2 * j + 1]);
+            hp[j] = *reinterpret_cast<const uint32_t*>(&h2);
+          }
+          if (c0 + xc < nvalid)
+            *reinterpret_cast<uint4*>(hout + (size_t)(hrow0 + c0 + xc) * Ig + un.m * 64 + hc) =
+                make_uint4(hp[0], hp[1], hp[2], hp[3]);
+          named_bar_sync(2, 128);   // the exchange tile is rewritten by the next slice
         }
         if (tid == 64 && li < 4) DMOE_TRACE_AT(54 + li);
         ptx::tc_fence_before();
