@@ -187,10 +187,12 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 //
 // Top-P accumulates the sorted values in order in fp32 and stops at the first running sum
 // >= p (p >= 1: at the last nonzero entry); the floor extends the coreset to k entries
-// (zero entries in id order). For p < 1 every warp sorts its 32 entries by rank, then one
-// warp merges the sorted lists by a tournament over their heads until both rules are met;
-// for p >= 1 every nonzero S~ counts the nonzero entries that beat it (larger, or equal
-// with a lower id), all in parallel. Needs blockDim.x == kMaxExperts.
+// (zero entries in id order). For p <= 0 (block top-k) the coreset is the k largest sums,
+// taken by one warp without the normalisation. For 0 < p < 1 every warp sorts its 32
+// entries by rank, then one warp merges the sorted lists by a tournament over their heads
+// until both rules are met; for p >= 1 every nonzero S~ counts the nonzero entries that
+// beat it (larger, or equal with a lower id), all in parallel. Needs blockDim.x ==
+// kMaxExperts.
 template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
@@ -215,6 +217,35 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
       for (int u = 0; u < 8; ++u)
         if (i0 + u < B) S += h[u];
     }
+  }
+  if (top_p <= 0.f) {
+    // p <= 0 (block top-k): Top-P stops at the first entry and the floor extends the coreset
+    // to the k best. S~ = S / sum(S) has the order of S (exactly so, where the fp32 division
+    // would round two sums to one value), so the k best sums are taken directly: warp 0
+    // holds all E sums, eight per lane, and selects them by a sort and k reductions.
+    st_s[tid] = live ? S : 0.f;
+    __syncthreads();
+    if (warp == 0) {
+      float v[8];
+      int id[8];
+      uint32_t valid = 0;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int e = lane + 32 * j;
+        id[j] = e;
+        v[j] = e < E ? st_s[e] : 0.f;
+        if (e < E) valid |= 1u << j;
+      }
+      int my_e;
+      float my_v;
+      warp_topk(v, id, valid, k, my_e, my_v);
+      if (lane < k) order[lane] = my_e;
+    }
+    __syncthreads();
+    if (coreset != nullptr && live) coreset[tid] = (tid < k) ? order[tid] : -1;
+    if (coreset_size != nullptr && tid == 0) coreset_size[0] = k;
+    __syncthreads();   // st_s and order are rewritten by a later block of the same CTA
+    return k;
   }
   // Normalize: L1
   const float tot = block_sum(S, fscr);
