@@ -172,6 +172,7 @@ class Arm:
         if on and not hasattr(self, "x_host"):
             self.x_host = [x.cpu().pin_memory() for x in self.x]
             self.y_host = [self.torch.empty_like(x, device="cpu").pin_memory() for x in self.x]
+            self.s_in, self.s_out = self.torch.cuda.Stream(), self.torch.cuda.Stream()
 
     def step(self, i):
         L = self.layers[i % len(self.layers)]
@@ -198,13 +199,53 @@ class Arm:
         torch = self.torch
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
-            for i in range(n_steps):
+            if self.host_io:
+                self.capture_host_io(n_steps, first)
+            else:
+                for i in range(n_steps):
+                    if events is not None:
+                        self.dm.dmoe_set_profile_events("experts", *events[i])
+                    self.step(first + i)
                 if events is not None:
-                    self.dm.dmoe_set_profile_events("experts", *events[i])
-                self.step(first + i)
-            if events is not None:
-                self.dm.dmoe_set_profile_events("experts", None, None)
+                    self.dm.dmoe_set_profile_events("experts", None, None)
         return g
+
+    def capture_host_io(self, n_steps, first):
+        """Steps with x copied in from pinned host memory and y copied back, pipelined one
+        step deep as a double-buffered serving loop would run them: the copy of step j+1's x
+        (on its own stream) starts once step j-1's forward has ended and overlaps step j's
+        forward; the copy of y_j back overlaps step j+1's forward. Every step's two copies
+        are inside the captured steps."""
+        torch = self.torch
+        main = torch.cuda.current_stream()
+        n = len(self.layers)
+        self.s_in.wait_stream(main)
+        self.s_out.wait_stream(main)
+        ev_x = [torch.cuda.Event() for _ in range(n_steps)]
+        ev_y = [torch.cuda.Event() for _ in range(n_steps)]
+
+        def copy_in(j):
+            idx = (first + j) % n
+            with torch.cuda.stream(self.s_in):
+                if j >= 2:
+                    self.s_in.wait_event(ev_y[j - 2])
+                self.x[idx].copy_(self.x_host[idx], non_blocking=True)
+                ev_x[j].record(self.s_in)
+
+        if n_steps > 0:
+            copy_in(0)
+        for j in range(n_steps):
+            if j + 1 < n_steps:
+                copy_in(j + 1)
+            idx = (first + j) % n
+            main.wait_event(ev_x[j])
+            y = self.layers[idx].forward(self.x[idx])
+            ev_y[j].record(main)
+            with torch.cuda.stream(self.s_out):
+                self.s_out.wait_event(ev_y[j])
+                self.y_host[idx].copy_(y, non_blocking=True)
+        main.wait_stream(self.s_in)
+        main.wait_stream(self.s_out)
 
 
 def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):

@@ -8,7 +8,8 @@
 //      give the partial logits [T x 32], pushed over distributed shared memory to the CTA
 //      that owns each token (t mod 8); CTA r then adds, in rank order, the eight partials of
 //      its tokens and writes those logits.
-//   2. one atomic ticket: the last cluster to finish continues; the others exit.
+//   2. one atomic ticket per CTA: the cluster of the last CTA to finish continues; the
+//      others exit.
 //   3. scores: one warp per token (8 CTAs x 8 warps = 64 tokens): softmax, top-k (token
 //      mode: the routing; block mode: TopKMask, whose k nonzeros are stored straight into
 //      the shared memory of the CTA that routes the token's block).
@@ -198,6 +199,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           : "memory");
   }
   for (int e = tid; e < E; e += 256) s_bias[e] = a.bias != nullptr ? a.bias[e] : 0.f;
+  if (tid == 0) s_last = 0u;   // set by the last CTA's ticket (after the next cluster barrier)
   __syncthreads();
   {
     uint64_t t0;
@@ -319,22 +321,23 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
       }
     }
   }
-  // every CTA of the cluster has written its logits and candidates (cluster scope); rank 0
-  // then publishes the cluster at GPU scope
-  cluster_sync();
+  // this CTA's logits and candidates are written (no shared memory of a peer is touched
+  // after this point unless the cluster goes on)
+  __syncthreads();
   CT_AT(3);
   if (f.logits_only) {
     KLOG(DMOE_KERNEL_ROUTER, 1);
     return;
   }
 
-  // ---- 2. the last cluster to finish routes the forward
-  if (rank == 0 && tid == 0) {
-    // release this cluster's logits and candidates, acquire the others' (GPU scope)
+  // ---- 2. the cluster of the last CTA to finish routes the forward: one ticket per CTA
+  // (releases this CTA's logits and candidates, acquires everyone's at GPU scope); the last
+  // CTA flags its cluster, whose barrier then passes the acquired writes on to its peers
+  if (tid == 0) {
     uint32_t old;
     asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;" : "=r"(old) : "l"(f.ticket) : "memory");
-    const uint32_t last = (old == (uint32_t)n_clusters - 1) ? 1u : 0u;
-    for (uint32_t q = 0; q < (uint32_t)kCl; ++q) st_peer_u32(peer_addr(&s_last, q), last);
+    if (old == (uint32_t)(n_clusters * kCl) - 1)
+      for (uint32_t q = 0; q < (uint32_t)kCl; ++q) st_peer_u32(peer_addr(&s_last, q), 1u);
   }
   cluster_sync();
   if (!s_last) {
