@@ -220,9 +220,11 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E);
 // gate-weighted combine of the expert rows into y (the last launch of both expert paths);
 // it also clears zero[0 .. n_zero) and zero2[0 .. n_zero2) once the launch before it has
-// ended
+// ended. meta_early: the slot indices and gates may be read before that launch ends (they
+// were complete before it released the combine)
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = nullptr,
-                           int n_zero = 0, uint32_t* zero2 = nullptr, int n_zero2 = 0);
+                           int n_zero = 0, uint32_t* zero2 = nullptr, int n_zero2 = 0,
+                           bool meta_early = false);
 
 // Words of one block's published coreset (three 8-bit ids and a marker byte per word).
 __host__ __device__ inline int spec_words(int k) { return (k + 2) / 3; }

@@ -856,8 +856,11 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
+  // the expert launch releases the combine at its end, after its wait for the routing
+  // launch (which wrote the slot indices and gates): the combine may read them at once
   return launch_combine(a, s, a.h_ready, a.E + 1, a.spec_words,
-                        a.spec_words != nullptr ? a.spec_blocks * spec_words(a.k) : 0);
+                        a.spec_words != nullptr ? a.spec_blocks * spec_words(a.k) : 0,
+                        /*meta_early=*/true);
 }
 
 }  // namespace dmoe

@@ -579,35 +579,61 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
 
 // y[t, :] = bf16( sum_j g[t,j] * yslot[pos[t*k + j], :] (slot order) + yshared[t, :] );
 // block (0, 0) also clears `zero[0 .. n_zero)` and `zero2[0 .. n_zero2)` (counters and
-// flags of the launches before, now done)
+// flags of the launches before, now done). With meta_early the slot indices and gates are
+// read before the dependency wait: the caller guarantees that they were complete before the
+// launch before this one could let this one start (the decode-size expert launch releases
+// it only at its end, after its own wait for the routing launch that wrote them).
 __global__ void __launch_bounds__(256)
 combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshared,
                const int32_t* __restrict__ pos, const float* __restrict__ gate,
                __nv_bfloat16* __restrict__ y, int k, int d, int has_shared, int32_t* zero,
-               int n_zero, uint32_t* zero2, int n_zero2) {
+               int n_zero, uint32_t* zero2, int n_zero2, int meta_early) {
   pdl_launch_dependents();
+  const int t = blockIdx.y;
+  const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  int r[kMaxTopK];
+  float gj[kMaxTopK];
+  if (meta_early) {
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j)
+      if (j < k) {
+        r[j] = __ldcg(pos + t * k + j);
+        gj[j] = __ldcg(gate + t * k + j);
+      }
+  }
   pdl_wait();
   KLOG(DMOE_KERNEL_COMBINE, 0);
   if (blockIdx.x == 0 && blockIdx.y == 0) {
     for (int i = threadIdx.x; i < n_zero; i += blockDim.x) zero[i] = 0;
     for (int i = threadIdx.x; i < n_zero2; i += blockDim.x) zero2[i] = 0u;
   }
-  const int t = blockIdx.y;
-  const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
   if (c >= d) return;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-  for (int j = 0; j < k; ++j) {
-    const int r = pos[t * k + j];
-    const float gj = gate[t * k + j];
-    const float4 v = *reinterpret_cast<const float4*>(yslot + (size_t)r * d + c);
-    acc.x = fmaf(gj, v.x, acc.x);
-    acc.y = fmaf(gj, v.y, acc.y);
-    acc.z = fmaf(gj, v.z, acc.z);
-    acc.w = fmaf(gj, v.w, acc.w);
+  if (!meta_early) {
+#pragma unroll
+    for (int j = 0; j < kMaxTopK; ++j)
+      if (j < k) {
+        r[j] = pos[t * k + j];
+        gj[j] = gate[t * k + j];
+      }
   }
+  // every row load is issued before the first product; the sum keeps the slot order
+  float4 v[kMaxTopK];
+#pragma unroll
+  for (int j = 0; j < kMaxTopK; ++j)
+    if (j < k) v[j] = *reinterpret_cast<const float4*>(yslot + (size_t)r[j] * d + c);
+  float4 vs = make_float4(0.f, 0.f, 0.f, 0.f);
+  if (has_shared) vs = *reinterpret_cast<const float4*>(yshared + (size_t)t * d + c);
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int j = 0; j < kMaxTopK; ++j)
+    if (j < k) {
+      acc.x = fmaf(gj[j], v[j].x, acc.x);
+      acc.y = fmaf(gj[j], v[j].y, acc.y);
+      acc.z = fmaf(gj[j], v[j].z, acc.z);
+      acc.w = fmaf(gj[j], v[j].w, acc.w);
+    }
   if (has_shared) {
-    const float4 v = *reinterpret_cast<const float4*>(yshared + (size_t)t * d + c);
-    acc.x += v.x; acc.y += v.y; acc.z += v.z; acc.w += v.w;
+    acc.x += vs.x; acc.y += vs.y; acc.z += vs.z; acc.w += vs.w;
   }
   __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
   __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
@@ -771,12 +797,12 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
 }
 
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero, int n_zero,
-                           uint32_t* zero2, int n_zero2) {
+                           uint32_t* zero2, int n_zero2, bool meta_early) {
   dim3 cgrid((a.d / 4 + 255) / 256, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
   cudaError_t e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared,
                             a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero,
-                            zero2, n_zero2);
+                            zero2, n_zero2, meta_early ? 1 : 0);
   prof_end(DMOE_KERNEL_COMBINE, s);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();
