@@ -248,6 +248,23 @@ class Arm:
         main.wait_stream(self.s_out)
 
 
+def max_over_ranks(secs: float, dist, world: int, device: str = "cuda") -> float:
+    """The timed region's length for the whole job: the slowest rank's seconds (every rank
+    gets the same value). One scalar all-reduce, outside any timed region."""
+    if dist is None or world <= 1:
+        return secs
+    import torch
+    t = torch.tensor([secs], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_step: int, steps: int, world: int, secs_max: float) -> float:
+    """Whole-job tokens/s of N independent replicas (weak scaling): the tokens all ranks
+    processed over the slowest rank's time."""
+    return tokens_per_step * steps * world / secs_max
+
+
 def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
     """W warm-up steps, then exactly K steps from graph replays; returns (seconds over the
     timed region, max over ranks; mean gate/up launch seconds or None)."""
@@ -303,11 +320,7 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
             collect(r % NG)
     if dist is not None:
         dist.barrier()
-    secs = start.elapsed_time(end) / 1e3
-    if dist is not None and world > 1:
-        t = torch.tensor([secs], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        secs = float(t.item())
+    secs = max_over_ranks(start.elapsed_time(end) / 1e3, dist, world)
     arm.check()
     kern = (float(np.mean(kernel_ms)) / 1e3) if kernel_ms else None
     return secs, kern, clocks
@@ -841,7 +854,7 @@ def main():
     U_mean = float(np.mean(U))
     T = shape.T
     tokens_total = T * args.steps * world
-    value = tokens_total / secs
+    value = job_throughput(T, args.steps, world, secs)
     ms_per_step = secs / args.steps * 1e3
 
     # end to end: x from pinned host memory in, y back to pinned host memory, every step
@@ -863,7 +876,8 @@ def main():
         _, k2, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world)
         u2 = float(np.mean(a2.unique_counts()))
         us = s2 / args.side_steps * 1e6
-        side[name] = {"us_per_forward": us, "tokens_per_s": T * args.side_steps * world / s2,
+        side[name] = {"us_per_forward": us,
+                      "tokens_per_s": job_throughput(T, args.side_steps, world, s2),
                       "unique_experts_mean": u2,
                       "hbm_roofline_frac": layer_bytes(sh, u2) / (us * 1e-6) / 1e9 / hbm,
                       "experts_us": k2 * 1e6 if k2 else None}
@@ -900,7 +914,8 @@ def main():
                      "launch_us": kern_s * 1e6 if kern_s else None,
                      "peak_source": f"{peak_src} hbm_gbs"},
         "side_by_side": side,
-        "e2e": None if secs_e2e is None else {"value": tokens_total / secs_e2e, "unit": UNIT,
+        "e2e": None if secs_e2e is None else {"value": job_throughput(T, args.steps, world, secs_e2e),
+                "unit": UNIT,
                 "h2d_bytes_per_step": T * shape.d_model * 2,
                 "d2h_bytes_per_step": T * shape.d_model * 2},
         "gpu_launches": args.steps * dm.dmoe_layer_forward_launches(arm.layers[0].desc),
