@@ -527,7 +527,8 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
             layers.append(MoELayer.from_shape(shape, w))
             xs.append(layer_inputs(shape, seed=args.seed + s, device="cuda",
                                    with_weights=False)["x"])
-        sec = graph_time(torch, [lambda L=L, x=x: L.forward(x) for L, x in zip(layers, xs)])
+        sec = graph_time(torch, [lambda L=L, x=x: L.forward(x) for L, x in zip(layers, xs)],
+                         args.suite_time)
         for L in layers:
             st, info = dm.dmoe_get_device_error(L.ws)
             if st != 0:
@@ -538,6 +539,14 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
               "bias_scale": shape.bias_scale, "T": shape.T, **stats(shape, sec, U)})
         return sec, U
 
+    if args.suite_point:
+        # one point only: "<block size>x<batch>:<block_p<p> | token>", e.g. 32x64:block_p0
+        size, routing = args.suite_point.split(":")
+        bsz, nb = (int(v) for v in size.split("x"))
+        mode, p = ((ROUTE_TOKEN, 0.0) if routing == "token"
+                   else (ROUTE_BLOCK, float(routing.replace("block_p", ""))))
+        point("point", LAYER.with_(block_size=bsz, n_blocks=nb, mode=mode, top_p=p))
+        return
     for mode, p in ((ROUTE_BLOCK, 0.0), (ROUTE_BLOCK, 0.6), (ROUTE_TOKEN, 0.0)):
         point("8x32", LAYER_B8.with_(mode=mode, top_p=p))
     # the coreset threshold as a performance axis: p over the paper's sweep values at block
@@ -804,6 +813,11 @@ def main():
     ap.add_argument("--suite", action="store_true",
                     help="measure the other workloads instead of the headline (one JSON line "
                          "per point; one GPU)")
+    ap.add_argument("--suite-point", default=None,
+                    help="with --suite: measure one point only, '<block size>x<batch>:<routing>' "
+                         "with routing block_p<p> or token (e.g. 32x64:block_p0)")
+    ap.add_argument("--suite-time", type=float, default=0.25,
+                    help="with --suite: seconds of graph replays per point")
     ap.add_argument("--decode-sim", action="store_true",
                     help="the synthetic block-diffusion decoding loop around the MoE stack "
                          "(MoE share of a step, CV of U across steps; one GPU)")
