@@ -30,7 +30,10 @@ STATUS_NAMES = {0: "DMOE_OK", 1: "DMOE_ERR_INVALID_ARG", 2: "DMOE_ERR_UNSUPPORTE
                 3: "DMOE_ERR_WORKSPACE", 4: "DMOE_ERR_CUDA", 5: "DMOE_ERR_DEVICE",
                 6: "DMOE_ERR_TIMEOUT"}
 
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libdmoe.so")
+# DMOE_LIB selects another build of the same library (the debug timeline tool sets it to
+# its -DDMOE_TRACE build); by default the in-tree libdmoe.so
+LIB_PATH = os.environ.get("DMOE_LIB") or os.path.join(
+    os.path.dirname(os.path.abspath(__file__)), "libdmoe.so")
 
 
 class LayerDesc(ctypes.Structure):

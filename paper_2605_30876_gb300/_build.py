@@ -40,17 +40,20 @@ def _stale(target: str, deps) -> bool:
     return any(os.path.getmtime(d) > t for d in deps)
 
 
-def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
-    """Compile (when sources changed) and return the path of libdmoe.so."""
+def build(verbose: bool = False, force: bool = False, extra_flags=(), build_dir: str = BUILD,
+          lib_path: str = LIB) -> str:
+    """Compile (when sources changed) and return the path of the library (libdmoe.so by
+    default; a debug variant with other flags goes to its own build_dir and lib_path)."""
     nvcc = _nvcc()
-    os.makedirs(BUILD, exist_ok=True)
+    BUILD_, LIB_ = build_dir, lib_path
+    os.makedirs(BUILD_, exist_ok=True)
     headers = [os.path.join(CSRC, f) for f in os.listdir(CSRC) if f.endswith((".cuh", ".h"))]
     headers += [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE)]
     objs = []
     jobs = []
     for src in SOURCES:
         s = os.path.join(CSRC, src)
-        o = os.path.join(BUILD, src.replace(".cu", ".o"))
+        o = os.path.join(BUILD_, src.replace(".cu", ".o"))
         objs.append(o)
         if force or _stale(o, [s] + headers):
             cmd = [nvcc, *ARCH, *FLAGS, *extra_flags, "-c", s, "-o", o]
@@ -68,9 +71,9 @@ def build(verbose: bool = False, force: bool = False, extra_flags=()) -> str:
     if jobs:
         with cf.ThreadPoolExecutor(max_workers=min(len(jobs), os.cpu_count() or 4)) as ex:
             list(ex.map(run, jobs))
-    if force or jobs or _stale(LIB, objs):
-        run([nvcc, *ARCH, "-shared", "-o", LIB, *objs, "-cudart", "static"])
-    return LIB
+    if force or jobs or _stale(LIB_, objs):
+        run([nvcc, *ARCH, "-shared", "-o", LIB_, *objs, "-cudart", "static"])
+    return LIB_
 
 
 if __name__ == "__main__":
