@@ -189,14 +189,21 @@ dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end
  * The caller still passes every input and output, exactly as for dmoe_router, and the
  * results are the same.
  *  - The call allocates nothing and frees nothing (no cudaMalloc/cudaFree, no allocating
- *    library routine). Shapes whose router scratch exceeds 4 MiB (partial logits + 2 x
- *    T*E fp32 + 512 bytes; e.g. T = 4096 tokens with 256 experts) return
+ *    library routine). The scratch it needs is the leading part of the workspace layout,
+ *    each region rounded up to 256 bytes: the fault record and the stage counters (1.3 KB),
+ *    the partial logits (T*E fp32, times the router's split of d when d is not a multiple
+ *    of 256), the scores and the masked scores (T*E fp32 each) and the top-k candidates
+ *    (T * ceil(E/32) * k_mask * 8 bytes, k_mask = block_top_k or k). With E = 256 and
+ *    k = 8 that is about 3.6 KB per token: at most 1169 tokens. Larger shapes return
  *    DMOE_ERR_UNSUPPORTED, with the sizes in dmoe_last_error_message().
  *  - The first call on each device looks up the array's device address (with that device
  *    current) and caches it; make that first call before any CUDA-graph stream capture.
- *  - All calls share the one array and it keeps the previous call's contents: each call
- *    clears the fault record it uses, its completion counter returns to zero at the end of
- *    every call, and everything else it reads it has written first.
+ *    A device reset (cudaDeviceReset) reloads the library's device code at a new address:
+ *    do not call this entry point on that device again in the same process.
+ *  - All calls share the one array and it keeps the previous call's contents: the stage
+ *    counters return to zero at the end of every call, and everything else a call reads it
+ *    has written first. A fault a kernel records (a bounded wait that ran out) stays in the
+ *    array until dmoe_router_no_alloc_device_error reads and clears it.
  *    Calls whose executions overlap on the GPU (two streams, or two host threads) race on
  *    the array and give wrong results: serialise them.
  * Arguments, layouts and errors otherwise as for dmoe_router. */
@@ -204,6 +211,18 @@ dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const void* x, con
                                  const float* bias, int32_t* topk_idx, float* topk_gate,
                                  int32_t* coreset, int32_t* coreset_size, float* probs,
                                  void* stream);
+
+/* The fault record of dmoe_router_no_alloc on the current device: synchronises `stream`,
+ * then reads and clears it. Returns and fills `info` (host, 4 int32, or NULL) as
+ * dmoe_get_device_error does for a workspace. */
+dmoe_status dmoe_router_no_alloc_device_error(void* stream, int32_t* info);
+
+/* Device address and size (host outputs) of the static scratch array of
+ * dmoe_router_no_alloc on the current device, looked up as that call does. For inspection
+ * and tests: the array starts with the same fault record as a workspace, so any call given
+ * it as a workspace shares it with dmoe_router_no_alloc (and the serialisation rule above
+ * applies). */
+dmoe_status dmoe_no_alloc_scratch(void** device_ptr, size_t* bytes);
 
 /* Synchronises `stream`, then reads and clears the fault code the kernels recorded in
  * `workspace`. Returns DMOE_OK if none, DMOE_ERR_TIMEOUT for a bounded wait that ran out,

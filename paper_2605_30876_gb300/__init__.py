@@ -30,8 +30,8 @@ STATUS_NAMES = {0: "DMOE_OK", 1: "DMOE_ERR_INVALID_ARG", 2: "DMOE_ERR_UNSUPPORTE
                 3: "DMOE_ERR_WORKSPACE", 4: "DMOE_ERR_CUDA", 5: "DMOE_ERR_DEVICE",
                 6: "DMOE_ERR_TIMEOUT"}
 
-# DMOE_LIB selects another build of the same library (the debug timeline tool sets it to
-# its -DDMOE_TRACE build); by default the in-tree libdmoe.so
+# DMOE_LIB selects another build of the same library (for example one compiled with other
+# flags); by default the in-tree libdmoe.so
 LIB_PATH = os.environ.get("DMOE_LIB") or os.path.join(
     os.path.dirname(os.path.abspath(__file__)), "libdmoe.so")
 
@@ -94,6 +94,12 @@ def _load() -> ctypes.CDLL:
     lib.dmoe_layer_forward_launches.restype = ctypes.c_int32
     lib.dmoe_set_profile_events.argtypes = [ctypes.c_int32, P, P]
     lib.dmoe_set_profile_events.restype = st
+    lib.dmoe_router_no_alloc.argtypes = [D, P, P, P, P, P, P, P, P, P]
+    lib.dmoe_router_no_alloc.restype = st
+    lib.dmoe_router_no_alloc_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_int32)]
+    lib.dmoe_router_no_alloc_device_error.restype = st
+    lib.dmoe_no_alloc_scratch.argtypes = [ctypes.POINTER(P), ctypes.POINTER(ctypes.c_size_t)]
+    lib.dmoe_no_alloc_scratch.restype = st
     return lib
 
 
@@ -205,6 +211,33 @@ def dmoe_get_device_error(workspace, stream=None) -> Tuple[int, Tuple[int, int, 
     st = _lib.dmoe_get_device_error(_ptr(workspace, torch.uint8, "workspace"), _stream(stream),
                                     info)
     return st, (info[0], info[1], info[2])
+
+
+def dmoe_router_no_alloc(desc, x, w_r, bias, topk_idx, topk_gate, coreset=None,
+                         coreset_size=None, probs=None, stream=None) -> None:
+    """dmoe_router without a workspace (the library's static scratch array)."""
+    _check(_lib.dmoe_router_no_alloc(
+        ctypes.byref(desc), _ptr(x, torch.bfloat16, "x"), _ptr(w_r, torch.float32, "w_r"),
+        _ptr(bias, torch.float32, "bias"), _ptr(topk_idx, torch.int32, "topk_idx"),
+        _ptr(topk_gate, torch.float32, "topk_gate"), _ptr(coreset, torch.int32, "coreset"),
+        _ptr(coreset_size, torch.int32, "coreset_size"), _ptr(probs, torch.float32, "probs"),
+        _stream(stream)), "dmoe_router_no_alloc")
+
+
+def dmoe_router_no_alloc_device_error(stream=None) -> Tuple[int, Tuple[int, int, int]]:
+    """Synchronises the stream; returns (status, (code, where, value)) of the static scratch
+    array's fault record and clears it."""
+    info = (ctypes.c_int32 * 4)()
+    st = _lib.dmoe_router_no_alloc_device_error(_stream(stream), info)
+    return st, (info[0], info[1], info[2])
+
+
+def dmoe_no_alloc_scratch() -> Tuple[int, int]:
+    """(device address, bytes) of the static scratch array on the current device."""
+    ptr, n = ctypes.c_void_p(0), ctypes.c_size_t(0)
+    _check(_lib.dmoe_no_alloc_scratch(ctypes.byref(ptr), ctypes.byref(n)),
+           "dmoe_no_alloc_scratch")
+    return int(ptr.value or 0), n.value
 
 
 KERNELS = {"router": 0, "dispatch": 1, "gather": 2, "experts": 3, "combine": 4}

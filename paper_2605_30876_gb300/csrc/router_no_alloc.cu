@@ -8,6 +8,9 @@
 // for the life of the process. Host code cannot pass the array's name to a kernel (on the
 // host it only names a stand-in, not a device address), so the device address is looked
 // up once per device with cudaGetSymbolAddress, with that device current, and cached.
+// The array's first bytes are the fault record of the router kernels (the first region of
+// the workspace layout, at offset 0 for every shape); dmoe_router_no_alloc_device_error
+// reads and clears it.
 #include <mutex>
 #include <stdio.h>
 
@@ -84,12 +87,9 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
     return DMOE_ERR_CUDA;
   }
   cudaStream_t s = static_cast<cudaStream_t>(stream);
-  // the array keeps the previous call's contents: start from a clear fault record
-  e = cudaMemsetAsync(static_cast<uint8_t*>(scratch) + plan.err, 0, sizeof(DevErrRecord), s);
-  if (e != cudaSuccess) {
-    set_last_error(e);
-    return DMOE_ERR_CUDA;
-  }
+  // The fault record is not cleared here: as in a caller workspace, a recorded fault stays
+  // until dmoe_router_no_alloc_device_error reads it (the array starts zero-filled when the
+  // library is loaded).
   uint8_t* base = static_cast<uint8_t*>(scratch);
   RouterArgs a{};
   a.x = static_cast<const __nv_bfloat16*>(x);
@@ -120,5 +120,30 @@ extern "C" dmoe_status dmoe_router_no_alloc(const dmoe_layer_desc* desc, const v
     set_last_error(e);
     return DMOE_ERR_CUDA;
   }
+  return DMOE_OK;
+}
+
+extern "C" dmoe_status dmoe_router_no_alloc_device_error(void* stream, int32_t* info) {
+  void* scratch = nullptr;
+  cudaError_t e = scratch_address(&scratch);
+  if (e != cudaSuccess) {
+    set_last_error(e);
+    return DMOE_ERR_CUDA;
+  }
+  // the fault record heads the workspace layout: the same reader as for a caller workspace
+  static_assert(sizeof(DevErrRecord) <= 256, "the fault record is the first region");
+  return dmoe_get_device_error(scratch, stream, info);
+}
+
+extern "C" dmoe_status dmoe_no_alloc_scratch(void** device_ptr, size_t* bytes) {
+  if (device_ptr == nullptr || bytes == nullptr) return DMOE_ERR_INVALID_ARG;
+  void* scratch = nullptr;
+  cudaError_t e = scratch_address(&scratch);
+  if (e != cudaSuccess) {
+    set_last_error(e);
+    return DMOE_ERR_CUDA;
+  }
+  *device_ptr = scratch;
+  *bytes = kRouterStaticScratchBytes;
   return DMOE_OK;
 }

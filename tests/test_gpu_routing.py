@@ -59,6 +59,9 @@ def test_routing_matches_oracle(name):
     g = P.gpu_router(shape, dev)
     orc = P.oracle_routing(shape, host)
     stats = P.check_routing(shape, g, orc)
+    # tokens at an oracle near tie (margin < 1e-5) are checked for validity only; report
+    # how many there were
+    print(f"{name}: {stats}")
     assert stats["exact"] >= 0.9 * stats["tokens"], stats
     if shape.mode == ROUTE_BLOCK and shape.top_p == 0.0:
         for b in range(shape.n_blocks):

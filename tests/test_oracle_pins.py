@@ -230,6 +230,59 @@ def test_topk_tie_goes_to_lower_index():
     assert O.topk_desc(f32([0.3, 0.3, 0.3]), 2).tolist() == [0, 1]
 
 
+
+def test_topk_margins_hand_values():
+    """TopK margins (reading R11): v = [.5, .3, .29, .1], k = 2 -> the set decision is .30
+    vs .29 (margin .01), the slot order .5 vs .3 (margin .2). A margin that is always 0
+    would turn every token ambiguous; one taken from the wrong end would hide near ties."""
+    sm, om = O.topk_margins(np.array([0.5, 0.3, 0.29, 0.1]), 2)
+    assert sm == pytest.approx(0.01, abs=1e-15)
+    assert om == pytest.approx(0.2, abs=1e-15)
+    # the same values permuted: margins depend on values, not positions
+    sm2, om2 = O.topk_margins(np.array([0.1, 0.29, 0.5, 0.3]), 2)
+    assert (sm2, om2) == (sm, om)
+    # k = 3: set .29 vs .1 = .19, order min(.5 - .3, .3 - .29) = .01
+    sm3, om3 = O.topk_margins(np.array([0.5, 0.3, 0.29, 0.1]), 3)
+    assert sm3 == pytest.approx(0.19, abs=1e-15) and om3 == pytest.approx(0.01, abs=1e-15)
+    # k = 1: no order decision; no (k+1)-th finite candidate -> infinite set margin
+    assert O.topk_margins(np.array([0.7, 0.2]), 1) == (pytest.approx(0.5), float("inf"))
+    assert O.topk_margins(np.array([0.7, -np.inf, -np.inf]), 1)[0] == float("inf")
+    # inside a coreset (MaskOutside fills -inf): only the members compete
+    sC = O.mask_outside(f32([0.5, 0.3, 0.29, 0.1]), np.array([0, 3, 1]))
+    sm4, om4 = O.topk_margins(sC, 2)
+    assert sm4 == pytest.approx(float(f32(0.3)) - float(f32(0.1)), abs=1e-12)
+    assert om4 == pytest.approx(float(f32(0.5)) - float(f32(0.3)), abs=1e-12)
+
+
+def test_topk_margins_order_margin_alone_can_be_near():
+    """A token whose set is clear but whose first two slots nearly tie: the order margin is
+    below 1e-5 while the set margin is large, so the parity check may accept either slot
+    order but must still demand the same set."""
+    v = np.array([0.4, 0.4 - 4e-6, 0.1, 0.05])
+    sm, om = O.topk_margins(v, 2)
+    assert sm == pytest.approx(0.4 - 4e-6 - 0.1, abs=1e-15)
+    assert om == pytest.approx(4e-6, abs=1e-15)
+    assert om < O.NEAR_TIE <= sm
+
+
+def test_gates_for_hand_values():
+    """R8 gates of a given selection, by hand: token 0 routed to (2, 0) with s = [.5, .2,
+    .3] -> (.3/.8, .5/.8) = (.375, .625); token 1 routed to (1, 2) with s = [.1, .6, .3] ->
+    (.6/.9, .3/.9). A transposed token index or a sum over the wrong row fails here."""
+    s = f32([[0.5, 0.2, 0.3], [0.1, 0.6, 0.3]])
+    idx = np.array([[2, 0], [1, 2]], np.int32)
+    g = O.gates_for(s, idx)
+    s64 = s.astype(np.float64)
+    exp0 = [s64[0, 2] / (s64[0, 2] + s64[0, 0]), s64[0, 0] / (s64[0, 2] + s64[0, 0])]
+    exp1 = [s64[1, 1] / (s64[1, 1] + s64[1, 2]), s64[1, 2] / (s64[1, 1] + s64[1, 2])]
+    np.testing.assert_allclose(g, [exp0, exp1], rtol=0, atol=1e-15)
+    np.testing.assert_allclose(g, [[0.375, 0.625], [2 / 3, 1 / 3]], rtol=0, atol=1e-7)
+    assert g.dtype == np.float64 and np.allclose(g.sum(axis=1), 1.0, atol=1e-15)
+    # the hand case of Algorithm 1 above: p = 0.6 gates through gates_for
+    r = O.route_block(S_HAND, 2, 2, 0.6)
+    np.testing.assert_allclose(O.gates_for(S_HAND, r.idx), [[0.625, 0.375], [0.8, 0.2]],
+                               rtol=0, atol=1e-7)
+
 @pytest.mark.parametrize("E", [5, 8, 10])
 def test_top_p_brute_force(E):
     """The p rule takes the fewest experts whose normalised mass reaches p (checked against

@@ -5,8 +5,10 @@ static device array of the library.
 
 Called through the C ABI twice in a row on the same inputs, it must give what dmoe_router
 (with a caller-allocated workspace) gives, within the parity tolerances of the other
-tests. This file is collected last so that a stop-at-first-failure run has run every other
-test before it; it also passes on its own in a fresh process.
+tests, and the oracle's routing. Its fault record, which lives in the static array, must be
+readable through dmoe_router_no_alloc_device_error. This file is collected last so that a
+stop-at-first-failure run has run every other test before it; it also passes on its own in
+a fresh process.
 """
 import ctypes
 
@@ -14,20 +16,18 @@ import numpy as np
 import pytest
 import torch
 
-from dmoe_synth import LAYER, ROUTE_TOKEN, TINY, layer_inputs
+from dmoe_synth import LAYER, LAYER_B8, ROUTE_TOKEN, TINY, layer_inputs, to_numpy
 from tests import parity as P
 
 pytestmark = pytest.mark.gpu
 
+# scratch of the router at E = 256, k = 8 (the header's formula): 1169 tokens fit in 4 MiB
+MAX_T_E256_K8 = 1169
+
 
 def _lib():
     m = P.dm()
-    lib = m._lib
-    fn = lib.dmoe_router_no_alloc
-    Vp = ctypes.c_void_p
-    fn.argtypes = [ctypes.POINTER(m.LayerDesc), Vp, Vp, Vp, Vp, Vp, Vp, Vp, Vp, Vp]
-    fn.restype = ctypes.c_int
-    return m, fn
+    return m, m._lib.dmoe_router_no_alloc
 
 
 def _outputs(shape):
@@ -49,18 +49,33 @@ def _no_alloc_call(m, fn, shape, dev, out, with_probs=True):
     return st
 
 
-@pytest.mark.parametrize("shape", [LAYER.with_(top_p=0.6), LAYER,
-                                   TINY.with_(mode=ROUTE_TOKEN)],
-                         ids=["layer_block_p06", "layer_block_p0", "tiny_token"])
-def test_no_alloc_router_matches_workspace_router(shape):
+SHAPES = {
+    "layer_block_p06": LAYER.with_(top_p=0.6),
+    "layer_block_p0": LAYER,
+    "tiny_token": TINY.with_(mode=ROUTE_TOKEN),
+    # more than 64 tokens: the tiled logits launch, the softmax launch, the block launch
+    "layer_b8_block_p0": LAYER_B8,
+    "layer_b8_token": LAYER_B8.with_(mode=ROUTE_TOKEN),
+    # d not a multiple of 256: the FFMA logits kernel split over d
+    "d384_block_p06": LAYER.with_(d_model=384, top_p=0.6),
+    # the largest token count whose scratch fits the 4 MiB array at E = 256, k = 8
+    "max_tokens_1169": LAYER.with_(block_size=167, n_blocks=7, top_p=0.6),
+}
+
+
+@pytest.mark.parametrize("name", list(SHAPES))
+def test_no_alloc_router_matches_workspace_router(name):
+    shape = SHAPES[name]
     m, fn = _lib()
     dev = layer_inputs(shape, seed=21, device="cuda", with_weights=False)
     ref = P.gpu_router(shape, dev)               # dmoe_router with a torch workspace
+    orc = P.oracle_routing(shape, to_numpy(dev))
     for call in range(2):                        # two calls in a row share the array
         out = _outputs(shape)
         st = _no_alloc_call(m, fn, shape, dev, out, with_probs=(call == 0))
         assert st == 0, m.dmoe_status_string(st)
-        torch.cuda.synchronize()
+        st, info = m.dmoe_router_no_alloc_device_error()
+        assert st == 0 and info == (0, 0, 0), (st, info)
         got = {k: v.cpu().numpy() for k, v in out.items()}
         assert np.array_equal(got["idx"], ref["idx"])
         np.testing.assert_allclose(got["gate"], ref["gate"], rtol=0, atol=P.GATE_ATOL)
@@ -68,15 +83,55 @@ def test_no_alloc_router_matches_workspace_router(shape):
         assert np.array_equal(got["coreset_size"], ref["coreset_size"])
         if call == 0:
             np.testing.assert_allclose(got["probs"], ref["probs"], rtol=1e-6, atol=1e-8)
+            # and the oracle's routing, under the same rules as dmoe_router's parity test
+            stats = P.check_routing(shape, got, orc)
+            print(f"{name}: {stats}")
 
 
-def test_no_alloc_router_rejects_oversized_shapes():
+def test_no_alloc_router_size_limit():
+    """One token past the documented limit is refused before anything is launched."""
     m, fn = _lib()
-    shape = LAYER.with_(block_size=64, n_blocks=64)     # 4096 tokens: 12 MiB of scratch
-    desc = P.desc_of(shape)
     dummy = torch.zeros(16, dtype=torch.int32, device="cuda")
     p = dummy.data_ptr()
-    st = fn(ctypes.byref(desc), p, p, None, p, p, None, None, None,
-            torch.cuda.current_stream().cuda_stream)
-    assert st == 2                                      # DMOE_ERR_UNSUPPORTED
-    assert b"static buffer" in m._lib.dmoe_last_error_message()
+    for shape in (LAYER.with_(block_size=117, n_blocks=10, top_p=0.6),   # 1170 tokens
+                  LAYER.with_(block_size=64, n_blocks=64)):              # 4096 tokens
+        desc = P.desc_of(shape)
+        st = fn(ctypes.byref(desc), p, p, None, p, p, None, None, None,
+                torch.cuda.current_stream().cuda_stream)
+        assert st == 2, shape                            # DMOE_ERR_UNSUPPORTED
+        assert b"static buffer" in m._lib.dmoe_last_error_message()
+    assert SHAPES["max_tokens_1169"].T == MAX_T_E256_K8
+
+
+def test_no_alloc_fault_record_is_readable():
+    """A fault recorded on the device into the static array's record is reported (and
+    cleared) by dmoe_router_no_alloc_device_error. The fault is a real device-side check:
+    the dispatch kernel, given the static array as its workspace, meets an expert id out of
+    range. Afterwards the record is clear and the router runs normally."""
+    m, fn = _lib()
+    ptr, nbytes = m.dmoe_no_alloc_scratch()
+    assert ptr != 0 and ptr % 256 == 0 and nbytes == 4 << 20
+    shape = TINY
+    desc = P.desc_of(shape)
+    assert m.dmoe_workspace_size(desc) <= nbytes
+    T, k, E = shape.T, shape.top_k, shape.n_experts
+    idx = torch.arange(T * k, dtype=torch.int32, device="cuda").reshape(T, k) % E
+    idx[3, 1] = E                                    # out of range: recorded, not trapped
+    outs = [torch.zeros(n, dtype=torch.int32, device="cuda") for n in (1, E, E + 1, T * k, T * k)]
+    st = m._lib.dmoe_dispatch(ctypes.byref(desc), idx.data_ptr(), *[o.data_ptr() for o in outs],
+                              ptr, nbytes, torch.cuda.current_stream().cuda_stream)
+    assert st == 0, m.dmoe_status_string(st)
+    st, info = m.dmoe_router_no_alloc_device_error()
+    assert st == 5, (st, info)                       # DMOE_ERR_DEVICE
+    assert info[0] == 2 and info[1] == 3 and info[2] == 3 * k + 1   # expert id, dispatch, slot
+    st, info = m.dmoe_router_no_alloc_device_error()
+    assert st == 0 and info == (0, 0, 0), (st, info)
+    # the router still works on the same array, twice
+    dev = layer_inputs(shape, seed=4, device="cuda", with_weights=False)
+    ref = P.gpu_router(shape, dev)
+    for _ in range(2):
+        out = _outputs(shape)
+        assert _no_alloc_call(m, fn, shape, dev, out) == 0
+        st, info = m.dmoe_router_no_alloc_device_error()
+        assert st == 0, (st, info)
+        assert np.array_equal(out["idx"].cpu().numpy(), ref["idx"])
