@@ -612,33 +612,36 @@ def run_suite(args, torch, dm, MoELayer, hbm: float, bf16_peak: float):
 
 
 # ----------------------------------------------------------------------------- decode sim
-def run_decode_sim(args, torch, dm, MoELayer):
-    """A synthetic block-diffusion decoding loop around the MoE stack, one JSON line per
-    routing: how much of a denoising step the MoE layers take, and how the unique-expert
-    count U varies across steps (its coefficient of variation, the statistic of the paper's
-    Table 1).
+def decode_sim(torch, dm, MoELayer, shape_base, n_layers, n_blocks, vocab, ctx, head_dim,
+               seed, modes, on_step=None, conf_target=0.95):
+    """A synthetic block-diffusion decoding loop around the MoE stack; returns one record per
+    routing mode: step latencies, the MoE and attention shares of a step, and the
+    unique-expert count U of every layer at every step (the statistic of the paper's Table 1
+    is U's coefficient of variation across steps).
 
     Model stand-in (random weights; only the costs and the data flow are real): one
-    sequence, a block of 32 positions decoded at a time; per step every position of the
-    block passes 20 layers, each an attention stand-in (RMS norm, q/k/v/o projections,
-    16 heads of 128 over a 1024-token cached context plus the block, by torch SDPA) and the
-    MoE layer of the benchmark shape (this library; RMS-normalised input, residual add),
-    then a tied embedding / LM head of a 128k vocabulary; the block's positions carry
+    sequence, a block of shape_base.block_size positions decoded at a time; per step every
+    position of the block passes n_layers layers, each an attention stand-in (RMS norm,
+    q/k/v/o projections, d / head_dim heads over a ctx-token cached context plus the block,
+    by torch SDPA) and an MoE layer of shape_base's shape (this library; RMS-normalised input,
+    residual add), then a tied embedding / LM head of `vocab` rows; the block's positions carry
     position embeddings. The stand-ins are plain torch, not tuned: their share is an upper
-    bound of what a tuned attention would take. Unmasking: every masked position
-    whose top softmax probability reaches 0.95 takes its argmax token, at least the most
-    confident one per step; the logit scale is fixed once so that about two of the 32
-    masked positions of the first step pass. A block ends when all its positions are
-    unmasked; the next block starts fully masked over the same context.
+    bound of what a tuned attention would take. Unmasking: every masked position whose top
+    softmax probability reaches conf_target takes its argmax token, at least the most
+    confident one per step; the logit scale is fixed once so that about two of the masked
+    positions of the first step pass. A block ends when all its positions are unmasked; the
+    next block starts fully masked over the same context.
 
     Each step is one CUDA graph replay (its device time is the step latency); the MoE and
-    attention shares come from graphs of the 20 MoE layers alone and the 20 attention
-    stand-ins alone, replayed on the same step's inputs."""
-    from dmoe_synth import LAYER, ROUTE_BLOCK, ROUTE_TOKEN, STACK20_LAYERS, layer_inputs
-    NL, B, V, H, HD, CTX = STACK20_LAYERS, 32, 128000, 16, 128, 1024
-    d = LAYER.d_model
+    attention shares come from graphs of the MoE layers alone and the attention stand-ins
+    alone, replayed on the same step's inputs. `on_step(name, step, layers)` is called after
+    every step's replay (the layers' routing outputs then hold that step's routing)."""
+    from dmoe_synth import layer_inputs
+    NL, B, V, CTX, HD = n_layers, shape_base.block_size, vocab, ctx, head_dim
+    d = shape_base.d_model
+    H = d // HD
     g = torch.Generator(device="cuda")
-    g.manual_seed(args.seed + 77)
+    g.manual_seed(seed + 77)
 
     def rnd(*shape, std=1.0):
         return (torch.randn(*shape, generator=g, device="cuda") * std).to(torch.bfloat16)
@@ -650,7 +653,7 @@ def run_decode_sim(args, torch, dm, MoELayer):
     # followed by the block's own rows (written in place every step)
     attn_w = [(rnd(d, 3 * d, std=d ** -0.5), rnd(d, d, std=d ** -0.5)) for _ in range(NL)]
     kv = [(rnd(1, H, CTX + B, HD), rnd(1, H, CTX + B, HD)) for _ in range(NL)]
-    moe_w = [layer_inputs(LAYER, seed=args.seed + 2000 + l, device="cuda", layer=l)
+    moe_w = [layer_inputs(shape_base, seed=seed + 2000 + l, device="cuda", layer=l)
              for l in range(NL)]
     x_in = torch.empty(B, d, dtype=torch.bfloat16, device="cuda")
     xs = [torch.empty(B, d, dtype=torch.bfloat16, device="cuda") for _ in range(2 * NL + 1)]
@@ -703,9 +706,7 @@ def run_decode_sim(args, torch, dm, MoELayer):
             best = t if best is None else min(best, t)
         return best
 
-    modes = [("block_p0", LAYER), ("block_p0.6", LAYER.with_(top_p=0.6)),
-             ("token", LAYER.with_(mode=ROUTE_TOKEN))]
-    n_blocks = args.sim_blocks
+    records = []
     for name, shape in modes:
         layers = [MoELayer.from_shape(shape, moe_w[l]) for l in range(NL)]
 
@@ -735,7 +736,7 @@ def run_decode_sim(args, torch, dm, MoELayer):
 
         embed()
         g_step, g_moe, g_attn = capture(step_fn), capture(moe_fn), capture(attn_fn)
-        # logit scale: about two of the first step's 32 masked positions reach 0.95
+        # logit scale: about two of the first step's masked positions reach conf_target
         g_step.replay()
         torch.cuda.synchronize()
         lo, hi = 1.0, 1e4
@@ -743,7 +744,7 @@ def run_decode_sim(args, torch, dm, MoELayer):
             mid = (lo * hi) ** 0.5
             scale.fill_(mid)
             head(xs[2 * NL - 1])
-            n_pass = int((conf >= 0.95).sum().item())
+            n_pass = int((conf >= conf_target).sum().item())
             lo, hi = (mid, hi) if n_pass < 2 else (lo, mid)
         scale.fill_(hi)
         t_step, t_moe, t_attn, U, per_step = [], [], [], [], []
@@ -752,13 +753,15 @@ def run_decode_sim(args, torch, dm, MoELayer):
             embed()
             t_step.append(timed(g_step, 1))
             U.append([int(L.n_unique.item()) for L in layers])
+            if on_step is not None:
+                on_step(name, len(t_step) - 1, layers)
             if len(t_step) % 4 == 1:      # component graphs on this step's inputs
                 t_moe.append(timed(g_moe))
                 t_attn.append(timed(g_attn))
                 g_step.replay()           # the state the unmasking below reads
                 torch.cuda.synchronize()
             c = torch.where(masked, conf, torch.full_like(conf, -1.0))
-            take = masked & (c >= 0.95)
+            take = masked & (c >= conf_target)
             if not bool(take.any()):
                 take = torch.zeros_like(masked)
                 take[int(c.argmax().item())] = True
@@ -773,25 +776,50 @@ def run_decode_sim(args, torch, dm, MoELayer):
             if st_ != 0:
                 raise RuntimeError(f"device fault {info}")
         Ua = np.array(U, dtype=np.float64)
-        mid = NL // 2
-        step_us = float(np.mean(t_step)) * 1e6
-        moe_us, attn_us = float(np.mean(t_moe)) * 1e6, float(np.mean(t_attn)) * 1e6
+        records.append(dict(routing=name, U=Ua, t_step=np.array(t_step), t_moe=np.array(t_moe),
+                            t_attn=np.array(t_attn), tokens_per_step=np.array(per_step)))
+        del layers, g_step, g_moe, g_attn
+        torch.cuda.empty_cache()
+    return records
+
+
+def unique_count_cv(U):
+    """Coefficient of variation (sigma / mu over the steps, population sigma) of each layer's
+    unique-expert count; U is [steps, layers]."""
+    U = np.asarray(U, np.float64)
+    return U.std(0) / np.maximum(U.mean(0), 1e-9)
+
+
+def run_decode_sim(args, torch, dm, MoELayer):
+    """The decoding-step harness at the benchmark shape (20 MoE layers of d=2048, 256
+    experts, top-8, block of 32; 128k vocabulary, 1024-token context, heads of 128): one JSON
+    line per routing (block top-k, block routing with p = 0.6, token routing)."""
+    from dmoe_synth import LAYER, ROUTE_TOKEN, STACK20_LAYERS
+    NL = STACK20_LAYERS
+    modes = [("block_p0", LAYER), ("block_p0.6", LAYER.with_(top_p=0.6)),
+             ("token", LAYER.with_(mode=ROUTE_TOKEN))]
+    recs = decode_sim(torch, dm, MoELayer, LAYER, NL, args.sim_blocks, 128000, 1024, 128,
+                      args.seed, modes)
+    mid = NL // 2
+    for r in recs:
+        Ua = r["U"]
+        cv = unique_count_cv(Ua)
+        step_us = float(np.mean(r["t_step"])) * 1e6
+        moe_us, attn_us = float(np.mean(r["t_moe"])) * 1e6, float(np.mean(r["t_attn"])) * 1e6
         print(json.dumps({
-            "suite": "decode_sim", "routing": name, "layers": NL, "block_size": B,
-            "vocab": V, "context": CTX, "blocks": n_blocks, "steps": len(t_step),
-            "tokens_per_step_mean": float(np.mean(per_step)),
+            "suite": "decode_sim", "routing": r["routing"], "layers": NL, "block_size": LAYER.block_size,
+            "vocab": 128000, "context": 1024, "blocks": args.sim_blocks, "steps": len(r["t_step"]),
+            "tokens_per_step_mean": float(np.mean(r["tokens_per_step"])),
             "step_us_mean": step_us, "moe_us": moe_us, "attention_us": attn_us,
             "other_us": max(step_us - moe_us - attn_us, 0.0), "moe_share": moe_us / step_us,
             "attention_share": attn_us / step_us,
             f"U_layer{mid}_mean": float(Ua[:, mid].mean()),
-            f"U_layer{mid}_cv": float(Ua[:, mid].std() / max(Ua[:, mid].mean(), 1e-9)),
+            f"U_layer{mid}_cv": float(cv[mid]),
             "U_mean_all_layers": float(Ua.mean()),
-            "U_cv_per_layer_mean": float(np.mean(Ua.std(0) / np.maximum(Ua.mean(0), 1e-9))),
+            "U_cv_per_layer_mean": float(np.mean(cv)),
             "note": "synthetic stand-ins for attention, embeddings and LM head; MoE by this "
                     "library; shares from graphs of each component replayed on the step's "
                     "inputs"}), flush=True)
-        del layers, g_step, g_moe, g_attn
-        torch.cuda.empty_cache()
 
 
 # ----------------------------------------------------------------------------- main

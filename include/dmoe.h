@@ -230,6 +230,17 @@ dmoe_status dmoe_no_alloc_scratch(void** device_ptr, size_t* bytes);
  * `info` (host, 4 int32, or NULL) receives {code, where, value, 0}. */
 dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info);
 
+/* Diagnostic, not part of the method: makes a bounded wait of the expert launch run out,
+ * so that the timeout path can be tested without any fault on the GPU. While `hold` is
+ * nonzero, every down tile of the decode-size expert launch (at most 64 tokens) of a call
+ * on `workspace` waits for `hold` more gate/up tiles of its group than exist; its wait runs
+ * out after 1 s, the launch records DMOE_ERR_TIMEOUT in the workspace and unwinds (no trap),
+ * and that call's outputs are unspecified. dmoe_get_device_error, which reads the fault,
+ * clears the hold with it; a hold of 0 clears it too. The hold is the last 32-bit word of
+ * the fault record at the head of the workspace. Synchronises `stream`, then writes it with
+ * a blocking copy. DMOE_ERR_INVALID_ARG for a null workspace or a negative hold. */
+dmoe_status dmoe_set_debug_hold(void* workspace, int32_t hold, void* stream);
+
 /* Static description of a status code (host). */
 const char* dmoe_status_string(dmoe_status status);
 

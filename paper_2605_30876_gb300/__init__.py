@@ -94,6 +94,8 @@ def _load() -> ctypes.CDLL:
     lib.dmoe_layer_forward_launches.restype = ctypes.c_int32
     lib.dmoe_set_profile_events.argtypes = [ctypes.c_int32, P, P]
     lib.dmoe_set_profile_events.restype = st
+    lib.dmoe_set_debug_hold.argtypes = [P, ctypes.c_int32, P]
+    lib.dmoe_set_debug_hold.restype = st
     lib.dmoe_router_no_alloc.argtypes = [D, P, P, P, P, P, P, P, P, P]
     lib.dmoe_router_no_alloc.restype = st
     lib.dmoe_router_no_alloc_device_error.argtypes = [P, ctypes.POINTER(ctypes.c_int32)]
@@ -238,6 +240,13 @@ def dmoe_no_alloc_scratch() -> Tuple[int, int]:
     _check(_lib.dmoe_no_alloc_scratch(ctypes.byref(ptr), ctypes.byref(n)),
            "dmoe_no_alloc_scratch")
     return int(ptr.value or 0), n.value
+
+
+def dmoe_set_debug_hold(workspace, hold: int, stream=None) -> None:
+    """Diagnostic: makes the decode-size expert launch's bounded waits run out while
+    `hold` is nonzero (see include/dmoe.h); cleared by dmoe_get_device_error."""
+    _check(_lib.dmoe_set_debug_hold(_ptr(workspace, torch.uint8, "workspace"), int(hold),
+                                    _stream(stream)), "dmoe_set_debug_hold")
 
 
 KERNELS = {"router": 0, "dispatch": 1, "gather": 2, "experts": 3, "combine": 4}

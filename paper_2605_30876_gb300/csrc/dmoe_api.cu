@@ -409,6 +409,18 @@ dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) 
   return rec.code == kErrTimeout ? DMOE_ERR_TIMEOUT : DMOE_ERR_DEVICE;
 }
 
+dmoe_status dmoe_set_debug_hold(void* workspace, int32_t hold, void* stream) {
+  if (workspace == nullptr || hold < 0) return DMOE_ERR_INVALID_ARG;
+  // the fault record heads the workspace; its last word is the hold
+  static_assert(offsetof(DevErrRecord, hold) == 12, "record layout");
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
+  if (e == cudaSuccess)
+    e = cudaMemcpy(static_cast<uint8_t*>(workspace) + offsetof(DevErrRecord, hold), &hold,
+                   sizeof(hold), cudaMemcpyHostToDevice);
+  return cuda_status(e);
+}
+
 dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end) {
   if (kernel < 0 || kernel >= DMOE_KERNEL_COUNT) return DMOE_ERR_INVALID_ARG;
   g_prof[kernel].begin = static_cast<cudaEvent_t>(ev_begin);

@@ -42,7 +42,7 @@ struct DevErrRecord {
   int32_t code;
   int32_t where;
   int32_t value;
-  int32_t pad;
+  int32_t hold;   // diagnostic (normally 0): see dmoe_set_debug_hold
 };
 
 __device__ __forceinline__ void record_error(DevErrRecord* rec, int code, int where, int value) {

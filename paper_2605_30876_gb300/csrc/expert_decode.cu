@@ -331,6 +331,9 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     // ================= TMA producer
     const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
     const uint64_t pol_x = ptx::policy_evict_last();    // x and H: re-read by many tiles
+    // diagnostic hold (normally 0): every down unit waits for this many more gate/up tiles
+    // than its group has, so that its bounded wait runs out
+    const int hold = *reinterpret_cast<volatile int32_t*>(&p.err->hold);
     int stage = 0, issued = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -386,7 +389,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       }
       if (first) ED_AT(5);
       // then the H rows, once every gate/up tile of the group is published
-      const int target = g.Ig / hg;
+      const int target = g.Ig / hg + hold;
       if (ok && ld_acquire(p.h_ready + gi) < target) {
         const uint64_t t0 = ptx::globaltimer_ns();
         while (ld_acquire(p.h_ready + gi) < target) {

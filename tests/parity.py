@@ -187,3 +187,34 @@ def oracle_output(host, idx, scores, tokens=None):
     return O.moe_forward_given_routing(host["x"], host["w_gate"], host["w_up"], host["w_down"],
                                        idx, gate, host.get("ws_gate"), host.get("ws_up"),
                                        host.get("ws_down"), tokens=tokens)
+
+
+class ExpertRows:
+    """w[e] of a device weight tensor as host bf16 bit patterns, copied on first use (the
+    oracle touches only the experts a selection names)."""
+
+    def __init__(self, t: torch.Tensor):
+        self.t, self.cache = t, {}
+
+    def __getitem__(self, e):
+        if e not in self.cache:
+            from dmoe_synth import bf16_bits
+            self.cache[e] = bf16_bits(self.t[e])
+        return self.cache[e]
+
+
+def lazy_host(dev):
+    """Host copies of a layer's inputs for the oracle, the routed experts' weights copied per
+    expert on first use."""
+    from dmoe_synth import bf16_bits
+    out = {}
+    for k_, v in dev.items():
+        if v is None:
+            out[k_] = None
+        elif k_ in ("w_gate", "w_up", "w_down"):
+            out[k_] = ExpertRows(v)
+        elif v.dtype == torch.bfloat16:
+            out[k_] = bf16_bits(v)
+        else:
+            out[k_] = v.cpu().numpy()
+    return out

@@ -35,6 +35,13 @@ LAYER_CASES = {
     "layer_b8_fewer_k4_of8": LAYER_B8.with_(top_k=4, block_top_k=8),
     "tiny_fewer_k1_of2_shared": TINY.with_(top_k=1, block_top_k=2, d_ff_shared=128),
     "layer_token_top4": LAYER.with_(mode=ROUTE_TOKEN, top_k=4),
+    # the paper's top-p sweep ends beside p = 0.6 (Table 3: p_test 0.4 ... 0.8)
+    "layer_block_p04": LAYER.with_(top_p=0.4),
+    "layer_block_p08": LAYER.with_(top_p=0.8),
+    # the block-size x batch x bias grid: its smallest corner, uniform router bias
+    "sweep_B4x1_bias0_block": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0),
+    "sweep_B4x1_bias0_token": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0,
+                                          mode=ROUTE_TOKEN),
 }
 SAMPLED = {"T300_multi_ntile"}
 
@@ -116,6 +123,52 @@ def test_stack_shape_layer_sampled():
     P.check_output(y, ref, tokens=tokens, label="stack_T2048")
 
 
+# Large forwards: every token of a few whole blocks (the oracle is slow at these sizes);
+# the routing of all tokens is checked against the oracle.
+LARGE_CASES = {
+    # the 2048-token stack layer with token routing (the general expert launch at its
+    # heaviest, every expert unique)
+    "stack_T2048_token": (STACK20.with_(mode=ROUTE_TOKEN), (0, 21, 42, 63)),
+    # the block-size x batch x bias grid's largest corner, most skewed router bias
+    "sweep_B64x32_bias1_block": (LAYER.with_(block_size=64, n_blocks=32, bias_scale=1.0),
+                                 (0, 31)),
+    "sweep_B64x32_bias1_token": (LAYER.with_(block_size=64, n_blocks=32, bias_scale=1.0,
+                                             mode=ROUTE_TOKEN), (0, 31)),
+}
+
+
+@pytest.mark.parametrize("name", list(LARGE_CASES))
+def test_large_forward_whole_blocks(name):
+    shape, blocks = LARGE_CASES[name]
+    m = P.dm()
+    from dmoe_synth import layer_inputs
+    from paper_2605_30876_gb300.layer import MoELayer
+    dev = layer_inputs(shape, seed=13, device="cuda")
+    layer = MoELayer.from_shape(shape, dev)
+    y = layer.forward(dev["x"]).clone()
+    st, info = m.dmoe_get_device_error(layer.ws)
+    assert st == 0, info
+    host = P.lazy_host(dev)
+    idx = layer.topk_idx.cpu().numpy()
+    orc = P.oracle_routing(shape, host)
+    near = 0
+    for t in range(shape.T):
+        if orc.set_margin[t] >= P.DELTA and (shape.mode == ROUTE_TOKEN or
+                                             orc.coreset_margin[t // shape.block_size] >= P.DELTA):
+            assert set(idx[t].tolist()) == set(orc.idx[t].tolist()), t
+        else:
+            near += 1
+    np.testing.assert_allclose(layer.topk_gate.cpu().numpy(), O.gates_for(orc.scores, idx),
+                               atol=P.GATE_ATOL)
+    assert int(layer.n_unique.item()) == len(np.unique(idx))
+    B = shape.block_size
+    tokens = np.concatenate([np.arange(b * B, (b + 1) * B) for b in blocks])
+    ref = P.oracle_output(host, idx, orc.scores, tokens=tokens)
+    r, mx = P.check_output(y, ref, tokens=tokens, label=name)
+    print(f"{name}: unique {int(layer.n_unique.item())}, near-tie tokens {near}, "
+          f"blocks {blocks}: rel-L2 {r:.2e} max-abs {mx:.2e}")
+
+
 def test_identical_experts_give_plain_ffn():
     """All routed experts equal: whatever the routing, y = FFN(x) + shared(x) (gates sum to 1)."""
     shape = LAYER.with_(top_p=0.6)
@@ -135,17 +188,7 @@ def test_identical_experts_give_plain_ffn():
     P.check_output(y, ref, label="identical_experts")
 
 
-class _ExpertRows:
-    """w[e] of a device weight tensor as host bf16 bit patterns, copied on first use."""
-
-    def __init__(self, t: torch.Tensor):
-        self.t, self.cache = t, {}
-
-    def __getitem__(self, e):
-        if e not in self.cache:
-            from dmoe_synth import bf16_bits
-            self.cache[e] = bf16_bits(self.t[e])
-        return self.cache[e]
+_ExpertRows = P.ExpertRows
 
 
 def _rms_norm(x: torch.Tensor) -> torch.Tensor:
