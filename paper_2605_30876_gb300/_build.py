@@ -20,7 +20,7 @@ BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libdmoe.so")
 
 SOURCES = ["dmoe_api.cu", "router.cu", "route_cluster.cu", "dispatch.cu", "expert_ffn.cu",
-           "expert_decode.cu", "router_no_alloc.cu"]
+           "expert_decode.cu", "router_no_alloc.cu", "router_logits_tc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2",
          "--expt-relaxed-constexpr", "-I", INCLUDE]

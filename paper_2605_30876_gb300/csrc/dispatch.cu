@@ -1,53 +1,163 @@
-// Dispatch kernel: one CTA computes the unique experts of the forward and the
-// expert -> (token, slot) lists (see dispatch_impl.cuh for the method).
-#include "dispatch_impl.cuh"
+// Dispatch of a forward in two launches over 32-token chunks (one CTA per chunk):
+//   dispatch_count_kernel  the chunk's token bitmap per expert (bits[c][e]: bit l for token
+//                          32c + l); the last CTA to finish (atomic ticket) adds the bitmaps'
+//                          counts over the chunks per expert (base[c][e] = pairs of e in
+//                          chunks before c) and scans over the experts: the offsets, the
+//                          unique list and U
+//   dispatch_place_kernel  each (token, slot) goes to row off[e] + base[c][e] + the popcount
+//                          of bits[c][e] below its token
+// Every sum runs in a fixed order (no order depends on atomics), and each expert's rows are
+// ordered by token, the canonical dispatch form. An id outside [0, E) or an expert twice in
+// one token is recorded as a fault; the outputs are then unspecified (rows stay in range).
+#include "block_reduce.cuh"
 #include "dmoe_internal.cuh"
 #include "trace_log.cuh"
 
 namespace dmoe {
 namespace {
 
-constexpr int kDispatchThreads = 1024;
+constexpr int kDispThreads = 256;
+constexpr int kDispPerThread = (32 * kMaxTopK + kDispThreads - 1) / kDispThreads;
 
-__global__ void __launch_bounds__(kDispatchThreads)
-dispatch_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
-                int32_t* __restrict__ n_unique, int32_t* __restrict__ unique_ids,
-                int32_t* __restrict__ offsets, int32_t* __restrict__ rows,
-                int32_t* __restrict__ pos, DevErrRecord* err) {
-  extern __shared__ __align__(16) uint8_t dsm[];
-  const int nchunks = (T + 31) / 32;
-  uint32_t* bits = reinterpret_cast<uint32_t*>(dsm);                        // [nchunks][E]
-  uint16_t* base = reinterpret_cast<uint16_t*>(bits + (size_t)nchunks * E);  // [nchunks][E]
+__global__ void __launch_bounds__(kDispThreads)
+dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
+                      uint32_t* __restrict__ gbits, int32_t* __restrict__ gbase,
+                      int32_t* __restrict__ goff, int32_t* __restrict__ n_unique,
+                      int32_t* __restrict__ unique_ids, int32_t* __restrict__ offsets,
+                      DevErrRecord* err, int32_t* ticket) {
+  __shared__ uint32_t bits[kMaxExperts];
+  __shared__ int iscr[32];
+  __shared__ int s_last;
+  const int c = blockIdx.x, tid = threadIdx.x;
+  const int t0 = c * 32, ntok = T - t0 < 32 ? T - t0 : 32, np = ntok * k;
+  const int nchunks = gridDim.x, pairs = T * k;
+  // the next launch reads the routing too: it may start once every CTA is past this wait
+  pdl_wait();
   pdl_launch_dependents();
+  KLOG(DMOE_KERNEL_DISPATCH, 0);
+  int ids[kDispPerThread];
+#pragma unroll
+  for (int j = 0; j < kDispPerThread; ++j) {
+    const int p = tid + j * kDispThreads;
+    ids[j] = p < np ? topk_idx[t0 * k + p] : 0;
+  }
+  for (int e = tid; e < E; e += kDispThreads) bits[e] = 0u;
+  __syncthreads();
+#pragma unroll
+  for (int j = 0; j < kDispPerThread; ++j) {
+    const int p = tid + j * kDispThreads;
+    if (p >= np) continue;
+    const int i = t0 * k + p, e = ids[j];
+    if (e < 0 || e >= E) {
+      record_error(err, kErrExpertId, kAtDispatch, i);
+      continue;
+    }
+    const uint32_t bit = 1u << ((i / k) & 31);
+    if (atomicOr(&bits[e], bit) & bit) record_error(err, kErrDupExpert, kAtDispatch, i);
+  }
+  __syncthreads();
+  for (int e = tid; e < E; e += kDispThreads) gbits[(size_t)c * E + e] = bits[e];
+  // the last CTA to get here sees every chunk's bitmap
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(ticket, 1) == nchunks - 1 ? 1 : 0;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  int cnt = 0;
+  if (tid < E) {
+    for (int c0 = 0; c0 < nchunks; c0 += 32) {
+      uint32_t w[32];   // one round of loads per 32 chunks
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        w[j] = c0 + j < nchunks ? __ldcg(gbits + (size_t)(c0 + j) * E + tid) : 0u;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (c0 + j < nchunks) {
+          gbase[(size_t)(c0 + j) * E + tid] = cnt;
+          cnt += __popc(w[j]);
+        }
+    }
+  }
+  int total_pairs = 0, n_u = 0;
+  const int off = block_exclusive_scan_i(tid < E ? cnt : 0, iscr, &total_pairs);
+  const int present = (tid < E && cnt > 0) ? 1 : 0;
+  const int upos = block_exclusive_scan_i(present, iscr, &n_u);
+  if (tid < E) {
+    goff[tid] = off;
+    if (present) {
+      unique_ids[upos] = tid;
+      offsets[upos] = off;
+    }
+  }
+  for (int u = n_u + tid; u < E; u += kDispThreads) unique_ids[u] = -1;
+  for (int u = n_u + tid; u <= E; u += kDispThreads) offsets[u] = pairs;
+  if (tid == 0) {
+    n_unique[0] = n_u;
+    if (total_pairs != pairs) record_error(err, kErrBadDispatch, kAtDispatch, total_pairs);
+    *ticket = 0;   // ready for the next call
+  }
+  KLOG(DMOE_KERNEL_DISPATCH, 1);
+}
+
+__global__ void __launch_bounds__(kDispThreads)
+dispatch_place_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
+                      const uint32_t* __restrict__ gbits, const int32_t* __restrict__ gbase,
+                      const int32_t* __restrict__ goff, int32_t* __restrict__ rows,
+                      int32_t* __restrict__ pos) {
+  __shared__ uint32_t bits[kMaxExperts];
+  __shared__ int base[kMaxExperts];
+  const int c = blockIdx.x, tid = threadIdx.x;
+  const int t0 = c * 32, ntok = T - t0 < 32 ? T - t0 : 32, np = ntok * k;
+  const int pairs = T * k;
+  pdl_launch_dependents();
+  // the routing was complete before the counting launch let this one start
+  int ids[kDispPerThread];
+#pragma unroll
+  for (int j = 0; j < kDispPerThread; ++j) {
+    const int p = tid + j * kDispThreads;
+    ids[j] = p < np ? __ldcg(topk_idx + t0 * k + p) : 0;
+  }
   pdl_wait();
   KLOG(DMOE_KERNEL_DISPATCH, 0);
-  dispatch_cta(topk_idx, T, E, k, n_unique, unique_ids, offsets, rows, pos, err, bits, base);
+  for (int e = tid; e < E; e += kDispThreads) {
+    bits[e] = gbits[(size_t)c * E + e];
+    base[e] = gbase[(size_t)c * E + e] + goff[e];
+  }
+  __syncthreads();
+#pragma unroll
+  for (int j = 0; j < kDispPerThread; ++j) {
+    const int p = tid + j * kDispThreads;
+    const int e = ids[j];
+    if (p >= np || e < 0 || e >= E) continue;
+    const int i = t0 * k + p, l = (i / k) & 31;
+    const int r = base[e] + __popc(bits[e] & ((1u << l) - 1u));
+    if (r >= 0 && r < pairs) {
+      rows[r] = i;
+      pos[i] = r;
+    }
+  }
   KLOG(DMOE_KERNEL_DISPATCH, 1);
 }
 
 }  // namespace
 
-size_t dispatch_smem_bytes(int T, int E) {
-  const size_t nchunks = (size_t)(T + 31) / 32;
-  return nchunks * E * (sizeof(uint32_t) + sizeof(uint16_t));
-}
-
 cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s) {
-  const size_t smem = dispatch_smem_bytes(a.T, a.E);
-  static int attr_dev_mask = 0;  // the dynamic smem limit is a per-device function attribute
-  int dev = 0;
-  cudaGetDevice(&dev);
-  if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
-    cudaError_t e = cudaFuncSetAttribute(dispatch_kernel,
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         200 * 1024);
-    if (e != cudaSuccess) return e;
-    if (dev < 31) attr_dev_mask |= 1 << dev;
-  }
+  if (a.bits == nullptr || a.base == nullptr || a.off == nullptr || a.ticket == nullptr ||
+      a.k > kMaxTopK || a.E > kMaxExperts)
+    return cudaErrorInvalidValue;
+  const int nchunks = (a.T + 31) / 32;
   prof_begin(DMOE_KERNEL_DISPATCH, s);
-  cudaError_t e = launch_ex(dispatch_kernel, dim3(1), dim3(kDispatchThreads), smem, s, true,
-                            a.topk_idx, a.T, a.E, a.k, a.n_unique, a.unique_ids, a.offsets,
-                            a.rows, a.pos, a.err);
+  cudaError_t e = launch_ex(dispatch_count_kernel, dim3(nchunks), dim3(kDispThreads), 0, s, true,
+                            a.topk_idx, a.T, a.E, a.k, a.bits, a.base, a.off, a.n_unique,
+                            a.unique_ids, a.offsets, a.err, a.ticket);
+  if (e == cudaSuccess)
+    e = launch_ex(dispatch_place_kernel, dim3(nchunks), dim3(kDispThreads), 0, s, true,
+                  a.topk_idx, a.T, a.E, a.k, static_cast<const uint32_t*>(a.bits),
+                  static_cast<const int32_t*>(a.base), static_cast<const int32_t*>(a.off),
+                  a.rows, a.pos);
   prof_end(DMOE_KERNEL_DISPATCH, s);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

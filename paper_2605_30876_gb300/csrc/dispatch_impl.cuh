@@ -1,13 +1,7 @@
-// The dispatch of one forward, computed by one CTA (any multiple of 32 threads, at least E):
-// the unique experts and the expert -> (token, slot) lists.
-//
-// Deterministic (no order depends on atomics):
-//   1. membership bitmaps: bits[c][e] has bit l set when token 32c+l routes to expert e
-//      (an id outside [0,E) or an expert twice in one token is recorded as a fault)
-//   2. per expert, the running count over 32-token chunks (base[c][e]) and the total
-//   3. CTA scans over the experts give the unique list and the offsets
-//   4. each (token, slot) lands at offset[e] + base[c][e] + popc(bits[c][e] below lane)
-// which orders every expert's list by token, as the canonical dispatch form requires.
+// The dispatch of a decode-sized forward (at most 64 tokens), computed by one CTA of the
+// routing launch: the unique experts and the expert -> (token, slot) lists, each expert's
+// rows ordered by token (the canonical dispatch form). No order depends on atomics. Larger
+// forwards take the two launches of dispatch.cu.
 #pragma once
 
 #ifndef DMOE_STAMP
@@ -19,79 +13,9 @@
 
 namespace dmoe {
 
-// `bits` and `base` are shared-memory buffers of ceil(T/32) * E entries.
-__device__ inline void dispatch_cta(const int32_t* topk_idx, int T, int E, int k,
-                                    int32_t* __restrict__ n_unique,
-                                    int32_t* __restrict__ unique_ids,
-                                    int32_t* __restrict__ offsets, int32_t* __restrict__ rows,
-                                    int32_t* __restrict__ pos, DevErrRecord* err, uint32_t* bits,
-                                    uint16_t* base) {
-  __shared__ int off_e[kMaxExperts];
-  __shared__ int iscr[32];
-  __shared__ int bad;
-  const int nchunks = (T + 31) / 32;
-  const int tid = threadIdx.x, nthr = blockDim.x;
-  const int pairs = T * k;
-
-  if (tid == 0) bad = 0;
-  for (int i = tid; i < nchunks * E; i += nthr) bits[i] = 0u;
-  __syncthreads();
-  for (int i = tid; i < pairs; i += nthr) {
-    const int t = i / k, e = topk_idx[i];
-    if (e < 0 || e >= E) {
-      record_error(err, kErrExpertId, kAtDispatch, i);
-      bad = 1;
-      continue;
-    }
-    const uint32_t bit = 1u << (t & 31);
-    const uint32_t old = atomicOr(&bits[(t >> 5) * E + e], bit);
-    if (old & bit) {
-      record_error(err, kErrDupExpert, kAtDispatch, i);
-      bad = 1;
-    }
-  }
-  __syncthreads();
-  if (bad) return;  // uniform: the outputs are unspecified after a recorded fault
-
-  // running counts per expert over chunks
-  int cnt = 0;
-  if (tid < E) {
-    for (int c = 0; c < nchunks; ++c) {
-      base[c * E + tid] = (uint16_t)cnt;
-      cnt += __popc(bits[c * E + tid]);
-    }
-  }
-  int total_pairs = 0, n_u = 0;
-  const int off = block_exclusive_scan_i(tid < E ? cnt : 0, iscr, &total_pairs);
-  const int present = (tid < E && cnt > 0) ? 1 : 0;
-  const int upos = block_exclusive_scan_i(present, iscr, &n_u);
-  if (tid < E) {
-    off_e[tid] = off;
-    if (present) {
-      unique_ids[upos] = tid;
-      offsets[upos] = off;
-    }
-  }
-  // tail of the fixed-size outputs
-  for (int u = n_u + tid; u < E; u += nthr) unique_ids[u] = -1;
-  for (int u = n_u + tid; u <= E; u += nthr) offsets[u] = pairs;
-  if (tid == 0) {
-    n_unique[0] = n_u;
-    if (total_pairs != pairs) record_error(err, kErrBadDispatch, kAtDispatch, total_pairs);
-  }
-  __syncthreads();
-  for (int i = tid; i < pairs; i += nthr) {
-    const int t = i / k, e = topk_idx[i], c = t >> 5, l = t & 31;
-    const uint32_t w = bits[c * E + e];
-    const int r = off_e[e] + base[c * E + e] + __popc(w & ((1u << l) - 1u));
-    rows[r] = i;
-    pos[i] = r;
-  }
-}
-
-// The same outputs for T <= 64 tokens, with a two-word token mask per expert: one 32-bit
-// atomic OR per (token, slot), one packed CTA scan for the offsets and the unique positions.
-// Needs blockDim.x >= E (a multiple of 32, at most 256).
+// A two-word token mask per expert: one 32-bit atomic OR per (token, slot), one packed CTA
+// scan for the offsets and the unique positions. Needs blockDim.x >= E (a multiple of 32,
+// at most 256).
 __device__ inline void dispatch_small_cta(const int32_t* topk_idx, int T, int E, int k,
                                           int32_t* __restrict__ n_unique,
                                           int32_t* __restrict__ unique_ids,

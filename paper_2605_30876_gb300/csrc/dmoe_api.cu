@@ -81,7 +81,10 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   const size_t T = (size_t)d.n_blocks * d.block_size, E = d.n_experts, k = d.top_k;
   const size_t dm = d.d_model, I = d.d_ff, Is = d.d_ff_shared;
   w.router_splits = router_splits(d);
-  w.n_max = expert_n_max((int)T);
+  const bool tc = !route_cluster_ok((int)T, (int)dm, (int)E) &&
+                  router_tc_ok((int)T, (int)dm, (int)E);
+  w.tc_splits = tc ? router_tc_splits((int)T, (int)dm) : 0;
+  w.n_max = expert_n_max(d);
   size_t off = 0;
   auto take = [&](size_t bytes) {
     const size_t o = off;
@@ -104,12 +107,19 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.xperm = take(2 * T * k * dm);
   w.h = take(2 * T * k * I);
   w.hs = take(2 * T * Is);
-  w.h_ready = take(sizeof(int32_t) * experts_ready_counters((int)T, (int)E));
+  w.h_ready = take(sizeof(int32_t) * experts_ready_counters((int)T, (int)E, w.n_max));
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
   const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
   w.hdense = take(dec ? 2 * (E + 1) * (size_t)((T + 15) / 16 * 16) * (I > Is ? I : Is) : 0);
   w.spec = take(dec ? sizeof(uint32_t) * d.n_blocks * spec_words((int)k) : 0);
+  const size_t nchunks = (T + 31) / 32;
+  w.disp_bits = take(sizeof(uint32_t) * nchunks * E);
+  w.disp_base = take(sizeof(int32_t) * nchunks * E);
+  w.disp_off = take(sizeof(int32_t) * E);
+  w.w_parts_bytes = tc ? router_tc_parts_bytes((int)dm, (int)E) : 0;
+  w.w_parts = take(w.w_parts_bytes);
+  w.tc_part = take(sizeof(float) * (size_t)w.tc_splits * T * E);
   w.total = off;
   return w;
 }
@@ -152,6 +162,13 @@ dmoe_status check_ws(const dmoe_layer_desc* d, void* ws, size_t ws_bytes, Worksp
 template <class T>
 T* at(void* ws, size_t off) {
   return reinterpret_cast<T*>(static_cast<uint8_t*>(ws) + off);
+}
+
+void set_dispatch_scratch(DispatchArgs* a, void* ws, const Workspace& plan) {
+  a->bits = at<uint32_t>(ws, plan.disp_bits);
+  a->base = at<int32_t>(ws, plan.disp_base);
+  a->off = at<int32_t>(ws, plan.disp_off);
+  a->ticket = at<int32_t>(ws, plan.tickets) + kDispatchTicket;
 }
 
 dmoe_status cuda_status(cudaError_t e) {
@@ -197,6 +214,9 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.top_p = desc->top_p;
   a.err = at<DevErrRecord>(ws, plan.err);
   a.shared_pf = shared_pf;
+  a.w_parts = plan.w_parts_bytes > 0 ? at<__nv_bfloat16>(ws, plan.w_parts) : nullptr;
+  a.tc_splits = plan.tc_splits;
+  a.tc_part = plan.tc_splits > 0 ? at<float>(ws, plan.tc_part) : nullptr;
   return cuda_status(launch_router(a, dsp, at<int32_t>(ws, plan.tickets), s));
 }
 
@@ -214,6 +234,7 @@ dmoe_status run_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx, i
   a.E = desc->n_experts;
   a.k = desc->top_k;
   a.err = at<DevErrRecord>(ws, plan.err);
+  set_dispatch_scratch(&a, ws, plan);
   return cuda_status(launch_dispatch(a, s));
 }
 
@@ -372,6 +393,7 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   dsp.E = desc->n_experts;
   dsp.k = desc->top_k;
   dsp.err = at<DevErrRecord>(workspace, plan.err);
+  set_dispatch_scratch(&dsp, workspace, plan);
   // block top-k through the decode-size launches: the expert launch starts streaming on the
   // early-published coresets, before the routing launch ends (only when every token keeps
   // the whole coreset, so that the coresets' union is the unique set)
@@ -453,8 +475,9 @@ int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc) {
     n += 1;                                                   // routing with the dispatch
   } else {
     n += 2;                                                   // logits, softmax / top-k
+    n += router_tc_ok(T, desc->d_model, desc->n_experts) ? 1 : 0;   // the split of W_r
     n += desc->mode == DMOE_ROUTE_BLOCK ? 1 : 0;              // Algorithm 1
-    n += 1;                                                   // dispatch
+    n += 2;                                                   // dispatch: count, place
   }
   if (experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared))
     n += 2;                                                   // experts, combine

@@ -74,21 +74,33 @@ struct Workspace {
   size_t h;            // bf16 [T*k, I]   SwiGLU intermediate of the routed experts
   size_t hs;           // bf16 [T, I_s]   shared-expert intermediate
   size_t h_ready;      // int32 [(E+1) * token tiles]: published gate/up tiles
-  size_t yslot;        // fp32 [T*k, d]   expert outputs per (token, slot)
-  size_t yshared;      // fp32 [T, d]
+  size_t yslot;        // [T*k, d] expert outputs per (token, slot): fp32 (decode-size path)
+                       // or bf16 (general path); sized for fp32
+  size_t yshared;      // [T, d], the same element type
   size_t hdense;       // bf16 [(E+1) * n_pad, max(I, I_s)]: H per group over all tokens
   size_t spec;         // int32 [n_blocks, k]: the coreset of every block (block top-k call)
                        // (decode-size forwards only)
+  size_t disp_bits;    // u32 [ceil(T/32), E]: dispatch, token bitmap per (32-token chunk, expert)
+  size_t disp_base;    // int32 [ceil(T/32), E]: dispatch, pairs of the expert in earlier chunks
+  size_t disp_off;     // int32 [E]: dispatch, first row of every expert (all experts)
+  size_t w_parts;      // bf16 [3E, d]: split of W_r for the tcgen05 router (large forwards)
+  size_t w_parts_bytes;
+  size_t tc_part;      // fp32 [tc_splits, T, E]: the tcgen05 router's partial logits
   size_t total;
   int router_splits;
+  int tc_splits;       // slices of d of the tcgen05 router logits (0: not used)
   int n_max;           // token tile (MMA N) of the expert GEMMs
 };
 
 // Token tile (MMA N) of the general expert kernel: every group's rows are covered by tiles
-// of n_max; 64 rows up to 256 tokens per forward, 128 above (measured: wider tiles leave two
-// pipeline stages in shared memory, narrower ones re-stream the weights for more tiles).
-inline int expert_n_max(int T) {
-  const int cap = T <= 256 ? 64 : 128;
+// of n_max rows (a tile of at most half of that loads a half-height box). Each tile streams
+// the group's weights through its SM again, so the tile is as wide as the forward allows:
+// 128 rows, or 256 in block mode with blocks of 16 or more tokens at 1024 or more tokens
+// (every unique expert then takes whole blocks, hundreds of rows; one K box per stage keeps
+// four stages in shared memory).
+inline int expert_n_max(const dmoe_layer_desc& d) {
+  const int T = d.n_blocks * d.block_size;
+  const int cap = (d.mode == DMOE_ROUTE_BLOCK && d.block_size >= 16 && T >= 1024) ? 256 : 128;
   int n = ((T + 15) / 16) * 16;
   return n > cap ? cap : (n < 16 ? 16 : n);
 }
@@ -159,6 +171,10 @@ struct RouterArgs {
   DevErrRecord* err;
   L2Prefetch shared_pf;   // the shared expert's weights (one "expert")
   bool probs_requested;   // the caller wants the scores in `probs`
+  __nv_bfloat16* w_parts; // [3E, d]: the bf16 split of W_r for the tcgen05 router, or null
+                          // (then the mma.sync / FFMA logits run)
+  int tc_splits;          // slices of d of the tcgen05 logits
+  float* tc_part;         // [tc_splits, T, E]: their partial sums
   // block top-k (p <= 0) in the fused decode-size call: every block's coreset, which is
   // then the block's routing, is published early here: spec_words(k) words per block, three
   // ids and a marker byte each, one 32-bit store per word (a word reads as zero until it is
@@ -175,7 +191,14 @@ struct DispatchArgs {
   int32_t* pos;
   int T, E, k;
   DevErrRecord* err;
+  // scratch of the multi-CTA dispatch (Workspace::disp_*) and its ticket (zero between calls)
+  uint32_t* bits;
+  int32_t* base;
+  int32_t* off;
+  int32_t* ticket;
 };
+// ticket index (in Workspace::tickets) of the dispatch launch
+constexpr int kDispatchTicket = 1;
 cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s);
 
 // Routing of one forward. With `dsp` set, the dispatch is computed too (inside the fused
@@ -188,6 +211,14 @@ bool route_cluster_ok(int T, int d, int E);
 // into a.logits_part [T, E] (no split).
 bool route_cluster_logits_ok(int d, int E);
 cudaError_t launch_logits_cluster(const RouterArgs& a, cudaStream_t s);
+// The logits of a large forward on tcgen05 (router_logits_tc.cu): the split of W_r into
+// a.w_parts, then the products over `splits` slices of d into a.tc_part [splits, T, E]
+// (router_softmax_kernel adds them in order, with the bias). Needs T >= 128, d % 64 == 0,
+// E % 16 == 0; router_tc_splits gives the split.
+bool router_tc_ok(int T, int d, int E);
+int router_tc_splits(int T, int d);
+size_t router_tc_parts_bytes(int d, int E);
+cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s);
 cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                                  cudaStream_t s);
 
@@ -202,7 +233,7 @@ struct ExpertArgs {
   __nv_bfloat16* y;
   // workspace
   __nv_bfloat16* xperm; __nv_bfloat16* h; __nv_bfloat16* hs;
-  float* yslot; float* yshared;
+  void* yslot; void* yshared;   // fp32 (decode-size path) or bf16 (general path) rows
   int32_t* h_ready;
   __nv_bfloat16* hdense;  // decode-size path: H per group over all tokens
   int32_t* tickets;       // kRouteTickets ints, zero between calls
@@ -217,14 +248,15 @@ struct ExpertArgs {
   int T, d, E, k, I, Is, n_max;
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
-int experts_ready_counters(int T, int E);
+int experts_ready_counters(int T, int E, int n_max);
 // gate-weighted combine of the expert rows into y (the last launch of both expert paths);
 // it also clears zero[0 .. n_zero) and zero2[0 .. n_zero2) once the launch before it has
 // ended. meta_early: the slot indices and gates may be read before that launch ends (they
 // were complete before it released the combine)
+// rows_bf16: the rows per (token, slot) and the shared rows are bf16 (general path), else fp32
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = nullptr,
                            int n_zero = 0, uint32_t* zero2 = nullptr, int n_zero2 = 0,
-                           bool meta_early = false);
+                           bool meta_early = false, bool rows_bf16 = false);
 
 // Words of one block's published coreset (three 8-bit ids and a marker byte per word).
 __host__ __device__ inline int spec_words(int k) { return (k + 2) / 3; }

@@ -820,8 +820,8 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.offsets = a.offsets;
   p.rows = a.rows;
   p.hdense = a.hdense;
-  p.yslot = a.yslot;
-  p.yshared = a.yshared;
+  p.yslot = static_cast<float*>(a.yslot);
+  p.yshared = static_cast<float*>(a.yshared);
   p.h_ready = a.h_ready;
   p.spec_words = a.spec_words;
   p.spec_blocks = a.spec_blocks;

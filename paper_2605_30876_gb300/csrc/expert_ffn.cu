@@ -14,7 +14,8 @@
 //                       warps holding "gate", which write h = silu(gate) * up as bf16 H and
 //                       then publish the tile (h_ready counter)
 //     down unit         (group, 128 rows of d, token tile): D = W_down * H^T; the epilogue
-//                       stores the fp32 rows per (token, slot)
+//                       stores the rows per (token, slot) as bf16 (half the bytes of fp32
+//                       through HBM twice; the combine adds them in fp32)
 //   combine_kernel      y_t = sum over slots (slot order) of g_tj * row + shared -> bf16
 //
 // A group is one unique expert (dispatch order) or the shared expert (all T tokens). The
@@ -38,10 +39,8 @@ namespace {
 
 constexpr int kThreads = 192;                      // 6 warps
 constexpr int kBoxBytes = 64 * 128;                // one TMA box: 64 rows x 128 B
-constexpr int kKBoxes = 2;                         // K boxes per stage: K = 128 per stage
-constexpr int kStageK = kKBoxes * kTileK;
+constexpr int kMaxKBoxes = 2;                      // K boxes per stage: 1 or 2 (K = 64, 128)
 constexpr int kATileBytes = kTileM * 128;          // 16 KB: 128 rows x 64 K (one K box)
-constexpr int kAStageBytes = kKBoxes * kATileBytes;  // 32 KB
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr int kMaxStages = 8;
@@ -53,14 +52,16 @@ struct GemmParams {
   const int32_t* offsets;
   __nv_bfloat16* h;       // [T*k, I]
   __nv_bfloat16* hs;      // [T, Is]
-  float* yslot;           // [T*k, d]
-  float* yshared;         // [T, d]
+  __nv_bfloat16* yslot;   // [T*k, d] bf16 (the combine sums them in fp32)
+  __nv_bfloat16* yshared; // [T, d] bf16
   int32_t* h_ready;       // [(E+1) * ntiles]: gate/up tiles done per (group, token tile)
   DevErrRecord* err;
   const void* w_down;     // routed W_down, prefetched into L2 for the unique experts
   const void* ws_gate; const void* ws_up; const void* ws_down;  // shared, prefetched if set
   int T, d, E, k, I, Is;
   int n_max;              // token tile = rows of the B box
+  int n_half;             // rows of the half box (token tiles of at most this many rows)
+  int kbs;                // K boxes per stage (1 for 256-row token tiles, else 2)
   int ntiles;             // token tiles per group at most
   int stages;
   int n_acc;              // accumulator buffers in TMEM
@@ -73,6 +74,7 @@ struct Maps {
   CUtensorMap wd, sd;           // down weights, 128-row boxes (routed [E*d,I], shared [d,Is])
   CUtensorMap xp, x;            // gate/up token rows: xperm [T*k,d], x [T,d]
   CUtensorMap h, hs;            // down token rows: H [T*k,I], Hs [T,Is]
+  CUtensorMap xph, hh;          // xperm and H with half-height boxes (small token tiles)
 };
 
 using ptx::epi_all;
@@ -110,10 +112,13 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   uint8_t* smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);  // 1024-B aligned
 
   const int stages = p.stages;
-  const uint32_t b_box = (uint32_t)p.n_max * 128u;            // one B box
-  const uint32_t b_stage = kKBoxes * b_box;
+  const int kbs = p.kbs;                                      // K boxes per stage
+  const int stage_k = kbs * kTileK;
+  const uint32_t a_stage = (uint32_t)kbs * kATileBytes;
+  const uint32_t b_box = (uint32_t)p.n_max * 128u;            // one B box (slot size)
+  const uint32_t b_stage = (uint32_t)kbs * b_box;
   const uint32_t off_a = 0;
-  const uint32_t off_b = off_a + (uint32_t)stages * kAStageBytes;
+  const uint32_t off_b = off_a + (uint32_t)stages * a_stage;
   const uint32_t off_x = off_b + (uint32_t)stages * b_stage;
   const uint32_t x_bytes = 2u * 64u * kXchgStride * 4u;        // [128][17] fp32
   const uint32_t off_bar = (off_x + x_bytes + 7u) & ~7u;
@@ -267,10 +272,12 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       if (pre[mid] <= v) lo = mid; else hi = mid - 1;
     }
     r.g = p.has_shared ? (lo == 0 ? U : lo - 1) : lo;
-    const int mt = r.gu ? ((r.g < U ? p.I : p.Is) / 64) : (p.d / kTileM);
+    // token tile innermost: the CTAs that take a weight tile's token tiles take them at
+    // the same time, so that the tile comes from HBM once and from L2 for the others
+    const int nt = (g_cnt[r.g] + p.n_max - 1) / p.n_max;
     const int local = v - pre[lo];
-    r.n = local / mt;
-    r.m = local - r.n * mt;
+    r.m = local / nt;
+    r.n = local - r.m * nt;
     return r;
   };
   auto wait = [&](uint64_t* bar, uint32_t parity, int value) -> bool {
@@ -292,9 +299,9 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   if (warp == 0) {
     // ================= TMA producer
     if (lane == 0) {
-      const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
+      const uint64_t pol_first = ptx::policy_evict_first();   // weights read by one tile
+      const uint64_t pol_norm = ptx::policy_evict_normal();   // ... or by several
       const uint64_t pol_x = ptx::policy_evict_last();    // activations: re-read by tiles
-      const uint32_t tx_bytes = kAStageBytes + b_stage;
       int stage = 0;
       uint32_t phase = 0;
       int issued = 0;
@@ -303,22 +310,27 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++li) {
         const Unit un = decode(u);
         const bool shared = un.g >= U;
+        const uint64_t pol_w = g_cnt[un.g] > p.n_max ? pol_norm : pol_first;
+        // a routed token tile of at most n_half rows loads the half-height box
+        const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
+        const bool half = !shared && nvalid <= p.n_half;
+        const uint32_t b_bytes = (uint32_t)kbs * (half ? (uint32_t)p.n_half * 128u : b_box);
+        const uint32_t tx_bytes = a_stage + b_bytes;
         if (li < 8) { DMOE_TRACE_SET(2 + 6 * li, u); DMOE_TRACE_AT(3 + 6 * li); }
         if (un.gu) {
           const int arow = shared ? un.m * 64 : g_e[un.g] * p.I + un.m * 64;
           const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
           const CUtensorMap* mg = shared ? &tm.sg : &tm.wg;
           const CUtensorMap* mu = shared ? &tm.su : &tm.wu;
-          const CUtensorMap* mb = shared ? &tm.x : &tm.xp;
-          const int kc = p.d / kStageK;
+          const CUtensorMap* mb = shared ? &tm.x : (half ? &tm.xph : &tm.xp);
+          const int kc = p.d / stage_k;
           for (int c = 0; c < kc; ++c) {
             if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
             ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
+            uint8_t* a_dst = smem + off_a + stage * a_stage;
             uint8_t* b_dst = smem + off_b + stage * b_stage;
-#pragma unroll
-            for (int kb = 0; kb < kKBoxes; ++kb) {
-              const int kx = c * kStageK + kb * kTileK;
+            for (int kb = 0; kb < kbs; ++kb) {
+              const int kx = c * stage_k + kb * kTileK;
               ptx::tma_load_2d(a_dst + kb * kATileBytes, mg, &full[stage], kx, arow, pol_w);
               ptx::tma_load_2d(a_dst + kb * kATileBytes + kBoxBytes, mu, &full[stage], kx, arow,
                                pol_w);
@@ -332,8 +344,8 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           const int arow = shared ? un.m * kTileM : g_e[un.g] * p.d + un.m * kTileM;
           const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
           const CUtensorMap* ma = shared ? &tm.sd : &tm.wd;
-          const CUtensorMap* mb = shared ? &tm.hs : &tm.h;
-          const int kc = Kg / kStageK;
+          const CUtensorMap* mb = shared ? &tm.hs : (half ? &tm.hh : &tm.h);
+          const int kc = Kg / stage_k;
           const int pre = kc < stages ? kc : stages;
           const int stage0 = stage;
           const uint32_t phase0 = phase;
@@ -341,10 +353,9 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           for (int c = 0; c < pre; ++c) {
             if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
             ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
-#pragma unroll
-            for (int kb = 0; kb < kKBoxes; ++kb)
-              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], c * kStageK + kb * kTileK,
+            uint8_t* a_dst = smem + off_a + stage * a_stage;
+            for (int kb = 0; kb < kbs; ++kb)
+              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], c * stage_k + kb * kTileK,
                                arow, pol_w);
             ++issued;
             if (++stage == stages) { stage = 0; phase ^= 1u; }
@@ -372,13 +383,12 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           for (int c = 0; c < pre; ++c) {
             if (ok) {
               uint8_t* b_dst = smem + off_b + st * b_stage;
-#pragma unroll
-              for (int kb = 0; kb < kKBoxes; ++kb)
-                ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], c * kStageK + kb * kTileK, brow,
+              for (int kb = 0; kb < kbs; ++kb)
+                ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], c * stage_k + kb * kTileK, brow,
                                  pol_x);
             } else {
               // keep the barrier accounting whole: complete the stage without B data
-              ptx::mbar_complete_tx_local(&full[st], b_stage);
+              ptx::mbar_complete_tx_local(&full[st], b_bytes);
             }
             if (++st == stages) st = 0;
           }
@@ -387,11 +397,10 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           for (int c = pre; c < kc; ++c) {
             if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
             ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * kAStageBytes;
+            uint8_t* a_dst = smem + off_a + stage * a_stage;
             uint8_t* b_dst = smem + off_b + stage * b_stage;
-#pragma unroll
-            for (int kb = 0; kb < kKBoxes; ++kb) {
-              const int kx = c * kStageK + kb * kTileK;
+            for (int kb = 0; kb < kbs; ++kb) {
+              const int kx = c * stage_k + kb * kTileK;
               ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], kx, arow, pol_w);
               ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], kx, brow, pol_x);
             }
@@ -426,7 +435,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         const Unit un = decode(u);
         const bool shared = un.g >= U;
         const int Kg = un.gu ? p.d : (shared ? p.Is : p.I);
-        const int kc = Kg / kStageK;
+        const int kc = Kg / stage_k;
         const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
         const uint32_t n_mma = (uint32_t)((nvalid + 15) & ~15);
         const uint32_t idesc = ptx::idesc_bf16(kTileM, n_mma);
@@ -437,10 +446,9 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           if (!wait(&full[stage], phase, u)) { ok = false; break; }
           ptx::tc_fence_after();
           if (!*s_abort) {
-            const uint32_t a0 = ptx::smem_addr(smem + off_a + stage * kAStageBytes);
+            const uint32_t a0 = ptx::smem_addr(smem + off_a + stage * a_stage);
             const uint32_t b0 = ptx::smem_addr(smem + off_b + stage * b_stage);
-#pragma unroll
-            for (int kb = 0; kb < kKBoxes; ++kb)
+            for (int kb = 0; kb < kbs; ++kb)
 #pragma unroll
               for (int kk = 0; kk < kTileK / 16; ++kk)
                 ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kATileBytes + kk * 32),
@@ -528,15 +536,15 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         if (tid == 64) red_release_add(p.h_ready + un.g * p.ntiles + un.n, 1);
       } else {
         const int drow = un.m * kTileM + q * 32 + lane;
-        float* out = shared ? p.yshared + (size_t)col0 * p.d
-                            : p.yslot + (size_t)(g_row0[un.g] + col0) * p.d;
+        __nv_bfloat16* out = shared ? p.yshared + (size_t)col0 * p.d
+                                    : p.yslot + (size_t)(g_row0[un.g] + col0) * p.d;
         for (int c0 = 0; c0 < n_mma; c0 += 16) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
           ptx::tmem_ld_wait();
 #pragma unroll
           for (int c = 0; c < 16; ++c)
-            if (c0 + c < nvalid) out[(size_t)(c0 + c) * p.d + drow] = v[c];
+            if (c0 + c < nvalid) out[(size_t)(c0 + c) * p.d + drow] = __float2bfloat16_rn(v[c]);
         }
         ptx::tc_fence_before();
         ptx::mbar_arrive(&acc_empty[acc]);
@@ -557,7 +565,11 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   }
 }
 
-// xperm[r, :] = x[rows[r] / k, :]; block 0 also clears the gate/up tile counters.
+// xperm[r, :] = x[rows[r] / k, :]; block 0 also clears the gate/up tile counters. A CTA
+// copies kGatherRows consecutive rows at a time (so that the rows being written at any
+// moment form one contiguous range of xperm): their indices are read in one round, then
+// every thread has one 16-byte piece of each row in flight.
+constexpr int kGatherRows = 8;
 __global__ void __launch_bounds__(256)
 gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ rows,
               __nv_bfloat16* __restrict__ xperm, int32_t* __restrict__ h_ready, int n_ready,
@@ -568,13 +580,43 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_ready; i += blockDim.x) h_ready[i] = 0;
   const int vec = d / 8;  // uint4 per row
-  for (int r = blockIdx.x; r < pairs; r += gridDim.x) {
-    const int t = rows[r] / k;
-    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)t * d);
-    uint4* dst = reinterpret_cast<uint4*>(xperm + (size_t)r * d);
-    for (int i = threadIdx.x; i < vec; i += blockDim.x) dst[i] = src[i];
+  for (int r0 = blockIdx.x * kGatherRows; r0 < pairs; r0 += gridDim.x * kGatherRows) {
+    const uint4* src[kGatherRows];
+#pragma unroll
+    for (int j = 0; j < kGatherRows; ++j)
+      src[j] = reinterpret_cast<const uint4*>(
+          x + (size_t)(r0 + j < pairs ? rows[r0 + j] / k : 0) * d);
+    uint4* dst = reinterpret_cast<uint4*>(xperm + (size_t)r0 * d);
+    for (int i = threadIdx.x; i < vec; i += blockDim.x) {
+      uint4 v[kGatherRows];
+#pragma unroll
+      for (int j = 0; j < kGatherRows; ++j)
+        if (r0 + j < pairs) v[j] = src[j][i];
+#pragma unroll
+      for (int j = 0; j < kGatherRows; ++j)
+        if (r0 + j < pairs) dst[(size_t)j * vec + i] = v[j];
+    }
   }
   KLOG(DMOE_KERNEL_GATHER, 1);
+}
+
+// kCombineCols consecutive row values as fp32 (fp32 rows of the decode-size path, bf16
+// rows of the general path): one 16-byte load per 8 bf16 or 4 fp32 values.
+constexpr int kCombineCols = 8;
+__device__ __forceinline__ void load8(const float* src, float (&v)[8]) {
+  const float4 a = *reinterpret_cast<const float4*>(src);
+  const float4 b = *reinterpret_cast<const float4*>(src + 4);
+  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+}
+__device__ __forceinline__ void load8(const __nv_bfloat16* src, float (&v)[8]) {
+  const uint4 u = *reinterpret_cast<const uint4*>(src);
+  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+    v[2 * i] = f.x;
+    v[2 * i + 1] = f.y;
+  }
 }
 
 // y[t, :] = bf16( sum_j g[t,j] * yslot[pos[t*k + j], :] (slot order) + yshared[t, :] );
@@ -583,14 +625,15 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
 // read before the dependency wait: the caller guarantees that they were complete before the
 // launch before this one could let this one start (the decode-size expert launch releases
 // it only at its end, after its own wait for the routing launch that wrote them).
+template <typename Row>
 __global__ void __launch_bounds__(256)
-combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshared,
+combine_kernel(const Row* __restrict__ yslot, const Row* __restrict__ yshared,
                const int32_t* __restrict__ pos, const float* __restrict__ gate,
                __nv_bfloat16* __restrict__ y, int k, int d, int has_shared, int32_t* zero,
                int n_zero, uint32_t* zero2, int n_zero2, int meta_early) {
   pdl_launch_dependents();
   const int t = blockIdx.y;
-  const int c = (blockIdx.x * blockDim.x + threadIdx.x) * 4;
+  const int c = (blockIdx.x * blockDim.x + threadIdx.x) * kCombineCols;
   int r[kMaxTopK];
   float gj[kMaxTopK];
   if (meta_early) {
@@ -617,30 +660,30 @@ combine_kernel(const float* __restrict__ yslot, const float* __restrict__ yshare
       }
   }
   // every row load is issued before the first product; the sum keeps the slot order
-  float4 v[kMaxTopK];
+  float v[kMaxTopK][kCombineCols];
 #pragma unroll
   for (int j = 0; j < kMaxTopK; ++j)
-    if (j < k) v[j] = *reinterpret_cast<const float4*>(yslot + (size_t)r[j] * d + c);
-  float4 vs = make_float4(0.f, 0.f, 0.f, 0.f);
-  if (has_shared) vs = *reinterpret_cast<const float4*>(yshared + (size_t)t * d + c);
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (j < k) load8(yslot + (size_t)r[j] * d + c, v[j]);
+  float vs[kCombineCols];
+  if (has_shared) load8(yshared + (size_t)t * d + c, vs);
+  float acc[kCombineCols];
+#pragma unroll
+  for (int i = 0; i < kCombineCols; ++i) acc[i] = 0.f;
 #pragma unroll
   for (int j = 0; j < kMaxTopK; ++j)
-    if (j < k) {
-      acc.x = fmaf(gj[j], v[j].x, acc.x);
-      acc.y = fmaf(gj[j], v[j].y, acc.y);
-      acc.z = fmaf(gj[j], v[j].z, acc.z);
-      acc.w = fmaf(gj[j], v[j].w, acc.w);
-    }
-  if (has_shared) {
-    acc.x += vs.x; acc.y += vs.y; acc.z += vs.z; acc.w += vs.w;
+    if (j < k)
+#pragma unroll
+      for (int i = 0; i < kCombineCols; ++i) acc[i] = fmaf(gj[j], v[j][i], acc[i]);
+  if (has_shared)
+#pragma unroll
+    for (int i = 0; i < kCombineCols; ++i) acc[i] += vs[i];
+  uint32_t out[kCombineCols / 2];
+#pragma unroll
+  for (int i = 0; i < kCombineCols / 2; ++i) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(acc[2 * i], acc[2 * i + 1]);
+    out[i] = *reinterpret_cast<const uint32_t*>(&h);
   }
-  __nv_bfloat162 lo = __floats2bfloat162_rn(acc.x, acc.y);
-  __nv_bfloat162 hi = __floats2bfloat162_rn(acc.z, acc.w);
-  uint2 out;
-  out.x = *reinterpret_cast<uint32_t*>(&lo);
-  out.y = *reinterpret_cast<uint32_t*>(&hi);
-  *reinterpret_cast<uint2*>(y + (size_t)t * d + c) = out;
+  *reinterpret_cast<uint4*>(y + (size_t)t * d + c) = make_uint4(out[0], out[1], out[2], out[3]);
   KLOG(DMOE_KERNEL_COMBINE, 1);
 }
 
@@ -710,18 +753,20 @@ extern "C" int dmoe_debug_trace_clear() {
 DMOE_KLOG_EXPORT(dmoe_debug_klog_experts)
 #endif
 
-int experts_ready_counters(int T, int E) {
-  const int n_max = expert_n_max(T);
+int experts_ready_counters(int T, int E, int n_max) {
   return (E + 1) * ((T + n_max - 1) / n_max);
 }
 
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   const int pairs = a.T * a.k;
   const bool has_shared = a.Is > 0;
-  const int n_ready = experts_ready_counters(a.T, a.E);
+  const int n_ready = experts_ready_counters(a.T, a.E, a.n_max);
   // 1. gather x in dispatch order; clear the gate/up tile counters
   {
-    int grid = pairs < 1024 ? pairs : 1024;
+    const int want = (pairs + kGatherRows - 1) / kGatherRows;
+    const int cap = device_sm_count() * 8;
+    int grid = want < cap ? want : cap;
+    if (grid < 1) grid = 1;
     prof_begin(DMOE_KERNEL_GATHER, s);
     cudaError_t e = launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, true, a.x, a.rows,
                               a.xperm, a.h_ready, n_ready, pairs, a.k, a.d);
@@ -734,8 +779,8 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   gp.offsets = a.offsets;
   gp.h = a.h;
   gp.hs = a.hs;
-  gp.yslot = a.yslot;
-  gp.yshared = a.yshared;
+  gp.yslot = static_cast<__nv_bfloat16*>(a.yslot);
+  gp.yshared = static_cast<__nv_bfloat16*>(a.yshared);
   gp.h_ready = a.h_ready;
   gp.err = a.err;
   gp.w_down = a.w_down;
@@ -746,6 +791,8 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   }
   gp.T = a.T; gp.d = a.d; gp.E = a.E; gp.k = a.k; gp.I = a.I; gp.Is = a.Is;
   gp.n_max = a.n_max;
+  gp.n_half = ((a.n_max / 2) + 15) & ~15;
+  gp.kbs = a.n_max >= 256 ? 1 : kMaxKBoxes;
   gp.ntiles = (a.T + a.n_max - 1) / a.n_max;
   gp.has_shared = has_shared ? 1 : 0;
 
@@ -756,7 +803,9 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
             make_map(&m.wd, a.w_down, (uint64_t)a.E * a.d, a.I, kTileM) &&
             make_map(&m.xp, a.xperm, (uint64_t)pairs, a.d, (uint32_t)a.n_max) &&
             make_map(&m.x, a.x, (uint64_t)a.T, a.d, (uint32_t)a.n_max) &&
-            make_map(&m.h, a.h, (uint64_t)pairs, a.I, (uint32_t)a.n_max);
+            make_map(&m.h, a.h, (uint64_t)pairs, a.I, (uint32_t)a.n_max) &&
+            make_map(&m.xph, a.xperm, (uint64_t)pairs, a.d, (uint32_t)gp.n_half) &&
+            make_map(&m.hh, a.h, (uint64_t)pairs, a.I, (uint32_t)gp.n_half);
   if (ok && has_shared)
     ok = make_map(&m.sg, a.ws_gate, (uint64_t)a.Is, a.d, 64) &&
          make_map(&m.su, a.ws_up, (uint64_t)a.Is, a.d, 64) &&
@@ -765,7 +814,7 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   if (!has_shared) { m.sg = m.wg; m.su = m.wu; m.sd = m.wd; m.hs = m.h; }
   if (!ok) return cudaErrorInvalidValue;
 
-  const size_t stage_bytes = (size_t)kAStageBytes + (size_t)kKBoxes * a.n_max * 128;
+  const size_t stage_bytes = (size_t)gp.kbs * ((size_t)kATileBytes + (size_t)a.n_max * 128);
   const size_t fixed = experts_fixed_smem();
   const int limit = max_smem_optin();
   int stages = (int)((limit - (int)fixed) / (int)stage_bytes);
@@ -792,17 +841,25 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
 
-  // 3. gate-weighted combine
-  return launch_combine(a, s);
+  // 3. gate-weighted combine of the bf16 rows
+  return launch_combine(a, s, nullptr, 0, nullptr, 0, false, true);
 }
 
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero, int n_zero,
-                           uint32_t* zero2, int n_zero2, bool meta_early) {
-  dim3 cgrid((a.d / 4 + 255) / 256, a.T);
+                           uint32_t* zero2, int n_zero2, bool meta_early, bool rows_bf16) {
+  dim3 cgrid((a.d / kCombineCols + 255) / 256, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
-  cudaError_t e = launch_ex(combine_kernel, cgrid, dim3(256), 0, s, true, a.yslot, a.yshared,
-                            a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero,
-                            zero2, n_zero2, meta_early ? 1 : 0);
+  cudaError_t e =
+      rows_bf16
+          ? launch_ex(combine_kernel<__nv_bfloat16>, cgrid, dim3(256), 0, s, true,
+                      static_cast<const __nv_bfloat16*>(a.yslot),
+                      static_cast<const __nv_bfloat16*>(a.yshared), a.pos, a.topk_gate,
+                      a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero, zero2, n_zero2,
+                      meta_early ? 1 : 0)
+          : launch_ex(combine_kernel<float>, cgrid, dim3(256), 0, s, true,
+                      static_cast<const float*>(a.yslot), static_cast<const float*>(a.yshared),
+                      a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero,
+                      zero2, n_zero2, meta_early ? 1 : 0);
   prof_end(DMOE_KERNEL_COMBINE, s);
   if (e != cudaSuccess) return e;
   return cudaGetLastError();

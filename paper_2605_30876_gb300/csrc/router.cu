@@ -2,10 +2,12 @@
 //
 // Decode-sized batches take the single cluster launch of route_cluster.cu. Larger batches
 // use one kernel per step:
-//   logits                 the logits stage of the cluster launch over 64-token tiles
-//                          (tensor cores, exact bf16 split of W_r), or where its shape rules
-//                          do not hold, router_logits_kernel: fp32 FFMA, 32 x 64 tiles,
-//                          optional split over d
+//   logits                 the split of W_r and tcgen05 tiles of 128 tokens x E experts over
+//                          slices of d (router_logits_tc.cu); where its shape rules do not
+//                          hold, the
+//                          logits stage of the cluster launch over 64-token tiles (mma.sync,
+//                          the same exact split of W_r), else router_logits_kernel (fp32
+//                          FFMA, 32 x 64 tiles, optional split over d)
 //   router_softmax_kernel  one warp per token: sum the partials in split order, + b,
 //                          softmax, top-k
 //   block_route_kernel     one CTA per diffusion block: Algorithm 1 (routing_device.cuh)
@@ -140,10 +142,16 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
     e = launch_route_cluster(a, dsp, tickets, s);
     if (e != cudaSuccess) return e;
   } else {
-    // logits (+ bias) on tensor cores in the cluster launch when the shape allows it, else
-    // the FFMA tiles with partial sums over a split of d
-    const bool cl = route_cluster_logits_ok(a.d, a.E);
-    if (cl) {
+    // logits (+ bias): on tcgen05 when the shape allows it (after the split of W_r), else
+    // on mma.sync in the cluster launch's logits stage, else the FFMA tiles with partial
+    // sums over a split of d; then softmax and top-k
+    const bool tc = a.w_parts != nullptr && a.tc_part != nullptr && a.tc_splits > 0 &&
+                    router_tc_ok(a.T, a.d, a.E);
+    const bool cl = !tc && route_cluster_logits_ok(a.d, a.E);
+    if (tc) {
+      e = launch_router_tc(a, a.tc_splits, s);
+      if (e != cudaSuccess) return e;
+    } else if (cl) {
       e = launch_logits_cluster(a, s);
       if (e != cudaSuccess) return e;
     } else {
@@ -152,9 +160,12 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
       router_logits_kernel<<<g1, 256, 0, s>>>(a.x, a.w_r, a.logits_part, a.T, a.d, a.E, dchunk,
                                               a.shared_pf);
     }
+    // partial sums over slices of d (tc: tc_splits, FFMA: splits, + bias) or one [T, E]
+    // array of logits with the bias in (cl)
     e = launch_ex(router_softmax_kernel, dim3((a.T + 7) / 8), dim3(256), 0, s, true,
-                  a.logits_part, cl ? 1 : a.splits, cl ? nullptr : a.bias, a.probs, a.probs_hat,
-                  a.topk_idx, a.topk_gate, a.T, a.E, a.kb, a.mode);
+                  tc ? a.tc_part : a.logits_part, tc ? a.tc_splits : (cl ? 1 : a.splits),
+                  cl ? nullptr : a.bias,
+                  a.probs, a.probs_hat, a.topk_idx, a.topk_gate, a.T, a.E, a.kb, a.mode);
     if (e != cudaSuccess) return e;
     if (a.mode == DMOE_ROUTE_BLOCK) {
       e = launch_ex(block_route_kernel, dim3(a.n_blocks), dim3(256), 0, s, true, a.probs,

@@ -133,13 +133,22 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
     v[j] = 0.f;
     if (e < E) valid |= 1u << j;
   }
-  // partial rows outermost: the J loads of one row are independent and go out together
-  for (int s = 0; s < nsum; ++s) {
-    float l[J];
+  // partial rows outermost, eight at a time: their 8 J loads go out together; the sum keeps
+  // the row order
+  for (int s0 = 0; s0 < nsum; s0 += 8) {
+    float l[8][J];
 #pragma unroll
-    for (int j = 0; j < J; ++j) l[j] = ((valid >> j) & 1u) ? lrow[(size_t)s * pstride + lane + 32 * j] : 0.f;
+    for (int q = 0; q < 8; ++q)
 #pragma unroll
-    for (int j = 0; j < J; ++j) v[j] += l[j];
+      for (int j = 0; j < J; ++j)
+        l[q][j] = (s0 + q < nsum && ((valid >> j) & 1u))
+                      ? lrow[(size_t)(s0 + q) * pstride + lane + 32 * j]
+                      : 0.f;
+#pragma unroll
+    for (int q = 0; q < 8; ++q)
+      if (s0 + q < nsum)
+#pragma unroll
+        for (int j = 0; j < J; ++j) v[j] += l[q][j];
   }
 #pragma unroll
   for (int j = 0; j < J; ++j) {
@@ -205,19 +214,20 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool live = tid < E;
 
-  // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k); eight rows are
+  // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k); 32 rows are
   // fetched at a time so that their loads overlap
   float S = 0.f;
   if (live) {
-    for (int i0 = 0; i0 < B; i0 += 8) {
-      float h[8];
+    for (int i0 = 0; i0 < B; i0 += 32) {
+      float h[32];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) h[u] = (i0 + u < B) ? hat(i0 + u, tid) : 0.f;
+      for (int u = 0; u < 32; ++u) h[u] = (i0 + u < B) ? hat(i0 + u, tid) : 0.f;
 #pragma unroll
-      for (int u = 0; u < 8; ++u)
+      for (int u = 0; u < 32; ++u)
         if (i0 + u < B) S += h[u];
     }
   }
+  DMOE_STAMP(22);
   if (top_p <= 0.f) {
     // p <= 0 (block top-k): Top-P stops at the first entry and the floor extends the coreset
     // to the k best. S~ = S / sum(S) has the order of S (exactly so, where the fp32 division
@@ -369,30 +379,43 @@ template <class ProbFn, class OutFn>
 __device__ inline void mask_topk_warps(int k, int B, int size, const int* order, ProbFn prob,
                                        OutFn out) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = (int)(blockDim.x >> 5);
   if (size <= 32) {
-    // one member per lane: k rounds of a tournament (larger score, ties to the lower id)
+    // one member per lane: k rounds of a tournament (larger score, ties to the lower id);
+    // the scores of up to eight of the warp's tokens are loaded before the first tournament
     const int e = lane < size ? order[lane] : -1;
-    for (int i = warp; i < B; i += (int)(blockDim.x >> 5)) {
-      uint32_t key = e >= 0 ? order_key(prob(i, e)) : 0u;
-      int my_e = -1;
-      float my_v = 0.f;
-      for (int r = 0; r < k; ++r) {
-        const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
-        const uint32_t imin =
-            __reduce_min_sync(0xffffffffu, key == kmax ? (uint32_t)e : 0xffffffffu);
-        if (lane == r) {
-          my_e = (int)imin;
-          my_v = key_value(kmax);
-        }
-        if (key == kmax && (uint32_t)e == imin) key = 0u;
+    for (int i0 = warp; i0 < B; i0 += 8 * nw) {
+      uint32_t keys[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = i0 + u * nw;
+        keys[u] = (i < B && e >= 0) ? order_key(prob(i, e)) : 0u;
       }
-      float g = 0.f;
-      for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
-      if (lane < k) out(i, lane, my_e, my_v / g);
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int i = i0 + u * nw;
+        if (i >= B) break;   // the same for the whole warp
+        uint32_t key = keys[u];
+        int my_e = -1;
+        float my_v = 0.f;
+        for (int r = 0; r < k; ++r) {
+          const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
+          const uint32_t imin =
+              __reduce_min_sync(0xffffffffu, key == kmax ? (uint32_t)e : 0xffffffffu);
+          if (lane == r) {
+            my_e = (int)imin;
+            my_v = key_value(kmax);
+          }
+          if (key == kmax && (uint32_t)e == imin) key = 0u;
+        }
+        float g = 0.f;
+        for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
+        if (lane < k) out(i, lane, my_e, my_v / g);
+      }
     }
     return;
   }
-  for (int i = warp; i < B; i += (int)(blockDim.x >> 5)) {
+  for (int i = warp; i < B; i += nw) {
     float cv[8];
     int ce[8];
     uint32_t valid = 0;
@@ -413,55 +436,6 @@ __device__ inline void mask_topk_warps(int k, int B, int size, const int* order,
     float g = 0.f;
     for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
     if (lane < k) out(i, lane, my_e, my_v / g);
-  }
-}
-
-// The same result for a coreset of at most 32 experts with every (token, member) pair in
-// parallel: a member's rank among its token's members is the number of members that beat it
-// (larger score, or equal score and lower id); ranks below k are the selection. `sv` is a
-// shared [B][32] buffer, `sel_e`/`sel_v` shared [B][kMaxTopK] buffers.
-template <class ProbFn, class OutFn>
-__device__ inline void mask_topk_small(int k, int B, int size, const int* order, ProbFn prob,
-                                       OutFn out, float* sv, int* sel_e, float* sel_v) {
-  const int tid = threadIdx.x, nthr = blockDim.x;
-  const int n = B * size;
-  for (int p0 = tid; p0 < n; p0 += 8 * nthr) {  // eight gathers in flight per thread
-    float v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int pidx = p0 + u * nthr;
-      v[u] = pidx < n ? prob(pidx / size, order[pidx % size]) : 0.f;
-    }
-#pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int pidx = p0 + u * nthr;
-      if (pidx < n) sv[(pidx / size) * 32 + pidx % size] = v[u];
-    }
-  }
-  __syncthreads();
-  DMOE_STAMP(23);
-  for (int pidx = tid; pidx < n; pidx += nthr) {
-    const int i = pidx / size, c = pidx % size;
-    const float* row = sv + i * 32;
-    const float v = row[c];
-    const int e = order[c];
-    int rank = 0;
-    for (int c2 = 0; c2 < size; ++c2) {
-      const float w = row[c2];
-      rank += (w > v || (w == v && order[c2] < e)) ? 1 : 0;
-    }
-    if (rank < k) {
-      sel_e[i * kMaxTopK + rank] = e;
-      sel_v[i * kMaxTopK + rank] = v;
-    }
-  }
-  __syncthreads();
-  DMOE_STAMP(24);
-  for (int pidx = tid; pidx < B * k; pidx += nthr) {
-    const int i = pidx / k, r = pidx % k;
-    float g = 0.f;
-    for (int r2 = 0; r2 < k; ++r2) g += sel_v[i * kMaxTopK + r2];
-    out(i, r, sel_e[i * kMaxTopK + r], sel_v[i * kMaxTopK + r] / g);
   }
 }
 

@@ -108,7 +108,8 @@ def test_null_and_misaligned_pointers_are_rejected_before_launch(dm):
 def test_layer_forward_launch_count(dm):
     # decode-size forward: one routing launch (dispatch fused), the expert launch, the combine
     assert dm.dmoe_layer_forward_launches(_desc(dm)) == 3
-    # 2048 tokens: logits, softmax / top-k, Algorithm 1, dispatch; gather, experts, combine
-    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64)) == 7
-    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64, mode=dm.DMOE_ROUTE_TOKEN)) == 6
+    # 2048 tokens: split of W_r, logits, softmax / top-k, Algorithm 1, dispatch (count,
+    # place); gather, experts, combine
+    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64)) == 9
+    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64, mode=dm.DMOE_ROUTE_TOKEN)) == 8
     assert dm.dmoe_layer_forward_launches(_desc(dm, top_k=0)) == -1
