@@ -121,7 +121,7 @@ dispatch_place_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
     ids[j] = p < np ? __ldcg(topk_idx + t0 * k + p) : 0;
   }
   pdl_wait();
-  KLOG(DMOE_KERNEL_DISPATCH, 0);
+  KLOG(7, 0);
   for (int e = tid; e < E; e += kDispThreads) {
     bits[e] = gbits[(size_t)c * E + e];
     base[e] = gbase[(size_t)c * E + e] + goff[e];
@@ -139,7 +139,7 @@ dispatch_place_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
       pos[i] = r;
     }
   }
-  KLOG(DMOE_KERNEL_DISPATCH, 1);
+  KLOG(7, 1);
 }
 
 }  // namespace

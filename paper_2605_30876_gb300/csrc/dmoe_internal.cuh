@@ -214,7 +214,7 @@ cudaError_t launch_logits_cluster(const RouterArgs& a, cudaStream_t s);
 // The logits of a large forward on tcgen05 (router_logits_tc.cu): the split of W_r into
 // a.w_parts, then the products over `splits` slices of d into a.tc_part [splits, T, E]
 // (router_softmax_kernel adds them in order, with the bias). Needs T >= 128, d % 64 == 0,
-// E % 16 == 0; router_tc_splits gives the split.
+// E % 32 == 0; router_tc_splits gives the split.
 bool router_tc_ok(int T, int d, int E);
 int router_tc_splits(int T, int d);
 size_t router_tc_parts_bytes(int d, int E);

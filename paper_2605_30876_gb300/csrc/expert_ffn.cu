@@ -19,9 +19,9 @@
 //   combine_kernel      y_t = sum over slots (slot order) of g_tj * row + shared -> bf16
 //
 // A group is one unique expert (dispatch order) or the shared expert (all T tokens). The
-// expert kernel is warp-specialised: warp 0 issues TMA, warp 1 issues MMAs, warps 2-5 run
-// the epilogue; each pipeline stage carries K = 128 (two 128-B-wide boxes per operand), the
-// access shape that keeps per-SM TMA streaming near its peak. The unit list is derived on
+// expert kernel is warp-specialised: warp 0 issues TMA, warp 1 issues MMAs, warps 2-9 run
+// the epilogue; each pipeline stage carries K = 128 (two 128-B-wide boxes per operand; 64
+// for 256-row token tiles). The unit list is derived on
 // the device from the dispatch output, so no host round-trip is needed. Consecutive
 // kernels are chained with programmatic dependent launch: each kernel's set-up (barriers,
 // TMEM, tensor-map prefetch) overlaps the previous kernel, and griddepcontrol.wait orders
@@ -37,19 +37,21 @@
 namespace dmoe {
 namespace {
 
-constexpr int kThreads = 192;                      // 6 warps
+constexpr int kThreads = 320;                      // 10 warps
+constexpr int kEpiThreads = 256;                   // warps 2-9: the epilogue
 constexpr int kBoxBytes = 64 * 128;                // one TMA box: 64 rows x 128 B
 constexpr int kMaxKBoxes = 2;                      // K boxes per stage: 1 or 2 (K = 64, 128)
 constexpr int kATileBytes = kTileM * 128;          // 16 KB: 128 rows x 64 K (one K box)
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr int kMaxStages = 8;
-constexpr int kXchgStride = 17;                    // floats per row of the exchange buffer
+constexpr int kXchgStride = 17;                    // floats per row of the exchange buffers
 
 struct GemmParams {
   const int32_t* n_unique;
   const int32_t* unique_ids;
   const int32_t* offsets;
+  const int32_t* rows;    // dispatch rows: t * k + slot (the x row of a routed token row)
   __nv_bfloat16* h;       // [T*k, I]
   __nv_bfloat16* hs;      // [T, Is]
   __nv_bfloat16* yslot;   // [T*k, d] bf16 (the combine sums them in fp32)
@@ -77,13 +79,27 @@ struct Maps {
   CUtensorMap xph, hh;          // xperm and H with half-height boxes (small token tiles)
 };
 
-using ptx::epi_all;
 using ptx::fence_proxy_async_global;
 using ptx::ld_acquire;
 using ptx::named_bar_sync;
 using ptx::red_release_add;
 
 __device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
+
+// AND of `v` over the kEpiThreads epilogue threads (named barrier 1), so that they take the
+// warp-collective TMEM loads, or leave the unit loop, together
+__device__ __forceinline__ bool epi_all_threads(bool v) {
+  uint32_t r;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 p, %1, 0;\n\t"
+      "bar.red.and.pred q, 1, %2, p;\n\t"
+      "selp.u32 %0, 1, 0, q;\n\t}"
+      : "=r"(r)
+      : "r"((uint32_t)v), "n"(kEpiThreads)
+      : "memory");
+  return r != 0;
+}
 
 // Debug builds (-DDMOE_TRACE) record a per-CTA timeline of the expert kernel: slot 0 entry,
 // 1 after the unit list, 62 exit; for the i-th unit of the CTA (i < 8), at 2 + 6i: unit id,
@@ -120,7 +136,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   const uint32_t off_a = 0;
   const uint32_t off_b = off_a + (uint32_t)stages * a_stage;
   const uint32_t off_x = off_b + (uint32_t)stages * b_stage;
-  const uint32_t x_bytes = 2u * 64u * kXchgStride * 4u;        // [128][17] fp32
+  const uint32_t x_bytes = 2u * 128u * kXchgStride * 4u;       // 2 x [128][17] fp32
   const uint32_t off_bar = (off_x + x_bytes + 7u) & ~7u;
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + off_bar);
   uint64_t* empty = full + stages;
@@ -149,7 +165,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     }
     for (int a = 0; a < 4; ++a) {
       ptx::mbar_init(&acc_full[a], 1);
-      ptx::mbar_init(&acc_empty[a], 128);
+      ptx::mbar_init(&acc_empty[a], kEpiThreads);
     }
     ptx::mbar_init(drain, 1);
     ptx::fence_mbarrier_init();
@@ -470,9 +486,15 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       }
     }
   } else {
-    // ================= epilogue: warps 2..5, TMEM lanes 32*(warp%4) ..
+    // ================= epilogue: warps 2..9, TMEM lanes 32*(warp%4) ..; two column groups
+    // (warps 2-5 and 6-9) take alternate 16-column slices of the accumulator, each with its
+    // own exchange tile and named barrier (the epilogue math is latency-bound: two groups
+    // finish a tile in about half the time)
     const int q = warp & 3;
+    const int cg = (warp - 2) >> 2;                 // column group
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+    float* xg = xchg + cg * (128 * kXchgStride);    // this group's exchange tile
+    const int gbar = 2 + cg;                        // this group's named barrier
     int acc = 0, li = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++li) {
@@ -480,7 +502,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       const bool shared = un.g >= U;
       const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
       const int n_mma = (nvalid + 15) & ~15;
-      if (!epi_all(wait(&acc_full[acc], acc_phase, u))) break;
+      if (!epi_all_threads(wait(&acc_full[acc], acc_phase, u))) break;
       ptx::tc_fence_after();
       if (tid == 64 && li < 8) DMOE_TRACE_AT(50 + li);
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)acc * (uint32_t)p.n_max;
@@ -493,26 +515,26 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         __nv_bfloat16* hout = shared ? p.hs : p.h;
         const int hrow0 = (shared ? 0 : g_row0[un.g]) + col0;
         // per 16-token slice: every accumulator row's 16 values go to the exchange tile
-        // (gate rows 0-63, up rows 64-127), then each of the 128 threads takes 8 adjacent
-        // H columns of one token (loads, SwiGLU, one 16-byte store). Interleaving the
-        // exchange loads with the H stores instead serialises them: the compiler cannot
-        // tell the two memories apart.
-        const int et = tid - 64, xc = et >> 3, hc = (et & 7) * 8;
-        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+        // (gate rows 0-63, up rows 64-127), then each of the group's 128 threads takes 8
+        // adjacent H columns of one token (loads, SwiGLU, one 16-byte store). Interleaving
+        // the exchange loads with the H stores instead serialises them: the compiler
+        // cannot tell the two memories apart.
+        const int et = tid - 64 - 128 * cg, xc = et >> 3, hc = (et & 7) * 8;
+        for (int c0 = 16 * cg; c0 < n_mma; c0 += 32) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
           ptx::tmem_ld_wait();
           {
-            float* xr = xchg + ((is_gate ? 0 : 64) + r64) * kXchgStride;
+            float* xr = xg + ((is_gate ? 0 : 64) + r64) * kXchgStride;
 #pragma unroll
             for (int c = 0; c < 16; ++c) xr[c] = v[c];
           }
-          named_bar_sync(2, 128);
+          named_bar_sync(gbar, 128);
           float gv[8], uv[8];
 #pragma unroll
           for (int j = 0; j < 8; ++j) {
-            gv[j] = xchg[(hc + j) * kXchgStride + xc];
-            uv[j] = xchg[(64 + hc + j) * kXchgStride + xc];
+            gv[j] = xg[(hc + j) * kXchgStride + xc];
+            uv[j] = xg[(64 + hc + j) * kXchgStride + xc];
           }
           uint32_t hp[4];
 #pragma unroll
@@ -524,21 +546,21 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           if (c0 + xc < nvalid)
             *reinterpret_cast<uint4*>(hout + (size_t)(hrow0 + c0 + xc) * Ig + un.m * 64 + hc) =
                 make_uint4(hp[0], hp[1], hp[2], hp[3]);
-          named_bar_sync(2, 128);   // the exchange tile is rewritten by the next slice
+          named_bar_sync(gbar, 128);   // the exchange tile is rewritten by the next slice
         }
         if (tid == 64 && li < 4) DMOE_TRACE_AT(54 + li);
         ptx::tc_fence_before();
         ptx::mbar_arrive(&acc_empty[acc]);
         // publish the tile: the barrier orders every epilogue thread's H stores before one
         // release add; a reader acquires the counter, then fences the async proxy
-        named_bar_sync(2, 128);
+        named_bar_sync(4, kEpiThreads);
         if (tid == 64 && li < 8) DMOE_TRACE_AT(58 + (li < 4 ? li : 3));
         if (tid == 64) red_release_add(p.h_ready + un.g * p.ntiles + un.n, 1);
       } else {
         const int drow = un.m * kTileM + q * 32 + lane;
         __nv_bfloat16* out = shared ? p.yshared + (size_t)col0 * p.d
                                     : p.yslot + (size_t)(g_row0[un.g] + col0) * p.d;
-        for (int c0 = 0; c0 < n_mma; c0 += 16) {
+        for (int c0 = 16 * cg; c0 < n_mma; c0 += 32) {
           float v[16];
           ptx::tmem_ld16(tbase + c0, v);
           ptx::tmem_ld_wait();
@@ -565,11 +587,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   }
 }
 
-// xperm[r, :] = x[rows[r] / k, :]; block 0 also clears the gate/up tile counters. A CTA
-// copies kGatherRows consecutive rows at a time (so that the rows being written at any
-// moment form one contiguous range of xperm): their indices are read in one round, then
-// every thread has one 16-byte piece of each row in flight.
-constexpr int kGatherRows = 8;
+// xperm[r, :] = x[rows[r] / k, :]; block 0 also clears the gate/up tile counters.
 __global__ void __launch_bounds__(256)
 gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ rows,
               __nv_bfloat16* __restrict__ xperm, int32_t* __restrict__ h_ready, int n_ready,
@@ -580,44 +598,46 @@ gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ r
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_ready; i += blockDim.x) h_ready[i] = 0;
   const int vec = d / 8;  // uint4 per row
-  for (int r0 = blockIdx.x * kGatherRows; r0 < pairs; r0 += gridDim.x * kGatherRows) {
-    const uint4* src[kGatherRows];
-#pragma unroll
-    for (int j = 0; j < kGatherRows; ++j)
-      src[j] = reinterpret_cast<const uint4*>(
-          x + (size_t)(r0 + j < pairs ? rows[r0 + j] / k : 0) * d);
-    uint4* dst = reinterpret_cast<uint4*>(xperm + (size_t)r0 * d);
-    for (int i = threadIdx.x; i < vec; i += blockDim.x) {
-      uint4 v[kGatherRows];
-#pragma unroll
-      for (int j = 0; j < kGatherRows; ++j)
-        if (r0 + j < pairs) v[j] = src[j][i];
-#pragma unroll
-      for (int j = 0; j < kGatherRows; ++j)
-        if (r0 + j < pairs) dst[(size_t)j * vec + i] = v[j];
-    }
+  for (int r = blockIdx.x; r < pairs; r += gridDim.x) {
+    const int t = rows[r] / k;
+    const uint4* src = reinterpret_cast<const uint4*>(x + (size_t)t * d);
+    uint4* dst = reinterpret_cast<uint4*>(xperm + (size_t)r * d);
+    for (int i = threadIdx.x; i < vec; i += blockDim.x) dst[i] = src[i];
   }
   KLOG(DMOE_KERNEL_GATHER, 1);
 }
 
-// kCombineCols consecutive row values as fp32 (fp32 rows of the decode-size path, bf16
-// rows of the general path): one 16-byte load per 8 bf16 or 4 fp32 values.
+// kCombineCols consecutive row values: the raw 16-byte pieces (one for 8 bf16, two for 8
+// fp32), loaded first and converted to fp32 as they are used (registers bound the CTAs per
+// SM, and with them the loads in flight).
 constexpr int kCombineCols = 8;
-__device__ __forceinline__ void load8(const float* src, float (&v)[8]) {
-  const float4 a = *reinterpret_cast<const float4*>(src);
-  const float4 b = *reinterpret_cast<const float4*>(src + 4);
-  v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w; v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-}
-__device__ __forceinline__ void load8(const __nv_bfloat16* src, float (&v)[8]) {
-  const uint4 u = *reinterpret_cast<const uint4*>(src);
-  const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
-    v[2 * i] = f.x;
-    v[2 * i + 1] = f.y;
+template <typename Row> struct Raw8;
+template <> struct Raw8<__nv_bfloat16> {
+  uint4 a;
+  __device__ __forceinline__ void load(const __nv_bfloat16* src) {
+    a = *reinterpret_cast<const uint4*>(src);
   }
-}
+  __device__ __forceinline__ void unpack(float (&v)[8]) const {
+    const uint32_t w[4] = {a.x, a.y, a.z, a.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+      v[2 * i] = f.x;
+      v[2 * i + 1] = f.y;
+    }
+  }
+};
+template <> struct Raw8<float> {
+  float4 a, b;
+  __device__ __forceinline__ void load(const float* src) {
+    a = *reinterpret_cast<const float4*>(src);
+    b = *reinterpret_cast<const float4*>(src + 4);
+  }
+  __device__ __forceinline__ void unpack(float (&v)[8]) const {
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+};
 
 // y[t, :] = bf16( sum_j g[t,j] * yslot[pos[t*k + j], :] (slot order) + yshared[t, :] );
 // block (0, 0) also clears `zero[0 .. n_zero)` and `zero2[0 .. n_zero2)` (counters and
@@ -634,16 +654,18 @@ combine_kernel(const Row* __restrict__ yslot, const Row* __restrict__ yshared,
   pdl_launch_dependents();
   const int t = blockIdx.y;
   const int c = (blockIdx.x * blockDim.x + threadIdx.x) * kCombineCols;
-  int r[kMaxTopK];
-  float gj[kMaxTopK];
-  if (meta_early) {
+  // the slot indices and gates, eight slots at a time
+  int r[8];
+  float gj[8];
+  auto load_meta = [&](int j0) {
 #pragma unroll
-    for (int j = 0; j < kMaxTopK; ++j)
-      if (j < k) {
-        r[j] = __ldcg(pos + t * k + j);
-        gj[j] = __ldcg(gate + t * k + j);
+    for (int j = 0; j < 8; ++j)
+      if (j0 + j < k) {
+        r[j] = __ldcg(pos + t * k + j0 + j);
+        gj[j] = __ldcg(gate + t * k + j0 + j);
       }
-  }
+  };
+  if (meta_early) load_meta(0);
   pdl_wait();
   KLOG(DMOE_KERNEL_COMBINE, 0);
   if (blockIdx.x == 0 && blockIdx.y == 0) {
@@ -651,32 +673,34 @@ combine_kernel(const Row* __restrict__ yslot, const Row* __restrict__ yshared,
     for (int i = threadIdx.x; i < n_zero2; i += blockDim.x) zero2[i] = 0u;
   }
   if (c >= d) return;
-  if (!meta_early) {
-#pragma unroll
-    for (int j = 0; j < kMaxTopK; ++j)
-      if (j < k) {
-        r[j] = pos[t * k + j];
-        gj[j] = gate[t * k + j];
-      }
-  }
-  // every row load is issued before the first product; the sum keeps the slot order
-  float v[kMaxTopK][kCombineCols];
-#pragma unroll
-  for (int j = 0; j < kMaxTopK; ++j)
-    if (j < k) load8(yslot + (size_t)r[j] * d + c, v[j]);
-  float vs[kCombineCols];
-  if (has_shared) load8(yshared + (size_t)t * d + c, vs);
+  // eight slots at a time: their row loads (and the shared row's) are issued before the
+  // first product; the sum keeps the slot order
   float acc[kCombineCols];
 #pragma unroll
   for (int i = 0; i < kCombineCols; ++i) acc[i] = 0.f;
+  Raw8<Row> raw_s;
+  if (has_shared) raw_s.load(yshared + (size_t)t * d + c);
+  for (int j0 = 0; j0 < k; j0 += 8) {
+    if (!meta_early || j0 > 0) load_meta(j0);
+    Raw8<Row> raw[8];
 #pragma unroll
-  for (int j = 0; j < kMaxTopK; ++j)
-    if (j < k)
+    for (int j = 0; j < 8; ++j)
+      if (j0 + j < k) raw[j].load(yslot + (size_t)r[j] * d + c);
 #pragma unroll
-      for (int i = 0; i < kCombineCols; ++i) acc[i] = fmaf(gj[j], v[j][i], acc[i]);
-  if (has_shared)
+    for (int j = 0; j < 8; ++j)
+      if (j0 + j < k) {
+        float v[kCombineCols];
+        raw[j].unpack(v);
+#pragma unroll
+        for (int i = 0; i < kCombineCols; ++i) acc[i] = fmaf(gj[j], v[i], acc[i]);
+      }
+  }
+  if (has_shared) {
+    float vs[kCombineCols];
+    raw_s.unpack(vs);
 #pragma unroll
     for (int i = 0; i < kCombineCols; ++i) acc[i] += vs[i];
+  }
   uint32_t out[kCombineCols / 2];
 #pragma unroll
   for (int i = 0; i < kCombineCols / 2; ++i) {
@@ -728,7 +752,7 @@ uint32_t pow2_cols(uint32_t c) {
 
 size_t experts_fixed_smem() {
   // alignment slack + exchange buffers + barriers + misc/group arrays
-  return 1024 + 2 * 64 * kXchgStride * 4 + 8 + 8 * (2 * kMaxStages + 9) +
+  return 1024 + 2 * 128 * kXchgStride * 4 + 8 + 8 * (2 * kMaxStages + 9) +
          sizeof(int) * (8 + 5 * (kMaxGroups + 1)) + 64;
 }
 
@@ -763,10 +787,7 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   const int n_ready = experts_ready_counters(a.T, a.E, a.n_max);
   // 1. gather x in dispatch order; clear the gate/up tile counters
   {
-    const int want = (pairs + kGatherRows - 1) / kGatherRows;
-    const int cap = device_sm_count() * 8;
-    int grid = want < cap ? want : cap;
-    if (grid < 1) grid = 1;
+    const int grid = pairs < 1024 ? pairs : 1024;
     prof_begin(DMOE_KERNEL_GATHER, s);
     cudaError_t e = launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, true, a.x, a.rows,
                               a.xperm, a.h_ready, n_ready, pairs, a.k, a.d);

@@ -15,14 +15,15 @@
 //   router_wsplit_kernel      the three parts of W_r, each stored K-major ([E, d] bf16: row
 //                             e holds expert e's weights over d), the MMA's B operand
 //   router_logits_tc_kernel   one CTA per (128 tokens, slice of d), all E experts (N = E,
-//                             at most 256), no cross-CTA step:
+//                             a multiple of 32, at most 256), no cross-CTA step:
 //     warp 0     TMA, two stages: x chunk (128 tokens x 64 of d, 128-B swizzle, rows past
 //                T read as zero) and the three parts' chunks (E rows x 64)
 //     warp 1     TMEM allocation; lane 0 issues D[128 x E] += x * part^T, 4 K-steps of 16
 //                per chunk and part (hi into one accumulator, mid and lo into the other)
 //     warps 0-3  (after the MMAs; one TMEM lane quadrant each) put hi + (mid + lo) into
-//                shared memory (the stages are free by then), then store the tile's
-//                partial rows, one row per warp at a time (1 KB at E = 256, coalesced)
+//                shared memory (the stages are free by then) as E / 32 boxes of 32
+//                experts x 128 tokens with the 128-B swizzle, which thread 0 then stores by
+//                TMA (rows past T are not written)
 // Every mbarrier wait is bounded (1 s): a timeout is recorded and the CTA unwinds.
 #include "dmoe_internal.cuh"
 #include "sm100_ptx.cuh"
@@ -30,7 +31,8 @@
 
 // Debug builds (-DDMOE_TRACE): per-CTA phase times of router_logits_tc_kernel (%globaltimer,
 // ns), g_rtc[cta * 16 + slot]: 0 entry, 1 set-up done, 2 last TMA issued, 3 first stage
-// landed, 4 last MMA issued, 5 accumulator ready, 6 rows stored.
+// landed, 4 last MMA issued, 5 accumulator ready, 7 rows staged in shared memory, 6 rows
+// stored.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_rtc[1024 * 16];
 #define RTC_AT(slot) \
@@ -52,7 +54,7 @@ constexpr uint64_t kLtTimeoutNs = 1000000000ull;
 struct LtArgs {
   CUtensorMap xmap;   // x [T, d] bf16, box 64 columns x 128 rows, 128-B swizzle
   CUtensorMap pmap;   // parts [3E, d] bf16, box 64 columns x E rows, 128-B swizzle
-  float* part;        // [S, T, E] partial logits
+  CUtensorMap omap;   // partials [S, T, E] fp32, box 32 x 128 x 1, 128-B swizzle
   DevErrRecord* err;
   L2Prefetch shared_pf;
   int T, d, E, ds;    // ds: d per slice (blockIdx.y)
@@ -68,6 +70,7 @@ router_wsplit_kernel(const float* __restrict__ w_r, __nv_bfloat16* __restrict__ 
   // the previous launch on the stream may still read the parts of the call before
   pdl_wait();
   pdl_launch_dependents();
+  KLOG(8, 0);
   if (e >= E) return;
   float w[8];
 #pragma unroll
@@ -90,6 +93,7 @@ router_wsplit_kernel(const float* __restrict__ w_r, __nv_bfloat16* __restrict__ 
   *reinterpret_cast<uint4*>(parts + o) = make_uint4(hp[0], hp[1], hp[2], hp[3]);
   *reinterpret_cast<uint4*>(parts + pe + o) = make_uint4(mp[0], mp[1], mp[2], mp[3]);
   *reinterpret_cast<uint4*>(parts + 2 * pe + o) = make_uint4(lp[0], lp[1], lp[2], lp[3]);
+  KLOG(8, 1);
 }
 
 __global__ void __launch_bounds__(kLtThreads, 1)
@@ -199,31 +203,32 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
   ptx::tc_fence_after();
   if (tid == 0) RTC_AT(5);
   {
-    // rows of E + 4 floats: the float4 writes of a warp's 32 rows spread over the banks
-    const int rs = E + 4;
-    float* tile = reinterpret_cast<float*>(smem);
+    // box b (experts 32b .. 32b + 31) at b * 16 KB: row r = token, 16-byte chunk j of the row
+    // at j xor (r mod 8); the eight rows of a lane group hit eight different chunks
+    uint8_t* boxes = smem;
     const int r = warp * 32 + lane;
     const uint32_t lanes = (uint32_t)(warp * 32) << 16;
-    for (int c0 = 0; c0 < E; c0 += 16) {
-      float h[16], ml[16];
-      ptx::tmem_ld16(tmem + lanes + (uint32_t)c0, h);
-      ptx::tmem_ld16(tmem + lanes + t_ml + (uint32_t)c0, ml);
+    for (int c0 = 0; c0 < E; c0 += 32) {
+      float h[32], ml[32];
+      ptx::tmem_ld32(tmem + lanes + (uint32_t)c0, h);
+      ptx::tmem_ld32(tmem + lanes + t_ml + (uint32_t)c0, ml);
       ptx::tmem_ld_wait();
+      uint8_t* row = boxes + (c0 / 32) * (kLtM * 128) + r * 128;
 #pragma unroll
-      for (int j = 0; j < 16; j += 4)
-        *reinterpret_cast<float4*>(tile + (size_t)r * rs + c0 + j) =
-            make_float4(h[j] + ml[j], h[j + 1] + ml[j + 1], h[j + 2] + ml[j + 2],
-                        h[j + 3] + ml[j + 3]);
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<float4*>(row + ((j ^ (r & 7)) << 4)) =
+            make_float4(h[4 * j] + ml[4 * j], h[4 * j + 1] + ml[4 * j + 1],
+                        h[4 * j + 2] + ml[4 * j + 2], h[4 * j + 3] + ml[4 * j + 3]);
     }
+    ptx::fence_proxy_async_smem();   // the boxes are read by the TMA store
+    if (tid == 0) RTC_AT(7);
     __syncthreads();
-    const int nrow = f.T - m0 < kLtM ? f.T - m0 : kLtM;
-    if (have_acc)
-      for (int rr = warp; rr < nrow; rr += kLtThreads / 32) {
-        float* dst = f.part + ((size_t)blockIdx.y * f.T + m0 + rr) * E;
-        for (int c = lane * 4; c < E; c += 128)
-          *reinterpret_cast<float4*>(dst + c) =
-              *reinterpret_cast<const float4*>(tile + (size_t)rr * rs + c);
-      }
+    if (tid == 0) {
+      if (have_acc)
+        for (int b = 0; b < E / 32; ++b)
+          ptx::tma_store_3d(&f.omap, boxes + b * (kLtM * 128), 32 * b, m0, (int)blockIdx.y);
+      ptx::bulk_commit_wait_read();   // the shared memory stays until the stores read it
+    }
   }
   ptx::tc_fence_before();
   __syncthreads();
@@ -267,10 +272,21 @@ bool encode_bf16_2d(EncodeFn enc, CUtensorMap* m, const void* base, uint64_t row
 
 size_t lt_smem_bytes(int E) { return 2 * ((size_t)kLtXBytes + 3 * (size_t)E * 128) + 1024; }
 
+bool encode_part_3d(EncodeFn enc, CUtensorMap* m, float* base, int S, int T, int E) {
+  const cuuint64_t dims[3] = {(cuuint64_t)E, (cuuint64_t)T, (cuuint64_t)S};
+  const cuuint64_t strides[2] = {(cuuint64_t)E * 4, (cuuint64_t)T * E * 4};
+  const cuuint32_t box[3] = {32u, (cuuint32_t)kLtM, 1u};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_128B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+         CUDA_SUCCESS;
+}
+
 }  // namespace
 
 bool router_tc_ok(int T, int d, int E) {
-  return T >= kLtM && d % kLtKC == 0 && E % 16 == 0 && E >= 16 && E <= kMaxExperts;
+  return T >= kLtM && d % kLtKC == 0 && E % 32 == 0 && E <= kMaxExperts;
 }
 
 // Slices of d: each CTA takes at most 256 of d; of the splits that divide d into whole
@@ -302,9 +318,9 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
   if (enc == nullptr) return cudaErrorInvalidValue;
   LtArgs f{};
   if (!encode_bf16_2d(enc, &f.xmap, a.x, (uint64_t)a.T, (uint64_t)a.d, kLtM) ||
-      !encode_bf16_2d(enc, &f.pmap, a.w_parts, 3 * (uint64_t)a.E, (uint64_t)a.d, (uint32_t)a.E))
+      !encode_bf16_2d(enc, &f.pmap, a.w_parts, 3 * (uint64_t)a.E, (uint64_t)a.d, (uint32_t)a.E) ||
+      !encode_part_3d(enc, &f.omap, a.tc_part, splits, a.T, a.E))
     return cudaErrorInvalidValue;
-  f.part = a.tc_part;
   f.err = a.err;
   f.shared_pf = a.shared_pf;
   f.T = a.T;
@@ -330,6 +346,7 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
 }  // namespace dmoe
 
 #ifdef DMOE_TRACE
+DMOE_KLOG_EXPORT(dmoe_debug_klog_routertc)
 extern "C" int dmoe_debug_rtc(void* host) {
   return (int)cudaMemcpyFromSymbol(host, g_rtc, sizeof(g_rtc));
 }

@@ -64,11 +64,11 @@ SHAPES = {
 
 
 def _same_logits_path(shape) -> bool:
-    """dmoe_router computes the logits of 128 or more tokens (d % 64 == 0, E % 16 == 0) on
+    """dmoe_router computes the logits of 128 or more tokens (d % 64 == 0, E % 32 == 0) on
     tcgen05 from a split of W_r kept in its workspace; the no-alloc call has no room for that
     split and keeps the mma.sync logits, so the two differ there by rounding order only."""
     T = shape.n_blocks * shape.block_size
-    tc = T >= 128 and shape.d_model % 64 == 0 and shape.n_experts % 16 == 0
+    tc = T >= 128 and shape.d_model % 64 == 0 and shape.n_experts % 32 == 0
     return not tc
 
 
