@@ -13,6 +13,23 @@
 #include "dmoe_internal.cuh"
 #include "trace_log.cuh"
 
+// Debug builds (-DDMOE_TRACE): phase times of dispatch_count_kernel (%globaltimer, ns),
+// g_dtr[cta * 16 + slot]: 0 entry, 1 ids loaded, 2 bitmap built, 3 bitmap stored, 4 ticket
+// taken; the last CTA: 5 prefix over the chunks, 6 scans, 7 outputs written.
+#ifdef DMOE_TRACE
+__device__ uint64_t g_dtr[1024 * 16];
+#define DTR_AT(slot)                                                                      \
+  do {                                                                                    \
+    if (threadIdx.x == 0) {                                                               \
+      uint64_t t_;                                                                        \
+      asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                             \
+      g_dtr[(blockIdx.x % 1024) * 16 + (slot)] = t_;                                      \
+    }                                                                                     \
+  } while (0)
+#else
+#define DTR_AT(slot) ((void)0)
+#endif
+
 namespace dmoe {
 namespace {
 
@@ -35,6 +52,7 @@ dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
   pdl_wait();
   pdl_launch_dependents();
   KLOG(DMOE_KERNEL_DISPATCH, 0);
+  DTR_AT(0);
   int ids[kDispPerThread];
 #pragma unroll
   for (int j = 0; j < kDispPerThread; ++j) {
@@ -43,6 +61,7 @@ dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
   }
   for (int e = tid; e < E; e += kDispThreads) bits[e] = 0u;
   __syncthreads();
+  DTR_AT(1);
 #pragma unroll
   for (int j = 0; j < kDispPerThread; ++j) {
     const int p = tid + j * kDispThreads;
@@ -56,14 +75,17 @@ dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
     if (atomicOr(&bits[e], bit) & bit) record_error(err, kErrDupExpert, kAtDispatch, i);
   }
   __syncthreads();
+  DTR_AT(2);
   for (int e = tid; e < E; e += kDispThreads) gbits[(size_t)c * E + e] = bits[e];
   // the last CTA to get here sees every chunk's bitmap
   __syncthreads();
+  DTR_AT(3);
   if (tid == 0) {
     __threadfence();
     s_last = atomicAdd(ticket, 1) == nchunks - 1 ? 1 : 0;
   }
   __syncthreads();
+  DTR_AT(4);
   if (!s_last) return;
   __threadfence();
   int cnt = 0;
@@ -81,10 +103,12 @@ dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
         }
     }
   }
+  DTR_AT(5);
   int total_pairs = 0, n_u = 0;
   const int off = block_exclusive_scan_i(tid < E ? cnt : 0, iscr, &total_pairs);
   const int present = (tid < E && cnt > 0) ? 1 : 0;
   const int upos = block_exclusive_scan_i(present, iscr, &n_u);
+  DTR_AT(6);
   if (tid < E) {
     goff[tid] = off;
     if (present) {
@@ -99,6 +123,7 @@ dispatch_count_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
     if (total_pairs != pairs) record_error(err, kErrBadDispatch, kAtDispatch, total_pairs);
     *ticket = 0;   // ready for the next call
   }
+  DTR_AT(7);
   KLOG(DMOE_KERNEL_DISPATCH, 1);
 }
 
@@ -112,7 +137,6 @@ dispatch_place_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
   const int c = blockIdx.x, tid = threadIdx.x;
   const int t0 = c * 32, ntok = T - t0 < 32 ? T - t0 : 32, np = ntok * k;
   const int pairs = T * k;
-  pdl_launch_dependents();
   // the routing was complete before the counting launch let this one start
   int ids[kDispPerThread];
 #pragma unroll
@@ -121,6 +145,7 @@ dispatch_place_kernel(const int32_t* __restrict__ topk_idx, int T, int E, int k,
     ids[j] = p < np ? __ldcg(topk_idx + t0 * k + p) : 0;
   }
   pdl_wait();
+  pdl_launch_dependents();   // after the wait: a waiting dependent would share the SMs
   KLOG(7, 0);
   for (int e = tid; e < E; e += kDispThreads) {
     bits[e] = gbits[(size_t)c * E + e];
@@ -167,4 +192,7 @@ cudaError_t launch_dispatch(const DispatchArgs& a, cudaStream_t s) {
 
 #ifdef DMOE_TRACE
 DMOE_KLOG_EXPORT(dmoe_debug_klog_dispatch)
+extern "C" int dmoe_debug_dtr(void* host) {
+  return (int)cudaMemcpyFromSymbol(host, g_dtr, sizeof(g_dtr));
+}
 #endif

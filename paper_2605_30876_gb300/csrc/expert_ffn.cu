@@ -180,7 +180,6 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
-  pdl_launch_dependents();
   pdl_wait();  // dispatch output and the gathered rows are complete from here on
 
   // ---------------- groups and unit lists (slot 0 = the shared expert when present)
@@ -579,6 +578,9 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  // the combine may start now: launched earlier, its waiting CTAs would share the SMs with
+  // this launch and slow it down
+  pdl_launch_dependents();
   if (tid == 0) DMOE_TRACE_AT(62);
   KLOG(DMOE_KERNEL_EXPERTS, 1);
   if (warp == 1) {
@@ -592,8 +594,8 @@ __global__ void __launch_bounds__(256)
 gather_kernel(const __nv_bfloat16* __restrict__ x, const int32_t* __restrict__ rows,
               __nv_bfloat16* __restrict__ xperm, int32_t* __restrict__ h_ready, int n_ready,
               int pairs, int k, int d) {
-  pdl_launch_dependents();
   pdl_wait();
+  pdl_launch_dependents();   // after the wait: a waiting dependent would share the SMs
   KLOG(DMOE_KERNEL_GATHER, 0);
   if (blockIdx.x == 0)
     for (int i = threadIdx.x; i < n_ready; i += blockDim.x) h_ready[i] = 0;

@@ -107,8 +107,8 @@ router_softmax_kernel(const float* __restrict__ part, int splits, const float* _
                       float* __restrict__ probs, float* __restrict__ probs_hat,
                       int32_t* __restrict__ topk_idx, float* __restrict__ topk_gate,
                       int T, int E, int k, int mode) {
-  pdl_launch_dependents();
   pdl_wait();
+  pdl_launch_dependents();   // after the wait: a waiting dependent would share the SMs
   KLOG(5, 0);
   const int t = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (t >= T) return;
@@ -123,8 +123,8 @@ block_route_kernel(const float* __restrict__ probs, const float* __restrict__ pr
                    int E, int kb, int k, int B, float top_p,
                    int32_t* __restrict__ topk_idx, float* __restrict__ topk_gate,
                    int32_t* __restrict__ coreset, int32_t* __restrict__ coreset_size) {
-  pdl_launch_dependents();
   pdl_wait();
+  pdl_launch_dependents();   // after the wait: a waiting dependent would share the SMs
   KLOG(6, 0);
   DMOE_STAMP(0);
   block_route_cta(blockIdx.x, probs, probs_hat, E, kb, k, B, top_p, topk_idx, topk_gate, coreset,
