@@ -244,9 +244,11 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
                         const int32_t* n_unique, const int32_t* unique_ids,
                         const int32_t* offsets, const int32_t* rows, const int32_t* pos,
                         void* y, void* ws, const Workspace& plan, cudaStream_t s,
-                        bool shared_prefetched = false, uint32_t* spec_words = nullptr) {
+                        bool shared_prefetched = false, uint32_t* spec_words = nullptr,
+                        bool gathered = false) {
   ExpertArgs a{};
   a.prefetch_shared = !shared_prefetched;
+  a.gathered = gathered;
   a.spec_words = spec_words;
   a.spec_blocks = desc->n_blocks;
   a.x = static_cast<const __nv_bfloat16*>(x);
@@ -394,6 +396,19 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   dsp.k = desc->top_k;
   dsp.err = at<DevErrRecord>(workspace, plan.err);
   set_dispatch_scratch(&dsp, workspace, plan);
+  const int T_all = desc->n_blocks * desc->block_size;
+  // general path: the dispatch placement also writes x in dispatch order and clears the
+  // expert launch's tile counters (no gather launch)
+  const bool gathered =
+      !route_cluster_ok(T_all, desc->d_model, desc->n_experts) &&
+      !experts_decode_ok(T_all, desc->d_model, desc->d_ff, desc->d_ff_shared);
+  if (gathered) {
+    dsp.x = static_cast<const __nv_bfloat16*>(x);
+    dsp.xperm = at<__nv_bfloat16>(workspace, plan.xperm);
+    dsp.d = desc->d_model;
+    dsp.zero = at<int32_t>(workspace, plan.h_ready);
+    dsp.n_zero = experts_ready_counters(T_all, desc->n_experts, plan.n_max);
+  }
   // block top-k through the decode-size launches: the expert launch starts streaming on the
   // early-published coresets, before the routing launch ends (only when every token keeps
   // the whole coreset, so that the coresets' union is the unique set)
@@ -408,7 +423,8 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
                   shared_pf, &dsp, spec_w);
   if (st != DMOE_OK) return st;
   return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid, offs,
-                     rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w);
+                     rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w,
+                     gathered);
 }
 
 dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) {
@@ -479,10 +495,10 @@ int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc) {
     n += desc->mode == DMOE_ROUTE_BLOCK ? 1 : 0;              // Algorithm 1
     n += 2;                                                   // dispatch: count, place
   }
-  if (experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared))
-    n += 2;                                                   // experts, combine
-  else
-    n += 3;                                                   // gather, experts, combine
+  // experts and combine; the general experts' gather is a launch of its own only after the
+  // fused routing launch (otherwise the dispatch placement does it)
+  const bool dec = experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared);
+  n += (!dec && route_cluster_ok(T, desc->d_model, desc->n_experts)) ? 3 : 2;
   return n;
 }
 

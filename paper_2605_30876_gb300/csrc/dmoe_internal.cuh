@@ -196,6 +196,14 @@ struct DispatchArgs {
   int32_t* base;
   int32_t* off;
   int32_t* ticket;
+  // optional (the fused layer call of the general path): the placement also copies x's
+  // rows into dispatch order (xperm [T*k, d]) and clears zero[0 .. n_zero) (the expert
+  // launch's tile counters), so that the expert launch needs no gather launch
+  const __nv_bfloat16* x;
+  __nv_bfloat16* xperm;
+  int d;
+  int32_t* zero;
+  int n_zero;
 };
 // ticket index (in Workspace::tickets) of the dispatch launch
 constexpr int kDispatchTicket = 1;
@@ -239,6 +247,7 @@ struct ExpertArgs {
   int32_t* tickets;       // kRouteTickets ints, zero between calls
   DevErrRecord* err;
   bool prefetch_shared;   // the shared expert's weights were not prefetched by the router
+  bool gathered;          // xperm is written and the tile counters cleared (by the dispatch)
   // decode-size path, block top-k: the unique experts are the union of the published
   // coresets (RouterArgs::spec_words), known before the routing launch ends; nullptr
   // otherwise

@@ -787,8 +787,9 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   const int pairs = a.T * a.k;
   const bool has_shared = a.Is > 0;
   const int n_ready = experts_ready_counters(a.T, a.E, a.n_max);
-  // 1. gather x in dispatch order; clear the gate/up tile counters
-  {
+  // 1. gather x in dispatch order; clear the gate/up tile counters (unless the dispatch
+  //    placement of the fused layer call has done both)
+  if (!a.gathered) {
     const int grid = pairs < 1024 ? pairs : 1024;
     prof_begin(DMOE_KERNEL_GATHER, s);
     cudaError_t e = launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, true, a.x, a.rows,

@@ -67,8 +67,12 @@ router_wsplit_kernel(const float* __restrict__ w_r, __nv_bfloat16* __restrict__ 
                      int E) {
   const int e = blockIdx.x * 32 + (threadIdx.x & 31);
   const int k0 = blockIdx.y * 64 + (threadIdx.x >> 5) * 8;
-  // the previous launch on the stream may still read the parts of the call before
-  pdl_wait();
+  // No dependency wait: this launch reads only W_r (an input) and writes only the parts,
+  // which only the logits launch of an earlier call reads. That launch is always followed
+  // by router_softmax_kernel, which releases its dependents only after its own dependency
+  // wait (the logits launch has ended by then); so by the time any later launch, this one
+  // included, can start, the earlier logits launch has ended. The logits launch after
+  // this one waits for it.
   pdl_launch_dependents();
   KLOG(8, 0);
   if (e >= E) return;
@@ -290,14 +294,14 @@ bool router_tc_ok(int T, int d, int E) {
 }
 
 // Slices of d: each CTA takes at most 256 of d; of the splits that divide d into whole
-// 64-wide chunks (at most 8, the partial rows the softmax warp loads in one round), the
+// 64-wide chunks (at most 16, two rounds of the softmax warp's partial-row loads), the
 // largest that still gives one wave of CTAs, else the smallest.
 int router_tc_splits(int T, int d) {
   const int tiles = (T + kLtM - 1) / kLtM;
   const int nch = d / kLtKC;
   const int s_min = (d + kLtMaxDS - 1) / kLtMaxDS;
   int best = 0;
-  for (int s = s_min; s <= nch && s <= 8; ++s)
+  for (int s = s_min; s <= nch && s <= 16; ++s)
     if (nch % s == 0 && (best == 0 || tiles * s <= 152)) best = s;
   if (best == 0)
     for (int s = s_min; s <= nch; ++s)

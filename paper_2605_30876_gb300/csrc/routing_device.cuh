@@ -381,36 +381,48 @@ __device__ inline void mask_topk_warps(int k, int B, int size, const int* order,
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int nw = (int)(blockDim.x >> 5);
   if (size <= 32) {
-    // one member per lane: k rounds of a tournament (larger score, ties to the lower id);
-    // the scores of up to eight of the warp's tokens are loaded before the first tournament
+    // one member per lane: k rounds of a tournament (larger score, ties to the lower id),
+    // run for four of the warp's tokens at once (their reductions are independent, so they
+    // overlap); the scores of those tokens are loaded before the first round
     const int e = lane < size ? order[lane] : -1;
-    for (int i0 = warp; i0 < B; i0 += 8 * nw) {
-      uint32_t keys[8];
+    constexpr int kTok = 4;
+    for (int i0 = warp; i0 < B; i0 += kTok * nw) {
+      uint32_t key[kTok];
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kTok; ++u) {
         const int i = i0 + u * nw;
-        keys[u] = (i < B && e >= 0) ? order_key(prob(i, e)) : 0u;
+        key[u] = (i < B && e >= 0) ? order_key(prob(i, e)) : 0u;
+      }
+      int my_e[kTok];
+      float my_v[kTok];
+#pragma unroll
+      for (int u = 0; u < kTok; ++u) {
+        my_e[u] = -1;
+        my_v[u] = 0.f;
+      }
+      for (int r = 0; r < k; ++r) {
+        uint32_t kmax[kTok], imin[kTok];
+#pragma unroll
+        for (int u = 0; u < kTok; ++u) kmax[u] = __reduce_max_sync(0xffffffffu, key[u]);
+#pragma unroll
+        for (int u = 0; u < kTok; ++u)
+          imin[u] = __reduce_min_sync(0xffffffffu, key[u] == kmax[u] ? (uint32_t)e : 0xffffffffu);
+#pragma unroll
+        for (int u = 0; u < kTok; ++u) {
+          if (lane == r) {
+            my_e[u] = (int)imin[u];
+            my_v[u] = key_value(kmax[u]);
+          }
+          if (key[u] == kmax[u] && (uint32_t)e == imin[u]) key[u] = 0u;
+        }
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
+      for (int u = 0; u < kTok; ++u) {
         const int i = i0 + u * nw;
         if (i >= B) break;   // the same for the whole warp
-        uint32_t key = keys[u];
-        int my_e = -1;
-        float my_v = 0.f;
-        for (int r = 0; r < k; ++r) {
-          const uint32_t kmax = __reduce_max_sync(0xffffffffu, key);
-          const uint32_t imin =
-              __reduce_min_sync(0xffffffffu, key == kmax ? (uint32_t)e : 0xffffffffu);
-          if (lane == r) {
-            my_e = (int)imin;
-            my_v = key_value(kmax);
-          }
-          if (key == kmax && (uint32_t)e == imin) key = 0u;
-        }
         float g = 0.f;
-        for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v, r);
-        if (lane < k) out(i, lane, my_e, my_v / g);
+        for (int r = 0; r < k; ++r) g += __shfl_sync(0xffffffffu, my_v[u], r);
+        if (lane < k) out(i, lane, my_e[u], my_v[u] / g);
       }
     }
     return;
