@@ -886,9 +886,10 @@ def main():
 
     # headline: block routing, p = 0
     arm = Arm(shape, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
-    # the headline pass records no events: an event between two kernels would serialise
-    # their programmatic-dependent-launch overlap; the expert kernel's launch duration is
-    # timed by CUDA events in a second pass over the same steps
+    # the headline pass records no events; the expert kernel's launch duration is timed by
+    # CUDA events in a second pass over the same steps (while the events are set, the
+    # library makes that launch without programmatic overlap, so that they bracket its own
+    # execution rather than an early start spent waiting for the routing)
     secs, _, clocks = timed_region(arm, args.steps, args.warmup, torch, dist, world,
                                    want_kernel=False, sampler=sampler)
     _, kern_s, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world)

@@ -175,8 +175,11 @@ typedef enum {
 /* Profiling aid, not part of the method: while set, every launch of `kernel` made by a
  * call on this host thread records `ev_begin` just before it and `ev_end` just after it on
  * the call's stream (cudaEvent_t handles passed as void*, created with timing enabled;
- * recorded as external events, so they also work inside a CUDA-graph capture). Passing
- * NULL for both clears the setting. Returns DMOE_ERR_INVALID_ARG for an unknown kernel. */
+ * recorded as external events, so they also work inside a CUDA-graph capture). The expert
+ * launch is then made without programmatic dependent launch: it starts once the launch
+ * before it has ended, so that the events bracket its own execution (not an early start
+ * spent waiting for the routing). Passing NULL for both clears the setting. Returns
+ * DMOE_ERR_INVALID_ARG for an unknown kernel. */
 dmoe_status dmoe_set_profile_events(int32_t kernel, void* ev_begin, void* ev_end);
 
 /* dmoe_router for callers that cannot allocate device memory. The paper has no

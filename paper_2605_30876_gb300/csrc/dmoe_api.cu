@@ -55,6 +55,7 @@ void prof_begin(int kernel, cudaStream_t s) {
 void prof_end(int kernel, cudaStream_t s) {
   if (g_prof[kernel].end != nullptr) prof_record(g_prof[kernel].end, s);
 }
+bool prof_serial(int kernel) { return g_prof[kernel].begin != nullptr; }
 
 void set_last_error(cudaError_t e) {
   snprintf(g_last_error, sizeof(g_last_error), "%s: %s", cudaGetErrorName(e),

@@ -277,6 +277,9 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s);
 // profiling events (dmoe_set_profile_events), per host thread
 void prof_begin(int kernel, cudaStream_t s);
 void prof_end(int kernel, cudaStream_t s);
+// events are set for `kernel` on this host thread: its launch is made without programmatic
+// dependent launch, so that the events bracket its own execution only
+bool prof_serial(int kernel);
 
 // Programmatic dependent launch: a kernel launched with `pdl` set may start while the
 // previous kernel on the stream is still running; it must call pdl_wait() before reading

@@ -856,7 +856,8 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   if (a.spec_words != nullptr && grid > 2 * kRouteClusterCtas) grid -= kRouteClusterCtas;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
-  cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s, true, m, p);
+  cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s,
+                            !prof_serial(DMOE_KERNEL_EXPERTS), m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
   // the expert launch releases the combine at its end, after its wait for the routing

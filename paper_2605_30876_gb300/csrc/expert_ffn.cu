@@ -45,6 +45,7 @@ constexpr int kATileBytes = kTileM * 128;          // 16 KB: 128 rows x 64 K (on
 constexpr int kMaxGroups = kMaxExperts + 1;
 constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr int kMaxStages = 8;
+constexpr int64_t kDownPrefetchMax = (int64_t)64 << 20;   // half of the 129 MB L2
 constexpr int kXchgStride = 17;                    // floats per row of the exchange buffers
 
 struct GemmParams {
@@ -255,14 +256,17 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   if (tid == 64) {
     // Pull the down-projection weights of every unique expert into L2 now, spread over all
     // CTAs: the down units of the second wave then read them from L2, and HBM keeps
-    // streaming while the gate/up results are produced and published.
+    // streaming while the gate/up results are produced and published. Only while they
+    // fit in half of L2: beyond that the prefetched lines are evicted before their use
+    // and only add HBM traffic (token routing at 2048 tokens: 256 experts, 537 MB).
     L2Prefetch pf;
     pf.ptr[2] = p.w_down;
     pf.bytes = (int64_t)p.d * p.I * 2;
     const int64_t per = (pf.bytes + kPrefetchChunk - 1) / kPrefetchChunk;
     const int total = (int)(3 * per * U);
-    for (int c = (int)(2 * per * U) + blockIdx.x; c < total; c += gridDim.x)
-      l2_prefetch_chunk(pf, p.unique_ids, U, c);
+    if (pf.bytes * U <= kDownPrefetchMax)
+      for (int c = (int)(2 * per * U) + blockIdx.x; c < total; c += gridDim.x)
+        l2_prefetch_chunk(pf, p.unique_ids, U, c);
     if (p.ws_gate != nullptr) {
       L2Prefetch sp;
       sp.ptr[0] = p.ws_gate;
@@ -861,7 +865,8 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   int grid = device_sm_count();
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
-  cudaError_t e = launch_ex(moe_experts_kernel, dim3(grid), dim3(kThreads), smem, s, true, m, gp);
+  cudaError_t e = launch_ex(moe_experts_kernel, dim3(grid), dim3(kThreads), smem, s,
+                            !prof_serial(DMOE_KERNEL_EXPERTS), m, gp);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
 
