@@ -65,6 +65,8 @@ struct GemmParams {
   int n_max;              // token tile = rows of the B box
   int n_half;             // rows of the half box (token tiles of at most this many rows)
   int kbs;                // K boxes per stage (1 for 256-row token tiles, else 2)
+  int dpair;              // 128-row tiles of W_down per down unit (2: a pair sharing the H
+                          // stages, K = 64 per stage; 1)
   int ntiles;             // token tiles per group at most
   int stages;
   int n_acc;              // accumulator buffers in TMEM
@@ -147,8 +149,8 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   int* misc = reinterpret_cast<int*>(drain + 1);
   uint32_t* s_tmem = reinterpret_cast<uint32_t*>(misc + 0);
   volatile int* s_abort = misc + 1;
-  int* s_sched = misc + 4;                         // G, U, gu_units, dn_units
-  int* gu_prefix = misc + 8;                       // [kMaxGroups + 1], by slot
+  int* s_sched = misc + 4;                         // G, U, gu_units, dn_units, dpair
+  int* gu_prefix = misc + 12;                      // [kMaxGroups + 1], by slot
   int* dn_prefix = gu_prefix + (kMaxGroups + 1);   // [kMaxGroups + 1], by slot
   int* g_row0 = dn_prefix + (kMaxGroups + 1);      // by group
   int* g_cnt = g_row0 + kMaxGroups;
@@ -237,6 +239,15 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       carry_gu += __shfl_sync(0xffffffffu, igu, 31);
       carry_dn += __shfl_sync(0xffffffffu, idn, 31);
     }
+    // pairs of down tiles only when the down units are many per CTA (a pair unit pulls 25 %
+    // less per tile but holds less of its weights before H is ready: with about one or two
+    // single units per CTA it lengthens the tail); a pair count is the single count / 2
+    const int dpair = (p.dpair == 2 && carry_dn >= 4 * (int)gridDim.x) ? 2 : 1;
+    if (dpair == 2) {
+      __syncwarp();
+      for (int i = lane; i <= G; i += 32) dn_prefix[i] /= 2;
+      carry_dn /= 2;
+    }
     if (lane == 0) {
       gu_prefix[0] = 0;
       dn_prefix[0] = 0;
@@ -244,6 +255,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       s_sched[1] = U;
       s_sched[2] = carry_gu;
       s_sched[3] = carry_dn;
+      s_sched[4] = dpair;
     }
   }
   ptx::tc_fence_before();
@@ -251,6 +263,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   ptx::tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
   const int G = s_sched[0], U = s_sched[1], n_gu = s_sched[2], n_dn = s_sched[3];
+  const int dpair = s_sched[4];   // 128-row tiles of W_down per down unit
   const int units = n_gu + n_dn;
   if (tid == 0) DMOE_TRACE_AT(1);
   if (tid == 64) {
@@ -359,23 +372,38 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
             if (++stage == stages) { stage = 0; phase ^= 1u; }
           }
         } else {
+          // a pair unit takes 128-row tiles 2m and 2m+1 of W_down over K = 64 per stage (its
+          // two A boxes side by side at the same K), both against the stage's one H box
+          const bool pr = dpair == 2;
+          const int ksz = pr ? kTileK : stage_k;               // K per stage
+          const int nbb = pr ? 1 : kbs;                        // B boxes per stage
+          const uint32_t b_bytes_d =
+              (uint32_t)nbb * (half ? (uint32_t)p.n_half * 128u : b_box);
+          const uint32_t tx_d = a_stage + b_bytes_d;
           const int Kg = shared ? p.Is : p.I;
-          const int arow = shared ? un.m * kTileM : g_e[un.g] * p.d + un.m * kTileM;
+          const int arow = (shared ? 0 : g_e[un.g] * p.d) + un.m * dpair * kTileM;
           const int brow = (shared ? 0 : g_row0[un.g]) + un.n * p.n_max;
           const CUtensorMap* ma = shared ? &tm.sd : &tm.wd;
           const CUtensorMap* mb = shared ? &tm.hs : (half ? &tm.hh : &tm.h);
-          const int kc = Kg / stage_k;
+          const int kc = Kg / ksz;
           const int pre = kc < stages ? kc : stages;
           const int stage0 = stage;
-          const uint32_t phase0 = phase;
+          auto load_a = [&](int st, int c) {
+            uint8_t* a_dst = smem + off_a + st * a_stage;
+            if (pr) {
+              ptx::tma_load_2d(a_dst, ma, &full[st], c * ksz, arow, pol_w);
+              ptx::tma_load_2d(a_dst + kATileBytes, ma, &full[st], c * ksz, arow + kTileM, pol_w);
+            } else {
+              for (int kb = 0; kb < kbs; ++kb)
+                ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[st], c * ksz + kb * kTileK,
+                                 arow, pol_w);
+            }
+          };
           // weights first: they do not depend on the gate/up phase
           for (int c = 0; c < pre; ++c) {
             if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
-            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * a_stage;
-            for (int kb = 0; kb < kbs; ++kb)
-              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], c * stage_k + kb * kTileK,
-                               arow, pol_w);
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_d);
+            load_a(stage, c);
             ++issued;
             if (++stage == stages) { stage = 0; phase ^= 1u; }
           }
@@ -402,27 +430,24 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           for (int c = 0; c < pre; ++c) {
             if (ok) {
               uint8_t* b_dst = smem + off_b + st * b_stage;
-              for (int kb = 0; kb < kbs; ++kb)
-                ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], c * stage_k + kb * kTileK, brow,
+              for (int kb = 0; kb < nbb; ++kb)
+                ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], c * ksz + kb * kTileK, brow,
                                  pol_x);
             } else {
               // keep the barrier accounting whole: complete the stage without B data
-              ptx::mbar_complete_tx_local(&full[st], b_bytes);
+              ptx::mbar_complete_tx_local(&full[st], b_bytes_d);
             }
             if (++st == stages) st = 0;
           }
-          (void)phase0;
           if (!ok) break;
           for (int c = pre; c < kc; ++c) {
             if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
-            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * a_stage;
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_d);
+            load_a(stage, c);
             uint8_t* b_dst = smem + off_b + stage * b_stage;
-            for (int kb = 0; kb < kbs; ++kb) {
-              const int kx = c * stage_k + kb * kTileK;
-              ptx::tma_load_2d(a_dst + kb * kATileBytes, ma, &full[stage], kx, arow, pol_w);
-              ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], kx, brow, pol_x);
-            }
+            for (int kb = 0; kb < nbb; ++kb)
+              ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], c * ksz + kb * kTileK, brow,
+                               pol_x);
             ++issued;
             if (++stage == stages) { stage = 0; phase ^= 1u; }
           }
@@ -453,33 +478,56 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       for (int u = blockIdx.x; u < units && ok; u += gridDim.x, ++li) {
         const Unit un = decode(u);
         const bool shared = un.g >= U;
+        const bool pr = !un.gu && dpair == 2;     // a pair of down tiles, two accumulators
         const int Kg = un.gu ? p.d : (shared ? p.Is : p.I);
-        const int kc = Kg / stage_k;
+        const int kc = Kg / (pr ? kTileK : stage_k);
         const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
         const uint32_t n_mma = (uint32_t)((nvalid + 15) & ~15);
         const uint32_t idesc = ptx::idesc_bf16(kTileM, n_mma);
+        // the second accumulator of a pair: the next slot
+        int acc2 = acc + 1;
+        uint32_t acc2_phase = acc_phase;
+        if (acc2 == p.n_acc) { acc2 = 0; acc2_phase ^= 1u; }
         if (!wait(&acc_empty[acc], acc_phase ^ 1u, u)) { ok = false; break; }
+        if (pr && !wait(&acc_empty[acc2], acc2_phase ^ 1u, u)) { ok = false; break; }
         ptx::tc_fence_after();
         const uint32_t d0 = tmem_base + (uint32_t)acc * (uint32_t)p.n_max;
+        const uint32_t d1 = tmem_base + (uint32_t)acc2 * (uint32_t)p.n_max;
         for (int c = 0; c < kc; ++c) {
           if (!wait(&full[stage], phase, u)) { ok = false; break; }
           ptx::tc_fence_after();
           if (!*s_abort) {
             const uint32_t a0 = ptx::smem_addr(smem + off_a + stage * a_stage);
             const uint32_t b0 = ptx::smem_addr(smem + off_b + stage * b_stage);
-            for (int kb = 0; kb < kbs; ++kb)
+            if (pr) {
 #pragma unroll
-              for (int kk = 0; kk < kTileK / 16; ++kk)
-                ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kATileBytes + kk * 32),
-                              ptx::sdesc_k_sw128(b0 + kb * b_box + kk * 32), idesc,
-                              (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
+              for (int kk = 0; kk < kTileK / 16; ++kk) {
+                const uint64_t bd = ptx::sdesc_k_sw128(b0 + kk * 32);
+                const uint32_t accum = (c > 0 || kk > 0) ? 1u : 0u;
+                ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kk * 32), bd, idesc, accum);
+                ptx::mma_bf16(d1, ptx::sdesc_k_sw128(a0 + kATileBytes + kk * 32), bd, idesc,
+                              accum);
+              }
+            } else {
+              for (int kb = 0; kb < kbs; ++kb)
+#pragma unroll
+                for (int kk = 0; kk < kTileK / 16; ++kk)
+                  ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * kATileBytes + kk * 32),
+                                ptx::sdesc_k_sw128(b0 + kb * b_box + kk * 32), idesc,
+                                (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
+            }
           }
           ptx::mma_commit(&empty[stage]);
           if (++stage == stages) { stage = 0; phase ^= 1u; }
         }
         if (!ok) break;
         ptx::mma_commit(&acc_full[acc]);
+        if (pr) ptx::mma_commit(&acc_full[acc2]);
         if (li < 8) DMOE_TRACE_AT(6 + 6 * li);
+        if (pr) {
+          acc = acc2;
+          acc_phase = acc2_phase;
+        }
         if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
       }
       // make sure no MMA is still running when TMEM is released
@@ -505,7 +553,13 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       const bool shared = un.g >= U;
       const int nvalid = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
       const int n_mma = (nvalid + 15) & ~15;
-      if (!epi_all_threads(wait(&acc_full[acc], acc_phase, u))) break;
+      const bool pr = !un.gu && dpair == 2;     // a pair of down tiles: two accumulators
+      int acc2 = acc + 1;
+      uint32_t acc2_phase = acc_phase;
+      if (acc2 == p.n_acc) { acc2 = 0; acc2_phase ^= 1u; }
+      if (!epi_all_threads(wait(&acc_full[acc], acc_phase, u) &&
+                           (!pr || wait(&acc_full[acc2], acc2_phase, u))))
+        break;
       ptx::tc_fence_after();
       if (tid == 64 && li < 8) DMOE_TRACE_AT(50 + li);
       const uint32_t tbase = tmem_base + lane_off + (uint32_t)acc * (uint32_t)p.n_max;
@@ -560,21 +614,30 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         if (tid == 64 && li < 8) DMOE_TRACE_AT(58 + (li < 4 ? li : 3));
         if (tid == 64) red_release_add(p.h_ready + un.g * p.ntiles + un.n, 1);
       } else {
-        const int drow = un.m * kTileM + q * 32 + lane;
         __nv_bfloat16* out = shared ? p.yshared + (size_t)col0 * p.d
                                     : p.yslot + (size_t)(g_row0[un.g] + col0) * p.d;
-        for (int c0 = 16 * cg; c0 < n_mma; c0 += 32) {
-          float v[16];
-          ptx::tmem_ld16(tbase + c0, v);
-          ptx::tmem_ld_wait();
+        for (int h = 0; h < (pr ? 2 : 1); ++h) {
+          const int slot = h == 0 ? acc : acc2;
+          const uint32_t tb = tmem_base + lane_off + (uint32_t)slot * (uint32_t)p.n_max;
+          const int drow = (un.m * dpair + h) * kTileM + q * 32 + lane;
+          for (int c0 = 16 * cg; c0 < n_mma; c0 += 32) {
+            float v[16];
+            ptx::tmem_ld16(tb + c0, v);
+            ptx::tmem_ld_wait();
 #pragma unroll
-          for (int c = 0; c < 16; ++c)
-            if (c0 + c < nvalid) out[(size_t)(c0 + c) * p.d + drow] = __float2bfloat16_rn(v[c]);
+            for (int c = 0; c < 16; ++c)
+              if (c0 + c < nvalid)
+                out[(size_t)(c0 + c) * p.d + drow] = __float2bfloat16_rn(v[c]);
+          }
+          ptx::tc_fence_before();
+          ptx::mbar_arrive(&acc_empty[slot]);
         }
-        ptx::tc_fence_before();
-        ptx::mbar_arrive(&acc_empty[acc]);
       }
       if (tid == 64 && li < 8) DMOE_TRACE_AT(7 + 6 * li);
+      if (pr) {
+        acc = acc2;
+        acc_phase = acc2_phase;
+      }
       if (++acc == p.n_acc) { acc = 0; acc_phase ^= 1u; }
     }
   }
@@ -652,7 +715,7 @@ template <> struct Raw8<float> {
 // launch before this one could let this one start (the decode-size expert launch releases
 // it only at its end, after its own wait for the routing launch that wrote them).
 template <typename Row>
-__global__ void __launch_bounds__(256)
+__global__ void __launch_bounds__(256, sizeof(Row) == 2 ? 3 : 1)   // bf16 rows: three CTAs per SM
 combine_kernel(const Row* __restrict__ yslot, const Row* __restrict__ yshared,
                const int32_t* __restrict__ pos, const float* __restrict__ gate,
                __nv_bfloat16* __restrict__ y, int k, int d, int has_shared, int32_t* zero,
@@ -759,7 +822,7 @@ uint32_t pow2_cols(uint32_t c) {
 size_t experts_fixed_smem() {
   // alignment slack + exchange buffers + barriers + misc/group arrays
   return 1024 + 2 * 128 * kXchgStride * 4 + 8 + 8 * (2 * kMaxStages + 9) +
-         sizeof(int) * (8 + 5 * (kMaxGroups + 1)) + 64;
+         sizeof(int) * (12 + 5 * (kMaxGroups + 1)) + 64;
 }
 
 int max_smem_optin() {
@@ -821,6 +884,10 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   gp.n_max = a.n_max;
   gp.n_half = ((a.n_max / 2) + 15) & ~15;
   gp.kbs = a.n_max >= 256 ? 1 : kMaxKBoxes;
+  // pairs of down tiles share their H stages: 25 % less to pull per SM and half the down
+  // units, so that each CTA takes about one (needs two K boxes per stage for the pair's A
+  // and an even number of 128-row tiles of d)
+  gp.dpair = (gp.kbs == 2 && (a.d / kTileM) % 2 == 0) ? 2 : 1;
   gp.ntiles = (a.T + a.n_max - 1) / a.n_max;
   gp.has_shared = has_shared ? 1 : 0;
 
