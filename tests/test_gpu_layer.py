@@ -82,7 +82,8 @@ def test_layer_forward_matches_oracle(name):
     assert torch.equal(y, y2)
 
 
-@pytest.mark.parametrize("name", ["tiny_block_p06", "layer_block_p06", "layer_token"])
+@pytest.mark.parametrize("name", ["tiny_block_p06", "layer_block_p06", "layer_token",
+                                  "layer_b8_block_p0", "T300_multi_ntile"])
 def test_moe_forward_on_injected_oracle_routing(name):
     """dmoe_dispatch + dmoe_moe_forward on the oracle's own routing (ids and gates)."""
     shape = LAYER_CASES[name]

@@ -43,6 +43,14 @@ ROUTING_CASES = {
     "block_size_128": LAYER.with_(block_size=128, n_blocks=2, top_p=0.6),
     # the Top-4 token-level baseline
     "layer_token_top4": LAYER.with_(mode=ROUTE_TOKEN, top_k=4),
+    # the logits of 128+ tokens: tcgen05 with N = E < 256 and a ragged last token tile;
+    # the mma.sync cluster stage where E % 32 != 0; the FFMA tiles where d % 256 != 0 too
+    "tc_E64_T200": LAYER.with_(n_experts=64, block_size=40, n_blocks=5, top_p=0.6),
+    "tc_E224_T384_token": LAYER.with_(n_experts=224, block_size=32, n_blocks=12,
+                                      mode=ROUTE_TOKEN),
+    "cluster_logits_E40_T256": LAYER.with_(n_experts=40, block_size=32, n_blocks=8),
+    "ffma_logits_E40_d384_T256": LAYER.with_(n_experts=40, d_model=384, block_size=32,
+                                             n_blocks=8, top_p=0.6),
 }
 
 
