@@ -55,7 +55,8 @@ constexpr int kMaxTok = 64;                     // tokens of a decode-sized forw
 // stage landed, 3 gate/up MMAs committed, 4 gate/up tile published, 5 down weights issued,
 // 6 H ready seen, 7 down MMAs committed, 8 down rows stored, 9 exit, 10 gate/up unit id,
 // 11 down unit id, 12/13 first/last down stage landed, 14 down accumulator ready, 15 down
-// accumulator staged, 16 staging complete, 17 row copies issued.
+// accumulator staged, 16 staging complete, 17 row copies issued, 18 coresets seen by the
+// polling warp.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_dtrace[kMaxPersistentCtas * 32];
 #define ED_AT(slot) (g_dtrace[blockIdx.x * 32 + (slot)] = ptx::globaltimer_ns())
@@ -144,6 +145,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   volatile int* s_abort = reinterpret_cast<volatile int*>(s_tmem + 1);
   int* s_u = const_cast<int*>(s_abort) + 1;
   uint8_t* s_spec = reinterpret_cast<uint8_t*>(s_u + 1);   // [kMaxExperts]: unique ids
+  uint32_t* s_mask = reinterpret_cast<uint32_t*>(s_spec + kMaxExperts);   // [kMaxExperts / 32]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nb = gridDim.x, b = blockIdx.x;
@@ -172,6 +174,23 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
+  // What does not depend on the unit list is read and derived before any wait, so that
+  // nothing but the list is left once the coresets or the dispatch are in: the producer's
+  // diagnostic hold (normally 0: every down unit waits for this many more gate/up tiles
+  // than its group has, so that its bounded wait runs out) and the shapes of both unit
+  // heights.
+  int hold = 0;
+  if (tid == 0) hold = *reinterpret_cast<volatile int32_t*>(&p.err->hold);
+  const int has_shared = p.has_shared, pI = p.I, pIs = p.Is;
+  const int ngu64_s = has_shared ? pIs / 64 : 0, ngu64_r = pI / 64;
+  const int slot32 = kAStage + (kTileM / 32) * bbox, slot64 = kAStage + (kTileM / 64) * bbox;
+  const int S32 = min(p.ring_bytes / slot32, kMaxStagesD);
+  const int S64 = min(p.ring_bytes / slot64, kMaxStagesD);
+  const int ngu_s32 = has_shared ? pIs / 32 : 0, ngu_r32 = pI / 32;
+  const int kc32 = p.d / (kMaxKBG * kTileK), kc64 = p.d / (2 * kTileK);
+  const int ndn = p.d / kTileM;
+  const bool h32_ok = p.h32_ok != 0;
+
   // Block top-k: the unique experts are the union of the blocks' coresets (every token of a
   // block is routed to all k experts of its coreset), published by the routing launch
   // before it ends; the weight stream starts on them, and only the down epilogue waits for
@@ -180,9 +199,11 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   if (spec) {
     if (warp == 0) {
       // poll every block's words until all are nonzero; a nonzero word is complete (one
-      // 32-bit store), so its ids go into the mask as it is seen (or-ing twice is harmless)
+      // 32-bit store), so its ids go into the shared mask as it is seen (or-ing twice is
+      // harmless)
       const int nw = spec_words(p.k), total = p.spec_blocks * nw;
-      uint32_t m[kMaxExperts / 32] = {};
+      if (lane < kMaxExperts / 32) s_mask[lane] = 0u;
+      __syncwarp();
       bool bad = false;
       const uint64_t t0 = ptx::globaltimer_ns();
       for (;;) {
@@ -199,26 +220,36 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
             if (r0 + j >= p.k) break;
             const int e = (int)((w >> (8 * j)) & 0xffu);
             if (e >= p.E) bad = true;
-            else m[e >> 5] |= 1u << (e & 31);
+            else atomicOr(&s_mask[e >> 5], 1u << (e & 31));
           }
         }
-        if (__all_sync(0xffffffffu, all)) break;
+        if (__all_sync(0xffffffffu, all)) {
+          if (lane == 0) ED_AT(18);
+          break;
+        }
         if (ptx::globaltimer_ns() - t0 > kTimeoutNs) {   // the coresets did not come
           bad = true;
           break;
         }
       }
       bad = __any_sync(0xffffffffu, bad);
+      __syncwarp();
+      // the ascending id list: lane w expands mask word w at its prefix position
+      const uint32_t mw = lane < kMaxExperts / 32 ? s_mask[lane] : 0u;
+      const int c = __popc(mw);
+      int incl = c;
 #pragma unroll
-      for (int w = 0; w < kMaxExperts / 32; ++w) m[w] = __reduce_or_sync(0xffffffffu, m[w]);
-      if (lane == 0) {
-        int u = 0;
-        if (!bad)
-          for (int w = 0; w < kMaxExperts / 32; ++w)
-            for (uint32_t bits = m[w]; bits != 0u; bits &= bits - 1u)
-              s_spec[u++] = (uint8_t)(w * 32 + __ffs((int)bits) - 1);
-        *s_u = bad ? -1 : u;
+      for (int o = 1; o < kMaxExperts / 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
       }
+      const int u_all = __shfl_sync(0xffffffffu, incl, kMaxExperts / 32 - 1);
+      if (!bad) {
+        int u = incl - c;
+        for (uint32_t bits = mw; bits != 0u; bits &= bits - 1u)
+          s_spec[u++] = (uint8_t)(lane * 32 + __ffs((int)bits) - 1);
+      }
+      if (lane == 0) *s_u = bad ? -1 : u_all;
     }
     __syncthreads();
     spec = *s_u >= 0;
@@ -239,23 +270,23 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   ptx::tc_fence_after();
   const uint32_t tmem_base = *s_tmem;
   const int U = *s_u;
-  const int G = U + p.has_shared;
+  const int G = U + has_shared;
   // gate/up unit height: 32 rows of I when even the 32-row units fit in one round over the
   // CTAs (a forward with few unique experts), else 64
-  const int ngu64 = (p.has_shared ? p.Is / 64 : 0) + U * (p.I / 64);
-  const int hg = (p.h32_ok && 2 * ngu64 <= nb) ? 32 : 64;
-  const int kbg = kTileM / hg;                    // K boxes per gate/up stage (32 KB)
-  const int slot = kAStage + kbg * bbox;
-  const int S = p.ring_bytes / slot < kMaxStagesD ? p.ring_bytes / slot : kMaxStagesD;
+  const bool h32 = h32_ok && 2 * (ngu64_s + U * ngu64_r) <= nb;
+  const int hg = h32 ? 32 : 64;
+  const int kbg = h32 ? kTileM / 32 : kTileM / 64;   // K boxes per gate/up stage (32 KB)
+  const int slot = h32 ? slot32 : slot64;
+  const int S = h32 ? S32 : S64;
   auto slot_a = [&](int st) { return ring + st * slot; };
   auto slot_b = [&](int st) { return ring + st * slot + kAStage; };
   const int abox_g = 2 * hg * 128;                // one K box of the stacked gate|up rows
-  const int ngu_s = p.has_shared ? p.Is / hg : 0, ngu_r = p.I / hg;
-  const int ndn = p.d / kTileM;
+  const int ngu_s = h32 ? ngu_s32 : ngu64_s, ngu_r = h32 ? ngu_r32 : ngu64_r;
   const int NGU = ngu_s + U * ngu_r;
   const int ND = G * ndn;
   // first down unit of this CTA: the round-robin continues after the NGU gate/up units
-  const int v0 = ((b - NGU % nb) % nb + nb) % nb;
+  const int nrem = NGU % nb;
+  const int v0 = b >= nrem ? b - nrem : b - nrem + nb;
   if (tid == 0) ED_AT(1);
 
   // the group's expert and size (all the weight stream needs)
@@ -325,15 +356,12 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       }
     }
   };
-  const int kc = p.d / (kbg * kTileK);   // stages of one gate/up tile
+  const int kc = h32 ? kc32 : kc64;   // stages of one gate/up tile
 
   if (warp == 0 && lane == 0) {
     // ================= TMA producer
     const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
     const uint64_t pol_x = ptx::policy_evict_last();    // x and H: re-read by many tiles
-    // diagnostic hold (normally 0): every down unit waits for this many more gate/up tiles
-    // than its group has, so that its bounded wait runs out
-    const int hold = *reinterpret_cast<volatile int32_t*>(&p.err->hold);
     int stage = 0, issued = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -746,7 +774,7 @@ uint32_t pow2_cols(uint32_t n) {
 // Shared memory besides the ring: staging tile, SwiGLU exchange, token list, barriers.
 size_t fixed_smem(int n_pad) {
   return 1024 /* alignment */ + (size_t)kTileM * (n_pad + 1) * 4 + kXchgBytes + kMaxTok * 4 +
-         (size_t)(2 * kMaxStagesD + 9) * 8 + 16 + kMaxExperts + 48;
+         (size_t)(2 * kMaxStagesD + 9) * 8 + 16 + kMaxExperts + kMaxExperts / 8 + 48;
 }
 
 // Pipeline ring: the shared memory left by the fixed part. A slot holds 32 KB of weights

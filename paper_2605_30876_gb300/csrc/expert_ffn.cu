@@ -943,16 +943,20 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
 
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero, int n_zero,
                            uint32_t* zero2, int n_zero2, bool meta_early, bool rows_bf16) {
-  dim3 cgrid((a.d / kCombineCols + 255) / 256, a.T);
+  // CTAs of 256 threads; fewer (down to 32) while that leaves fewer than 128 CTAs, so
+  // that a decode-sized forward spreads its rows over most SMs
+  int thr = 256;
+  while (thr > 32 && (a.d / kCombineCols + thr - 1) / thr * a.T < 128) thr >>= 1;
+  dim3 cgrid((a.d / kCombineCols + thr - 1) / thr, a.T);
   prof_begin(DMOE_KERNEL_COMBINE, s);
   cudaError_t e =
       rows_bf16
-          ? launch_ex(combine_kernel<__nv_bfloat16>, cgrid, dim3(256), 0, s, true,
+          ? launch_ex(combine_kernel<__nv_bfloat16>, cgrid, dim3(thr), 0, s, true,
                       static_cast<const __nv_bfloat16*>(a.yslot),
                       static_cast<const __nv_bfloat16*>(a.yshared), a.pos, a.topk_gate,
                       a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero, zero2, n_zero2,
                       meta_early ? 1 : 0)
-          : launch_ex(combine_kernel<float>, cgrid, dim3(256), 0, s, true,
+          : launch_ex(combine_kernel<float>, cgrid, dim3(thr), 0, s, true,
                       static_cast<const float*>(a.yslot), static_cast<const float*>(a.yshared),
                       a.pos, a.topk_gate, a.y, a.k, a.d, a.Is > 0 ? 1 : 0, zero, n_zero,
                       zero2, n_zero2, meta_early ? 1 : 0);

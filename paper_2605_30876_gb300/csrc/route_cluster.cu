@@ -22,7 +22,7 @@
 #include <math.h>
 
 // Debug builds (-DDMOE_TRACE): per-CTA timeline in g_ctrace[cta * 64 + stage] (stages 0
-// and 7: globaltimer, others: 1 = reached; + 32: clock64): 0 entry, 1 TMA landed, 8 x converted,
+// 7 and 25: globaltimer, others: 1 = reached; + 32: clock64): 0 entry, 1 TMA landed, 8 x converted,
 // 2 partial logits done, 3 logits reduced, 4 ticket, 9 score loads issued, 10 softmax,
 // 11 top-k, 5 scores, 12 coreset, 13 MaskOutside, 6 Algorithm 1, 7 dispatch; 16-24: steps
 // inside the dispatch, the coreset and MaskOutside (DMOE_STAMP in the shared headers);
@@ -34,7 +34,7 @@ __device__ uint64_t g_ctrace[64 * 8 * 64];
   do {                                                                                  \
     if (threadIdx.x == 0) {                                                             \
       const int c_ = ((blockIdx.y * gridDim.x + blockIdx.x) % 512) * 64 + (st);         \
-      if ((st) == 0 || (st) == 7) {                                                     \
+      if ((st) == 0 || (st) == 7 || (st) == 25) {                                       \
         uint64_t t_;                                                                    \
         asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t_));                          \
         g_ctrace[c_] = t_;                                                              \
