@@ -20,13 +20,15 @@
 // leave half of the SMs on down tiles only, and one SM's TMA rate, not HBM, would set the
 // pace of the gate/up stream; the 32-row units put a gate/up tile on every SM and keep the
 // weight bytes per SM near the mean. Every stage carries 32 KB of weights: K = 128 for
-// hg = 64 and for the down tiles, K = 256 for hg = 32 (four 128-B boxes per weight row,
-// which also streams faster from HBM than two).
+// hg = 64 and for the down tiles, K = 256 for hg = 32 (four 128-B boxes per weight row).
+// The combine launch that follows clears the group counters for the next call.
 //
-// Warp roles (192 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues MMAs, warps 2-5
-// run the epilogues (TMEM lane quadrant = warp % 4). Every wait is bounded (1 s): a timeout
-// is recorded and the CTA unwinds. The combine launch that follows clears the group
-// counters for the next call.
+// Warp roles (224 threads): warp 0 lane 0 issues TMA, lane 0 of warps 1 and 6 issue the MMAs
+// (each the first or second half of every stage's K boxes, into its own part of the
+// accumulator: one thread issues a tcgen05.mma only every ~58 cycles, whatever its shape,
+// and these chains are short), warps 2-5 run the epilogues (TMEM lane quadrant = warp % 4),
+// which add the two parts. Every wait is bounded (1 s): a timeout is recorded and the CTA
+// unwinds.
 #include <math.h>
 
 #include <mutex>
@@ -38,7 +40,7 @@
 namespace dmoe {
 namespace {
 
-constexpr int kThr = 192;
+constexpr int kThr = 224;
 constexpr int kKB = 2;                          // K boxes per down stage: K = 128
 constexpr int kStageK = kKB * kTileK;
 constexpr int kABox = kTileM * 128;             // 128 rows x 128 B (W_down)
@@ -56,7 +58,8 @@ constexpr int kMaxTok = 64;                     // tokens of a decode-sized forw
 // 6 H ready seen, 7 down MMAs committed, 8 down rows stored, 9 exit, 10 gate/up unit id,
 // 11 down unit id, 12/13 first/last down stage landed, 14 down accumulator ready, 15 down
 // accumulator staged, 16 staging complete, 17 row copies issued, 18 coresets seen by the
-// polling warp.
+// polling warp, 26/27 fourth / last gate/up stage landed, 28/29 first / last gate/up stage
+// issued.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_dtrace[kMaxPersistentCtas * 32];
 #define ED_AT(slot) (g_dtrace[blockIdx.x * 32 + (slot)] = ptx::globaltimer_ns())
@@ -155,13 +158,13 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   if (tid == 0) {
     for (int s = 0; s < kMaxStagesD; ++s) {
       ptx::mbar_init(&full[s], 1);
-      ptx::mbar_init(&empty[s], 1);
+      ptx::mbar_init(&empty[s], 2);       // both MMA issuers commit
     }
     for (int a = 0; a < 4; ++a) {
-      ptx::mbar_init(&acc_full[a], 1);
+      ptx::mbar_init(&acc_full[a], 2);
       ptx::mbar_init(&acc_empty[a], 128);
     }
-    ptx::mbar_init(drain, 1);
+    ptx::mbar_init(drain, 2);
     ptx::fence_mbarrier_init();
     *s_abort = 0;
   } else if (tid == 32) {
@@ -378,6 +381,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (first) ED_SET(10, u);
       for (int c = 0; c < kc; ++c) {
         if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+        if (first && c == 0) ED_AT(28);
+        if (first && c == kc - 1) ED_AT(29);
         ptx::mbar_arrive_expect_tx(&full[stage], kAStage + kbg * bbox);
         uint8_t* a_dst = slot_a(stage);
         uint8_t* b_dst = slot_b(stage);
@@ -477,32 +482,37 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
         }
       }
     }
-  } else if (warp == 1 && lane == 0) {
-    // ================= MMA issuer
+  } else if ((warp == 1 || warp == 6) && lane == 0) {
+    // ================= MMA issuers: `half` 0 takes the first half of every stage's K boxes
+    // into part 0 of the accumulator, `half` 1 the second half into part 1
+    const int half = warp == 6 ? 1 : 0;
     int stage = 0, acc = 0;
     uint32_t phase = 0, acc_phase = 0;
-    bool ok = true, first = true;
+    bool ok = true, first = half == 0;
     // nstages stages of kboxes K boxes each; A boxes abox bytes apart, M = mrows
     auto run = [&](int nstages, int kboxes, int abox, uint32_t mrows, int value, bool gu) {
       const uint32_t n_mma = (uint32_t)((p.T + 15) & ~15);
       const uint32_t idesc = ptx::idesc_bf16(mrows, n_mma);
       if (!wait(&acc_empty[acc], acc_phase ^ 1u, value)) { ok = false; return; }
       ptx::tc_fence_after();
-      const uint32_t d0 = tmem_base + (uint32_t)(acc * p.n_pad);
+      const uint32_t d0 = tmem_base + (uint32_t)((half * p.n_acc + acc) * p.n_pad);
+      const int kb0 = half * (kboxes / 2), kb1 = kb0 + kboxes / 2;
       for (int c = 0; c < nstages; ++c) {
         if (!wait(&full[stage], phase, value)) { ok = false; return; }
         if (gu && first && c == 0) ED_AT(2);
+        if (gu && first && c == 3) ED_AT(26);
+        if (gu && first && c == nstages - 1) ED_AT(27);
         if (!gu && first && c == 0) ED_AT(12);
         if (!gu && first && c == nstages - 1) ED_AT(13);
         ptx::tc_fence_after();
         const uint32_t a0 = ptx::smem_addr(slot_a(stage));
         const uint32_t b0 = ptx::smem_addr(slot_b(stage));
-        for (int kb = 0; kb < kboxes; ++kb)
+        for (int kb = kb0; kb < kb1; ++kb)
 #pragma unroll
           for (int kk = 0; kk < kTileK / 16; ++kk)
             ptx::mma_bf16(d0, ptx::sdesc_k_sw128(a0 + kb * abox + kk * 32),
                           ptx::sdesc_k_sw128(b0 + kb * bbox + kk * 32), idesc,
-                          (c > 0 || kb > 0 || kk > 0) ? 1u : 0u);
+                          (c > 0 || kb > kb0 || kk > 0) ? 1u : 0u);
         ptx::mma_commit(&empty[stage]);
         if (++stage == S) { stage = 0; phase ^= 1u; }
       }
@@ -517,7 +527,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (first) ED_AT(3);
       first = false;
     }
-    first = true;
+    first = half == 0;
     for (int v = v0; v < ND && ok; v += nb) {
       const Grp g = group_w(v / ndn);
       run(g.Ig / kStageK, kKB, kABox, (uint32_t)kTileM, v, false);
@@ -529,7 +539,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     const uint64_t t0 = ptx::globaltimer_ns();
     while (!ptx::mbar_try_wait(drain, 0) && ptx::globaltimer_ns() - t0 < kTimeoutNs) {
     }
-  } else if (warp >= 2) {
+  } else if (warp >= 2 && warp <= 5) {
     // ================= epilogue: warps 2..5, TMEM lanes 32*(warp%4) ..
     const int q = warp & 3;
     const int et = tid - 64;                      // 0..127
@@ -543,6 +553,19 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     const bool g_act = lane < rq;
     const int rr = (q & 1) * rq + lane;           // row within the hg-row slice
     const int n_mma = (p.T + 15) & ~15;
+    const uint32_t part1 = (uint32_t)(p.n_acc * p.n_pad);   // column offset of part 1
+    // 16 columns of an accumulator: the sum of its two parts
+    auto acc_ld16 = [&](uint32_t taddr, float (&v)[16]) {
+      float w[16];
+      ptx::tmem_ld16(taddr, v);
+      ptx::tmem_ld16(taddr + part1, w);
+      ptx::tmem_ld_wait();
+#pragma unroll
+      for (int c = 0; c < 16; ++c) {
+        asm volatile("" : "+f"(v[c]), "+f"(w[c]));   // the values exist only after the wait
+        v[c] += w[c];
+      }
+    };
     int acc = 0;
     uint32_t acc_phase = 0;
     bool first = true;
@@ -564,8 +587,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       uint8_t* hdst = hbox + (col0 >> 5) * p.n_pad * 64 + (col0 & 31) * 2;
       for (int c0 = 0; c0 < n_mma; c0 += 16) {
         float v[16];
-        ptx::tmem_ld16(tbase + c0, v);
-        ptx::tmem_ld_wait();
+        acc_ld16(tbase + c0, v);
         if (first && et == 0 && c0 == 0) ED_AT(23);
         if (g_act) {
           float* xr = xchg + ((is_gate ? 0 : hg) + rr) * kXStride;
@@ -644,8 +666,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       float* stg = stage_t;
       for (int c0 = 0; c0 < n_mma; c0 += 16) {
         float vv[16];
-        ptx::tmem_ld16(tbase + c0, vv);
-        ptx::tmem_ld_wait();
+        acc_ld16(tbase + c0, vv);
 #pragma unroll
         for (int c = 0; c < 16; ++c)
           if (c0 + c < p.T) stg[(c0 + c) * kTileM + row] = vv[c];
@@ -860,8 +881,8 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.ring_bytes = ring.bytes;
   p.h32_ok = ring.h32_ok;
   p.has_shared = has_shared ? 1 : 0;
-  p.n_acc = 512 / n_pad > 4 ? 4 : 512 / n_pad;
-  p.tmem_cols = pow2_cols((uint32_t)(p.n_acc * n_pad));
+  p.n_acc = 256 / n_pad > 4 ? 4 : 256 / n_pad;   // accumulators of two parts each
+  p.tmem_cols = pow2_cols((uint32_t)(2 * p.n_acc * n_pad));
   const size_t smem = (size_t)ring.bytes + fixed_smem(n_pad);
 
   static std::mutex mu;
