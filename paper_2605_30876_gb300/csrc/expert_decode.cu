@@ -58,8 +58,9 @@ constexpr int kMaxTok = 64;                     // tokens of a decode-sized forw
 // 6 H ready seen, 7 down MMAs committed, 8 down rows stored, 9 exit, 10 gate/up unit id,
 // 11 down unit id, 12/13 first/last down stage landed, 14 down accumulator ready, 15 down
 // accumulator staged, 16 staging complete, 17 row copies issued, 18 coresets seen by the
-// polling warp, 26/27 fourth / last gate/up stage landed, 28/29 first / last gate/up stage
-// issued.
+// polling warp, 19 its CTA past the barrier after the poll, 26/27 fourth / last gate/up
+// stage landed, 28/29 first / last gate/up stage issued, 30 past the TMEM barrier, 31 the
+// producer's cache policies made.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_dtrace[kMaxPersistentCtas * 32];
 #define ED_AT(slot) (g_dtrace[blockIdx.x * 32 + (slot)] = ptx::globaltimer_ns())
@@ -255,6 +256,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (lane == 0) *s_u = bad ? -1 : u_all;
     }
     __syncthreads();
+    if (tid == 0) ED_AT(19);
     spec = *s_u >= 0;
   }
   if (!spec) {
@@ -271,6 +273,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   ptx::tc_fence_before();
   __syncthreads();
   ptx::tc_fence_after();
+  if (tid == 0) ED_AT(30);
   const uint32_t tmem_base = *s_tmem;
   const int U = *s_u;
   const int G = U + has_shared;
@@ -365,6 +368,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     // ================= TMA producer
     const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
     const uint64_t pol_x = ptx::policy_evict_last();    // x and H: re-read by many tiles
+    ED_AT(31);
     int stage = 0, issued = 0;
     uint32_t phase = 0;
     bool ok = true;
