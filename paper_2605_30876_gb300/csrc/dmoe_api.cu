@@ -108,12 +108,14 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.xperm = take(2 * T * k * dm);
   w.h = take(2 * T * k * I);
   w.hs = take(2 * T * Is);
-  w.h_ready = take(sizeof(int32_t) * experts_ready_counters((int)T, (int)E, w.n_max));
+  // gate/up tile counters, then (block top-k on the general path) the rows copied per group
+  w.h_ready = take(sizeof(int32_t) * (experts_ready_counters((int)T, (int)E, w.n_max) + E + 1));
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
   const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
   w.hdense = take(dec ? 2 * (E + 1) * (size_t)((T + 15) / 16 * 16) * (I > Is ? I : Is) : 0);
-  w.spec = take(dec ? sizeof(uint32_t) * d.n_blocks * spec_words((int)k) : 0);
+  w.spec = take(dec || d.mode == DMOE_ROUTE_BLOCK
+                    ? sizeof(uint32_t) * d.n_blocks * spec_words((int)k) : 0);
   const size_t nchunks = (T + 31) / 32;
   w.disp_bits = take(sizeof(uint32_t) * nchunks * E);
   w.disp_base = take(sizeof(int32_t) * nchunks * E);
@@ -188,9 +190,12 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
                        const float* bias, int32_t* topk_idx, float* topk_gate, int32_t* coreset,
                        int32_t* coreset_size, float* probs, void* ws, const Workspace& plan,
                        cudaStream_t s, const L2Prefetch& shared_pf = L2Prefetch(),
-                       const DispatchArgs* dsp = nullptr, uint32_t* spec_words = nullptr) {
+                       const DispatchArgs* dsp = nullptr, uint32_t* spec_words = nullptr,
+                       int32_t* ready_clear = nullptr, int n_ready_clear = 0) {
   RouterArgs a{};
   a.spec_words = spec_words;
+  a.ready_clear = ready_clear;
+  a.n_ready_clear = n_ready_clear;
   a.x = static_cast<const __nv_bfloat16*>(x);
   a.w_r = w_r;
   a.bias = bias;
@@ -246,8 +251,14 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
                         const int32_t* offsets, const int32_t* rows, const int32_t* pos,
                         void* y, void* ws, const Workspace& plan, cudaStream_t s,
                         bool shared_prefetched = false, uint32_t* spec_words = nullptr,
-                        bool gathered = false) {
+                        bool gathered = false, int32_t* topk_idx = nullptr,
+                        int32_t* pos_out = nullptr, int32_t* n_unique_out = nullptr,
+                        int32_t* unique_ids_out = nullptr) {
   ExpertArgs a{};
+  a.topk_idx = topk_idx;
+  a.pos_out = pos_out;
+  a.n_unique_out = n_unique_out;
+  a.unique_ids_out = unique_ids_out;
   a.prefetch_shared = !shared_prefetched;
   a.gathered = gathered;
   a.spec_words = spec_words;
@@ -399,10 +410,12 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   set_dispatch_scratch(&dsp, workspace, plan);
   const int T_all = desc->n_blocks * desc->block_size;
   // general path: the dispatch placement also writes x in dispatch order and clears the
-  // expert launch's tile counters (no gather launch)
-  const bool gathered =
-      !route_cluster_ok(T_all, desc->d_model, desc->n_experts) &&
-      !experts_decode_ok(T_all, desc->d_model, desc->d_ff, desc->d_ff_shared);
+  // expert launch's tile counters (no gather launch); with block top-k the expert launch
+  // does the dispatch itself (spec_general)
+  const bool general = !route_cluster_ok(T_all, desc->d_model, desc->n_experts) &&
+                       !experts_decode_ok(T_all, desc->d_model, desc->d_ff, desc->d_ff_shared);
+  const bool spec_general = general && experts_spec_ok(*desc, plan.n_max);
+  const bool gathered = general && !spec_general;
   if (gathered) {
     dsp.x = static_cast<const __nv_bfloat16*>(x);
     dsp.xperm = at<__nv_bfloat16>(workspace, plan.xperm);
@@ -419,6 +432,17 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
       route_cluster_ok(T, desc->d_model, desc->n_experts) &&
       experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared)) {
     spec_w = at<uint32_t>(workspace, plan.spec);
+  }
+  if (spec_general) {
+    spec_w = at<uint32_t>(workspace, plan.spec);
+    st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
+                    shared_pf, nullptr, spec_w, at<int32_t>(workspace, plan.h_ready),
+                    experts_ready_counters(T, desc->n_experts, plan.n_max) +
+                        desc->n_experts + 1);
+    if (st != DMOE_OK) return st;
+    return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid,
+                       offs, rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w,
+                       false, idx, pos, nu, uid);
   }
   st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
                   shared_pf, &dsp, spec_w);
@@ -497,9 +521,12 @@ int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc) {
     n += 2;                                                   // dispatch: count, place
   }
   // experts and combine; the general experts' gather is a launch of its own only after the
-  // fused routing launch (otherwise the dispatch placement does it)
+  // fused routing launch (otherwise the dispatch placement does it); with block top-k on the
+  // general path the expert launch does the dispatch (no dispatch launches)
   const bool dec = experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared);
-  n += (!dec && route_cluster_ok(T, desc->d_model, desc->n_experts)) ? 3 : 2;
+  const bool cluster = route_cluster_ok(T, desc->d_model, desc->n_experts);
+  if (!cluster && !dec && experts_spec_ok(*desc, expert_n_max(*desc))) n -= 2;
+  n += (!dec && cluster) ? 3 : 2;
   return n;
 }
 

@@ -180,6 +180,11 @@ struct RouterArgs {
   // ids and a marker byte each, one 32-bit store per word (a word reads as zero until it is
   // complete; zero between calls); nullptr otherwise
   uint32_t* spec_words;
+  // with spec_words on the general path: the gate/up tile counters of the expert launch that
+  // follows, cleared by the block routing launch before it lets that launch start (the
+  // dispatch launches, which clear them otherwise, do not run then)
+  int32_t* ready_clear;
+  int n_ready_clear;
 };
 
 struct DispatchArgs {
@@ -253,11 +258,21 @@ struct ExpertArgs {
   // otherwise
   uint32_t* spec_words;
   int spec_blocks;
+  // general path with spec_words (block top-k): the expert launch writes the dispatch's
+  // outputs from the published coresets and the routing's topk_idx
+  const int32_t* topk_idx;
+  int32_t* pos_out;
+  int32_t* n_unique_out;
+  int32_t* unique_ids_out;
   // shape
   int T, d, E, k, I, Is, n_max;
 };
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s);
 int experts_ready_counters(int T, int E, int n_max);
+// Block top-k on the general path (every token keeps its block's whole coreset): the expert
+// launch plans from the coresets the block routing launch publishes, reads the token rows
+// from x block by block and writes the dispatch's outputs, so that no dispatch launch runs.
+bool experts_spec_ok(const dmoe_layer_desc& d, int n_max);
 // gate-weighted combine of the expert rows into y (the last launch of both expert paths);
 // it also clears zero[0 .. n_zero) and zero2[0 .. n_zero2) once the launch before it has
 // ended. meta_early: the slot indices and gates may be read before that launch ends (they

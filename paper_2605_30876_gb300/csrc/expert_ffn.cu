@@ -47,6 +47,8 @@ constexpr uint64_t kWaitTimeoutNs = 1000000000ull;  // 1 s
 constexpr int kMaxStages = 8;
 constexpr int64_t kDownPrefetchMax = (int64_t)64 << 20;   // half of the 129 MB L2
 constexpr int kXchgStride = 17;                    // floats per row of the exchange buffers
+constexpr int kSpecBlocks = 64;                    // blocks of a block top-k forward, at most
+constexpr int kSpecPairs = kSpecBlocks * kMaxTopK;   // (block, coreset member) pairs, at most
 
 struct GemmParams {
   const int32_t* n_unique;
@@ -72,6 +74,22 @@ struct GemmParams {
   int n_acc;              // accumulator buffers in TMEM
   uint32_t tmem_cols;
   int has_shared;
+  // Block top-k (spec_words != nullptr): the groups come from the coresets that the block
+  // routing launch publishes (n_blocks blocks of blk rows). The unique experts are their
+  // union, ascending; an expert's token rows are its blocks' rows in block order, which is
+  // the dispatch's order. This launch then does the dispatch itself: its CTAs copy every
+  // (block, coreset member) pair's rows of x to their place in xperm (x_ready[g] counts a
+  // group's copied rows; a gate/up unit loads them once they are all there) and write
+  // n_unique, unique_ids and pos (the row of every (token, slot), from topk_idx).
+  const uint32_t* spec_words;
+  int n_blocks, blk;
+  const int32_t* topk_idx;
+  int32_t* pos_out;
+  int32_t* n_unique_out;
+  int32_t* unique_ids_out;
+  int32_t* x_ready;          // [kMaxGroups], zero at the start (the routing launch clears it)
+  const __nv_bfloat16* x;
+  __nv_bfloat16* xperm;
 };
 
 struct Maps {
@@ -106,7 +124,8 @@ __device__ __forceinline__ bool epi_all_threads(bool v) {
 
 // Debug builds (-DDMOE_TRACE) record a per-CTA timeline of the expert kernel: slot 0 entry,
 // 1 after the unit list, 62 exit; for the i-th unit of the CTA (i < 8), at 2 + 6i: unit id,
-// producer start, last TMA issued, H ready (down units), last MMA commit, epilogue done;
+// producer start, last TMA issued, H ready (down units; for block top-k gate/up units: the
+// group's token rows copied), last MMA commit, epilogue done;
 // at 50 + i: the epilogue's first TMEM read of that unit.
 #ifdef DMOE_TRACE
 __device__ uint64_t g_trace[kMaxPersistentCtas * 64];
@@ -155,6 +174,12 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   int* g_row0 = dn_prefix + (kMaxGroups + 1);      // by group
   int* g_cnt = g_row0 + kMaxGroups;
   int* g_e = g_cnt + kMaxGroups;
+  // block top-k planning: blocks per expert (bit b of s_bmask[2e + b / 32]), each block's
+  // coreset, per expert its group and the blocks of the groups before it
+  uint32_t* s_bmask = reinterpret_cast<uint32_t*>(g_e + kMaxGroups);   // [2 * kMaxExperts]
+  int16_t* s_upos = reinterpret_cast<int16_t*>(s_bmask + 2 * kMaxExperts);   // [kMaxExperts]
+  int16_t* s_bpos = s_upos + kMaxExperts;                                      // [kMaxExperts]
+  uint8_t* s_bcore = reinterpret_cast<uint8_t*>(s_bpos + kMaxExperts);   // [kSpecPairs]
   float* xchg = reinterpret_cast<float*>(smem + off_x);
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -183,14 +208,95 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
-  pdl_wait();  // dispatch output and the gathered rows are complete from here on
+  const bool spec = p.spec_words != nullptr;
+  if (!spec) pdl_wait();  // dispatch output and the gathered rows are complete from here on
 
   // ---------------- groups and unit lists (slot 0 = the shared expert when present)
   if (warp == 0) {
-    int U = *p.n_unique;
-    if (U < 0 || U > p.E) {
-      if (lane == 0) record_error(p.err, kErrBadDispatch, kAtGateUp, U);
-      U = 0;
+    int U;
+    if (spec) {
+      // Block top-k: poll every block's published coreset words until all are nonzero (a
+      // nonzero word is complete), recording each block's members and, per expert, the
+      // blocks that use it
+      const int nw = spec_words(p.k), total = p.n_blocks * nw;
+      for (int i = lane; i < 2 * kMaxExperts; i += 32) s_bmask[i] = 0u;
+      __syncwarp();
+      bool bad = false;
+      const uint64_t t0 = ptx::globaltimer_ns();
+      for (;;) {
+        bool all = true;
+        for (int i = lane; i < total; i += 32) {
+          const uint32_t w = ptx::ld_relaxed_u32(p.spec_words + i);
+          if (w == 0u) {
+            all = false;
+            continue;
+          }
+          const int b = i / nw, r0 = 3 * (i % nw);
+#pragma unroll
+          for (int j = 0; j < 3; ++j) {
+            if (r0 + j >= p.k) break;
+            const int e = (int)((w >> (8 * j)) & 0xffu);
+            if (e >= p.E) {
+              bad = true;
+            } else {
+              s_bcore[b * p.k + r0 + j] = (uint8_t)e;
+              atomicOr(&s_bmask[2 * e + (b >> 5)], 1u << (b & 31));
+            }
+          }
+        }
+        if (__all_sync(0xffffffffu, all)) break;
+        if (ptx::globaltimer_ns() - t0 > kWaitTimeoutNs) {   // the coresets did not come
+          if (lane == 0) record_error(p.err, kErrTimeout, kAtGateUp, -1);
+          bad = true;
+          break;
+        }
+      }
+      bad = __any_sync(0xffffffffu, bad);
+      __syncwarp();
+      // the unique experts ascending (lane l: experts 8l .. 8l + 7): group u's rows are its
+      // blocks' rows, so it starts at blk * (blocks of the groups before it)
+      int nbq[8], cu = 0, cb = 0;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const int e = 8 * lane + q;
+        nbq[q] = e < p.E ? __popc(s_bmask[2 * e]) + __popc(s_bmask[2 * e + 1]) : 0;
+        cu += nbq[q] > 0 ? 1 : 0;
+        cb += nbq[q];
+      }
+      int iu = cu, ib = cb;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const int a = __shfl_up_sync(0xffffffffu, iu, o);
+        const int c = __shfl_up_sync(0xffffffffu, ib, o);
+        if (lane >= o) { iu += a; ib += c; }
+      }
+      int u = iu - cu, bp = ib - cb;
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        if (nbq[q] > 0) {
+          const int e = 8 * lane + q;
+          s_upos[e] = (int16_t)u;
+          s_bpos[e] = (int16_t)bp;
+          g_e[u] = e;
+          g_row0[u] = p.blk * bp;
+          g_cnt[u] = p.blk * nbq[q];
+          ++u;
+          bp += nbq[q];
+        }
+      U = bad ? 0 : __shfl_sync(0xffffffffu, iu, 31);
+      if (bad && lane == 0) record_error(p.err, kErrBadDispatch, kAtGateUp, -1);
+      if (lane == 0 && p.has_shared) {
+        g_row0[U] = 0;
+        g_cnt[U] = p.T;
+        g_e[U] = -1;
+      }
+      __syncwarp();
+    } else {
+      U = *p.n_unique;
+      if (U < 0 || U > p.E) {
+        if (lane == 0) record_error(p.err, kErrBadDispatch, kAtGateUp, U);
+        U = 0;
+      }
     }
     const int G = U + (p.has_shared ? 1 : 0);
     int carry_gu = 0, carry_dn = 0;
@@ -200,7 +306,12 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
       if (slot < G) {
         const int g = p.has_shared ? (slot == 0 ? U : slot - 1) : slot;
         int cnt, row0, e, Ig;
-        if (g < U) {
+        if (spec) {
+          cnt = g_cnt[g];
+          row0 = g_row0[g];
+          e = g_e[g];
+          Ig = g < U ? p.I : p.Is;
+        } else if (g < U) {
           row0 = p.offsets[g];
           cnt = p.offsets[g + 1] - row0;
           e = p.unique_ids[g];
@@ -279,7 +390,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     const int total = (int)(3 * per * U);
     if (pf.bytes * U <= kDownPrefetchMax)
       for (int c = (int)(2 * per * U) + blockIdx.x; c < total; c += gridDim.x)
-        l2_prefetch_chunk(pf, p.unique_ids, U, c);
+        l2_prefetch_chunk(pf, spec ? g_e : p.unique_ids, U, c);
     if (p.ws_gate != nullptr) {
       L2Prefetch sp;
       sp.ptr[0] = p.ws_gate;
@@ -356,18 +467,63 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           const CUtensorMap* mu = shared ? &tm.su : &tm.wu;
           const CUtensorMap* mb = shared ? &tm.x : (half ? &tm.xph : &tm.xp);
           const int kc = p.d / stage_k;
-          for (int c = 0; c < kc; ++c) {
-            if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
-            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
-            uint8_t* a_dst = smem + off_a + stage * a_stage;
-            uint8_t* b_dst = smem + off_b + stage * b_stage;
+          auto load_gu = [&](int st, int c, bool with_a, bool with_b) {
+            uint8_t* a_dst = smem + off_a + st * a_stage;
+            uint8_t* b_dst = smem + off_b + st * b_stage;
             for (int kb = 0; kb < kbs; ++kb) {
               const int kx = c * stage_k + kb * kTileK;
-              ptx::tma_load_2d(a_dst + kb * kATileBytes, mg, &full[stage], kx, arow, pol_w);
-              ptx::tma_load_2d(a_dst + kb * kATileBytes + kBoxBytes, mu, &full[stage], kx, arow,
-                               pol_w);
-              ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[stage], kx, brow, pol_x);
+              if (with_a) {
+                ptx::tma_load_2d(a_dst + kb * kATileBytes, mg, &full[st], kx, arow, pol_w);
+                ptx::tma_load_2d(a_dst + kb * kATileBytes + kBoxBytes, mu, &full[st], kx, arow,
+                                 pol_w);
+              }
+              if (with_b) ptx::tma_load_2d(b_dst + kb * b_box, mb, &full[st], kx, brow, pol_x);
             }
+          };
+          int c0 = 0;
+          if (spec && !shared) {
+            // block top-k: the weight stages first, the token rows once this launch's copies
+            // of the group's rows are all in xperm
+            const int pre = kc < stages ? kc : stages;
+            const int stage0 = stage;
+            for (int c = 0; c < pre; ++c) {
+              if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+              ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
+              load_gu(stage, c, true, false);
+              ++issued;
+              if (++stage == stages) { stage = 0; phase ^= 1u; }
+            }
+            if (!ok) break;
+            const int32_t* flag = p.x_ready + un.g;
+            if (ld_acquire(flag) < g_cnt[un.g]) {
+              const uint64_t t0 = ptx::globaltimer_ns();
+              while (ld_acquire(flag) < g_cnt[un.g]) {
+                if (*s_abort) { ok = false; break; }
+                if (ptx::globaltimer_ns() - t0 > kWaitTimeoutNs) {
+                  record_error(p.err, kErrTimeout, kAtGather, u);
+                  *s_abort = 1;
+                  ok = false;
+                  break;
+                }
+              }
+            }
+            fence_proxy_async_global();   // the copies (generic stores) before these loads
+            if (li < 8) DMOE_TRACE_AT(5 + 6 * li);
+            int st = stage0;
+            for (int c = 0; c < pre; ++c) {
+              if (ok)
+                load_gu(st, c, false, true);
+              else
+                ptx::mbar_complete_tx_local(&full[st], b_bytes);   // keep the accounting whole
+              if (++st == stages) st = 0;
+            }
+            if (!ok) break;
+            c0 = pre;
+          }
+          for (int c = c0; c < kc; ++c) {
+            if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
+            ptx::mbar_arrive_expect_tx(&full[stage], tx_bytes);
+            load_gu(stage, c, true, true);
             ++issued;
             if (++stage == stages) { stage = 0; phase ^= 1u; }
           }
@@ -541,6 +697,72 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     // (warps 2-5 and 6-9) take alternate 16-column slices of the accumulator, each with its
     // own exchange tile and named barrier (the epilogue math is latency-bound: two groups
     // finish a tile in about half the time)
+    if (spec && U > 0) {
+      // this CTA's share of the dispatch's copies: the rows of pair (block b, coreset member
+      // e) go to xperm rows blk * (s_bpos[e] + rank of b among e's blocks), a pair split into
+      // up to four parts when the pairs are fewer than the CTAs; the group counts its copied
+      // rows (one release add per part, after every epilogue thread's stores)
+      const int et = tid - 64;
+      const int npairs = p.n_blocks * p.k;
+      int parts = (int)gridDim.x / npairs;
+      parts = parts < 1 ? 1 : (parts > 4 ? 4 : parts);
+      while (p.blk % parts != 0) --parts;
+      const int prow = p.blk / parts;                 // rows per part
+      const int n16 = prow * p.d / 8;                 // 16-byte pieces per part
+      for (int w = blockIdx.x; w < npairs * parts; w += gridDim.x) {
+        const int i = w / parts, part = w - i * parts;
+        const int b = i / p.k, e = s_bcore[i];
+        const uint32_t lo = s_bmask[2 * e], hi = s_bmask[2 * e + 1];
+        const int rank = b < 32 ? __popc(lo & ((1u << b) - 1u))
+                                : __popc(lo) + __popc(hi & ((1u << (b - 32)) - 1u));
+        const uint4* src = reinterpret_cast<const uint4*>(
+            p.x + ((size_t)b * p.blk + (size_t)part * prow) * p.d);
+        uint4* dst = reinterpret_cast<uint4*>(
+            p.xperm + ((size_t)p.blk * (s_bpos[e] + rank) + (size_t)part * prow) * p.d);
+        for (int v0 = et; v0 < n16; v0 += kEpiThreads * 16) {
+          uint4 r[16];
+#pragma unroll
+          for (int q = 0; q < 16; ++q)
+            if (v0 + q * kEpiThreads < n16) r[q] = __ldg(src + v0 + q * kEpiThreads);
+#pragma unroll
+          for (int q = 0; q < 16; ++q)
+            if (v0 + q * kEpiThreads < n16) dst[v0 + q * kEpiThreads] = r[q];
+        }
+        __threadfence();
+        named_bar_sync(4, kEpiThreads);
+        if (et == 0) red_release_add(p.x_ready + s_upos[e], prow);
+      }
+    }
+    if (spec && warp == 2) {
+      // the dispatch's outputs: the row of every (token, slot) of this CTA's share of the
+      // tokens (expert e = topk_idx[t, j] of block b: the group's rows start at
+      // blk * s_bpos[e], block b is its rank-th block), once the routing launch has ended
+      pdl_wait();
+      const int per = (p.T + (int)gridDim.x - 1) / (int)gridDim.x;
+      const int t_begin = (int)blockIdx.x * per;
+      const int t_end = min(p.T, t_begin + per);
+      for (int i = t_begin * p.k + lane; i < t_end * p.k; i += 32) {
+        const int t = i / p.k, b = t / p.blk;
+        const int e = __ldcg(p.topk_idx + i);
+        int r = -1;
+        if (U > 0 && e >= 0 && e < p.E && b < p.n_blocks) {
+          const uint32_t lo = s_bmask[2 * e], hi = s_bmask[2 * e + 1];
+          const bool in = b < 32 ? ((lo >> b) & 1u) != 0u : ((hi >> (b - 32)) & 1u) != 0u;
+          const int rank = b < 32 ? __popc(lo & ((1u << b) - 1u))
+                                  : __popc(lo) + __popc(hi & ((1u << (b - 32)) - 1u));
+          if (in) r = p.blk * (s_bpos[e] + rank) + (t - b * p.blk);
+        }
+        if (r < 0) {
+          record_error(p.err, kErrBadDispatch, kAtDown, i);
+          r = 0;
+        }
+        p.pos_out[i] = r;
+      }
+      if (blockIdx.x == 0) {
+        if (lane == 0) *p.n_unique_out = U;
+        for (int u = lane; u < p.E; u += 32) p.unique_ids_out[u] = u < U ? g_e[u] : -1;
+      }
+    }
     const int q = warp & 3;
     const int cg = (warp - 2) >> 2;                 // column group
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
@@ -820,9 +1042,10 @@ uint32_t pow2_cols(uint32_t c) {
 }
 
 size_t experts_fixed_smem() {
-  // alignment slack + exchange buffers + barriers + misc/group arrays
+  // alignment slack + exchange buffers + barriers + misc/group arrays + block top-k planning
   return 1024 + 2 * 128 * kXchgStride * 4 + 8 + 8 * (2 * kMaxStages + 9) +
-         sizeof(int) * (12 + 5 * (kMaxGroups + 1)) + 64;
+         sizeof(int) * (12 + 5 * (kMaxGroups + 1)) + 64 + 4 * 2 * kMaxExperts +
+         2 * 2 * kMaxExperts + kSpecPairs;
 }
 
 int max_smem_optin() {
@@ -850,13 +1073,23 @@ int experts_ready_counters(int T, int E, int n_max) {
   return (E + 1) * ((T + n_max - 1) / n_max);
 }
 
+bool experts_spec_ok(const dmoe_layer_desc& d, int n_max) {
+  // blocks of whole 8-row groups (a block's box starts on a 1 KB swizzle boundary), whole
+  // blocks per token tile, at most kSpecBlocks blocks (a 64-bit block mask per expert)
+  return d.mode == DMOE_ROUTE_BLOCK && d.top_p <= 0.f && mask_top_k(d) == d.top_k &&
+         d.n_blocks >= 1 && d.n_blocks <= kSpecBlocks && d.block_size % 8 == 0 &&
+         n_max % d.block_size == 0 && d.n_experts <= kMaxExperts;
+}
+
 cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   const int pairs = a.T * a.k;
   const bool has_shared = a.Is > 0;
   const int n_ready = experts_ready_counters(a.T, a.E, a.n_max);
+  const bool spec = a.spec_words != nullptr;
   // 1. gather x in dispatch order; clear the gate/up tile counters (unless the dispatch
-  //    placement of the fused layer call has done both)
-  if (!a.gathered) {
+  //    placement of the fused layer call has done both, or, for block top-k, the block
+  //    routing launch has cleared them and the token rows are read from x by block)
+  if (!a.gathered && !spec) {
     const int grid = pairs < 1024 ? pairs : 1024;
     prof_begin(DMOE_KERNEL_GATHER, s);
     cudaError_t e = launch_ex(gather_kernel, dim3(grid), dim3(256), 0, s, true, a.x, a.rows,
@@ -890,6 +1123,18 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   gp.dpair = (gp.kbs == 2 && (a.d / kTileM) % 2 == 0) ? 2 : 1;
   gp.ntiles = (a.T + a.n_max - 1) / a.n_max;
   gp.has_shared = has_shared ? 1 : 0;
+  if (spec) {
+    gp.spec_words = a.spec_words;
+    gp.n_blocks = a.spec_blocks;
+    gp.blk = a.T / a.spec_blocks;
+    gp.topk_idx = a.topk_idx;
+    gp.pos_out = a.pos_out;
+    gp.n_unique_out = a.n_unique_out;
+    gp.unique_ids_out = a.unique_ids_out;
+    gp.x_ready = a.h_ready + experts_ready_counters(a.T, a.E, a.n_max);
+    gp.x = a.x;
+    gp.xperm = a.xperm;
+  }
 
   // 2. gate/up + SwiGLU and down projection in one persistent launch
   Maps m;
@@ -930,6 +1175,9 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
     if (dev < 31) attr_dev_mask |= 1 << dev;
   }
   int grid = device_sm_count();
+  // block top-k with few blocks: the CTAs start while the block routing launch (one CTA
+  // per block) still runs; leave its SMs free, so that no CTA starts only when it ends
+  if (spec && a.spec_blocks <= 16 && grid > 4 * a.spec_blocks) grid -= a.spec_blocks;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
   cudaError_t e = launch_ex(moe_experts_kernel, dim3(grid), dim3(kThreads), smem, s,

@@ -456,12 +456,7 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
         // block top-k: the coreset (k experts) is the routing of every token of the block;
         // publish it for the expert launch, three ids and a marker byte per word
         const int nw = spec_words(k);
-        if (tid < nw) {
-          uint32_t w = 1u << 24;
-          for (int j = 0; j < 3 && 3 * tid + j < k; ++j) w |= (uint32_t)order[3 * tid + j] << (8 * j);
-          asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(a.spec_words + (size_t)b * nw + tid),
-                       "r"(w) : "memory");
-        }
+        if (tid < nw) publish_coreset(a.spec_words + (size_t)b * nw, order, k, tid);
       }
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order

@@ -122,13 +122,24 @@ __global__ void __launch_bounds__(256)
 block_route_kernel(const float* __restrict__ probs, const float* __restrict__ probs_hat,
                    int E, int kb, int k, int B, float top_p,
                    int32_t* __restrict__ topk_idx, float* __restrict__ topk_gate,
-                   int32_t* __restrict__ coreset, int32_t* __restrict__ coreset_size) {
+                   int32_t* __restrict__ coreset, int32_t* __restrict__ coreset_size,
+                   uint32_t* __restrict__ spec, int32_t* __restrict__ ready, int n_ready) {
   pdl_wait();
+  if (spec != nullptr) {
+    // the expert launch that follows polls this block's coreset words and counts on its
+    // gate/up tile counters being zero: both are cleared, and made visible, before this CTA
+    // lets it start (the previous call has ended: the wait above)
+    if ((int)threadIdx.x < spec_words(k)) spec[(size_t)blockIdx.x * spec_words(k) + threadIdx.x] = 0u;
+    if (blockIdx.x == 0)
+      for (int i = threadIdx.x; i < n_ready; i += blockDim.x) ready[i] = 0;
+    __threadfence();
+    __syncthreads();
+  }
   pdl_launch_dependents();   // after the wait: a waiting dependent would share the SMs
   KLOG(6, 0);
   DMOE_STAMP(0);
   block_route_cta(blockIdx.x, probs, probs_hat, E, kb, k, B, top_p, topk_idx, topk_gate, coreset,
-                  coreset_size);
+                  coreset_size, spec);
   KLOG(6, 1);
 }
 
@@ -170,7 +181,7 @@ cudaError_t launch_router(const RouterArgs& a, const DispatchArgs* dsp, int32_t*
     if (a.mode == DMOE_ROUTE_BLOCK) {
       e = launch_ex(block_route_kernel, dim3(a.n_blocks), dim3(256), 0, s, true, a.probs,
                     a.probs_hat, a.E, a.kb, a.k, a.B, a.top_p, a.topk_idx, a.topk_gate, a.coreset,
-                    a.coreset_size);
+                    a.coreset_size, a.spec_words, a.ready_clear, a.n_ready_clear);
       if (e != cudaSuccess) return e;
     } else {
       if (a.coreset != nullptr)

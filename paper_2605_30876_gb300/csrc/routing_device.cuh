@@ -451,12 +451,26 @@ __device__ inline void mask_topk_warps(int k, int B, int size, const int* order,
   }
 }
 
+// Block top-k publication: the block's coreset (its k members, best first), three 8-bit ids
+// and a marker byte per 32-bit word, one relaxed store per word (a word reads as zero until
+// it is complete). Called by threads 0 .. spec_words(k) - 1.
+__device__ inline void publish_coreset(uint32_t* __restrict__ words, const int* order, int k,
+                                       int i) {
+  uint32_t w = 1u << 24;
+  for (int j = 0; j < 3 && 3 * i + j < k; ++j) w |= (uint32_t)order[3 * i + j] << (8 * j);
+  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(words + i), "r"(w) : "memory");
+}
+
 template <class HatFn, class ProbFn, class OutFn>
 __device__ inline void block_route_steps(int E, int kb, int k, int B, float top_p, HatFn hat,
                                          ProbFn prob, OutFn out, int32_t* __restrict__ coreset,
-                                         int32_t* __restrict__ coreset_size) {
+                                         int32_t* __restrict__ coreset_size,
+                                         uint32_t* __restrict__ spec = nullptr) {
   __shared__ int order[kMaxExperts];
   const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size);
+  // block top-k (the coreset is every token's routing): published for the expert launch
+  if (spec != nullptr && size == k && (int)threadIdx.x < spec_words(k))
+    publish_coreset(spec, order, k, threadIdx.x);
   DMOE_STAMP(25);
   mask_topk_warps(k, B, size, order, prob, out);
   __syncthreads();
@@ -470,7 +484,8 @@ __device__ inline void block_route_cta(int b, const float* probs, const float* p
                                        int32_t* __restrict__ topk_idx,
                                        float* __restrict__ topk_gate,
                                        int32_t* __restrict__ coreset,
-                                       int32_t* __restrict__ coreset_size) {
+                                       int32_t* __restrict__ coreset_size,
+                                       uint32_t* __restrict__ spec = nullptr) {
   const size_t r0 = (size_t)b * B;
   block_route_steps(
       E, kb, k, B, top_p,
@@ -481,7 +496,8 @@ __device__ inline void block_route_cta(int b, const float* probs, const float* p
         topk_gate[(r0 + i) * k + r] = g;
       },
       coreset != nullptr ? coreset + (size_t)b * E : nullptr,
-      coreset_size != nullptr ? coreset_size + b : nullptr);
+      coreset_size != nullptr ? coreset_size + b : nullptr,
+      spec != nullptr ? spec + (size_t)b * spec_words(k) : nullptr);
 }
 
 }  // namespace dmoe

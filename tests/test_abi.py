@@ -108,8 +108,11 @@ def test_null_and_misaligned_pointers_are_rejected_before_launch(dm):
 def test_layer_forward_launch_count(dm):
     # decode-size forward: one routing launch (dispatch fused), the expert launch, the combine
     assert dm.dmoe_layer_forward_launches(_desc(dm)) == 3
-    # 2048 tokens: split of W_r, logits, softmax / top-k, Algorithm 1, dispatch (count,
-    # place with the gather); experts, combine
-    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64)) == 8
+    # 2048 tokens, block top-k: split of W_r, logits, softmax / top-k, Algorithm 1 (which
+    # publishes the coresets); experts (which do the dispatch), combine
+    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64)) == 6
+    # with p > 0 (a token keeps part of the coreset): dispatch (count, place with the
+    # gather) before the experts
+    assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64, top_p=0.6)) == 8
     assert dm.dmoe_layer_forward_launches(_desc(dm, n_blocks=64, mode=dm.DMOE_ROUTE_TOKEN)) == 7
     assert dm.dmoe_layer_forward_launches(_desc(dm, top_k=0)) == -1
