@@ -109,6 +109,20 @@ dmoe_status dmoe_router(const dmoe_layer_desc* desc, const void* x, const float*
                         int32_t* coreset, int32_t* coreset_size, float* probs,
                         void* workspace, size_t workspace_bytes, void* stream);
 
+/* Router weight preparation (optional, once per W_r, like a weight layout conversion at
+ * load time). Forwards of more than 64 tokens compute the fp32 router logits of §4.2 on
+ * the tensor cores from an exact three-part bf16 split of W_r (hi + mid + lo = w to 2^-27),
+ * which every router or layer call otherwise writes into the workspace first. This call
+ * writes that split into the workspace and remembers on the host that the workspace holds
+ * it for this w_r pointer; router and layer calls on the workspace with the same w_r then
+ * skip the split. Call it again after changing W_r in place. A call with another w_r
+ * splits that one, and the workspace then no longer holds this one's split. A no-op for
+ * shapes whose router reads W_r directly.
+ *   w_r      fp32 [d, E]     device, router weight (read)
+ *   workspace                as for dmoe_router; stream: the CUDA stream of the split */
+dmoe_status dmoe_router_prepare(const dmoe_layer_desc* desc, const float* w_r, void* workspace,
+                                size_t workspace_bytes, void* stream);
+
 /* Dispatch: the unique experts of one forward (the "unique expert count" of §3 and §5)
  * and the expert -> (token, slot) lists, computed on the device without a host round-trip.
  *   topk_idx   int32 [T, k]   routed experts (e.g. from dmoe_router); every id must be in
@@ -158,8 +172,9 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x,
                                void* workspace, size_t workspace_bytes, void* stream);
 
 /* Number of kernel launches one dmoe_layer_forward call makes for `desc` (the decode-size
- * path: routing 1, experts 1, combine 1). Returns -1 for an invalid or unsupported desc.
- * Host-only, no GPU needed. */
+ * path: routing 1, experts 1, combine 1), counting the split of W_r where the router uses
+ * it: a call on a workspace that dmoe_router_prepare prepared for its W_r makes one launch
+ * fewer then. Returns -1 for an invalid or unsupported desc. Host-only, no GPU needed. */
 int32_t dmoe_layer_forward_launches(const dmoe_layer_desc* desc);
 
 /* Kernels of the forward, for dmoe_set_profile_events. */

@@ -76,6 +76,8 @@ def _load() -> ctypes.CDLL:
     lib.dmoe_workspace_size.restype = st
     lib.dmoe_router.argtypes = [D, P, P, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.dmoe_router.restype = st
+    lib.dmoe_router_prepare.argtypes = [D, P, P, ctypes.c_size_t, P]
+    lib.dmoe_router_prepare.restype = st
     lib.dmoe_dispatch.argtypes = [D, P, P, P, P, P, P, P, ctypes.c_size_t, P]
     lib.dmoe_dispatch.restype = st
     lib.dmoe_moe_forward.argtypes = [D] + [P] * 14 + [P, ctypes.c_size_t, P]
@@ -167,6 +169,12 @@ def dmoe_router(desc, x, w_r, bias, topk_idx, topk_gate, coreset=None, coreset_s
                             _ptr(coreset_size, torch.int32, "coreset_size"),
                             _ptr(probs, torch.float32, "probs"), ws, nb, _stream(stream)),
            "dmoe_router")
+
+
+def dmoe_router_prepare(desc, w_r, workspace, stream=None) -> None:
+    ws, nb = _ws(workspace)
+    _check(_lib.dmoe_router_prepare(ctypes.byref(desc), _ptr(w_r, torch.float32, "w_r"), ws, nb,
+                                    _stream(stream)), "dmoe_router_prepare")
 
 
 def dmoe_dispatch(desc, topk_idx, n_unique, unique_ids, offsets, rows, pos, workspace=None,

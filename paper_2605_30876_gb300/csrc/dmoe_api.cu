@@ -3,12 +3,30 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
+#include <unordered_map>
+
 #include "dmoe_internal.cuh"
 
 namespace dmoe {
 
 namespace {
 thread_local char g_last_error[256] = "";
+
+// Workspaces whose W_r parts were written by dmoe_router_prepare, with the W_r they hold.
+std::mutex g_prep_mu;
+std::unordered_map<const void*, const void*> g_prep;
+
+// Does `ws` hold the parts of `w_r`? If not, the split this call makes writes w_r's parts
+// there, so an earlier preparation of the workspace no longer holds.
+bool parts_prepared(const void* ws, const void* w_r) {
+  std::lock_guard<std::mutex> lock(g_prep_mu);
+  auto it = g_prep.find(ws);
+  if (it == g_prep.end()) return false;
+  if (it->second == w_r) return true;
+  g_prep.erase(it);
+  return false;
+}
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
@@ -221,6 +239,7 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
   a.err = at<DevErrRecord>(ws, plan.err);
   a.shared_pf = shared_pf;
   a.w_parts = plan.w_parts_bytes > 0 ? at<__nv_bfloat16>(ws, plan.w_parts) : nullptr;
+  a.parts_ready = a.w_parts != nullptr && parts_prepared(ws, w_r);
   a.tc_splits = plan.tc_splits;
   a.tc_part = plan.tc_splits > 0 ? at<float>(ws, plan.tc_part) : nullptr;
   return cuda_status(launch_router(a, dsp, at<int32_t>(ws, plan.tickets), s));
@@ -325,6 +344,28 @@ dmoe_status dmoe_router(const dmoe_layer_desc* desc, const void* x, const float*
   if (st != DMOE_OK) return st;
   return run_router(desc, x, w_r, bias, topk_idx, topk_gate, coreset, coreset_size, probs,
                     workspace, plan, static_cast<cudaStream_t>(stream));
+}
+
+dmoe_status dmoe_router_prepare(const dmoe_layer_desc* desc, const float* w_r, void* workspace,
+                                size_t workspace_bytes, void* stream) {
+  dmoe_status st = check_desc(desc);
+  if (st != DMOE_OK) return st;
+  if (!all_aligned({w_r})) return DMOE_ERR_INVALID_ARG;
+  Workspace plan;
+  st = check_ws(desc, workspace, workspace_bytes, &plan);
+  if (st != DMOE_OK) return st;
+  {
+    std::lock_guard<std::mutex> lock(g_prep_mu);
+    g_prep.erase(workspace);
+  }
+  if (plan.w_parts_bytes == 0) return DMOE_OK;   // this shape's router reads W_r itself
+  const cudaError_t e = launch_router_wsplit(w_r, at<__nv_bfloat16>(workspace, plan.w_parts),
+                                             desc->d_model, desc->n_experts,
+                                             static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_status(e);
+  std::lock_guard<std::mutex> lock(g_prep_mu);
+  g_prep[workspace] = w_r;
+  return DMOE_OK;
 }
 
 dmoe_status dmoe_dispatch(const dmoe_layer_desc* desc, const int32_t* topk_idx,

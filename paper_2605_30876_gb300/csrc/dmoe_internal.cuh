@@ -175,6 +175,7 @@ struct RouterArgs {
                           // (then the mma.sync / FFMA logits run)
   int tc_splits;          // slices of d of the tcgen05 logits
   float* tc_part;         // [tc_splits, T, E]: their partial sums
+  bool parts_ready;       // w_parts already holds this W_r's split (dmoe_router_prepare)
   // block top-k (p <= 0) in the fused decode-size call: every block's coreset, which is
   // then the block's routing, is published early here: spec_words(k) words per block, three
   // ids and a marker byte each, one 32-bit store per word (a word reads as zero until it is
@@ -232,6 +233,9 @@ bool router_tc_ok(int T, int d, int E);
 int router_tc_splits(int T, int d);
 size_t router_tc_parts_bytes(int d, int E);
 cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s);
+// The split of W_r into its three bf16 parts (the first launch of launch_router_tc).
+cudaError_t launch_router_wsplit(const float* w_r, __nv_bfloat16* parts, int d, int E,
+                                 cudaStream_t s);
 cudaError_t launch_route_cluster(const RouterArgs& a, const DispatchArgs* dsp, int32_t* tickets,
                                  cudaStream_t s);
 

@@ -126,7 +126,8 @@ __device__ __forceinline__ bool epi_all_threads(bool v) {
 // 1 after the unit list, 62 exit; for the i-th unit of the CTA (i < 8), at 2 + 6i: unit id,
 // producer start, last TMA issued, H ready (down units; for block top-k gate/up units: the
 // group's token rows copied), last MMA commit, epilogue done;
-// at 50 + i: the epilogue's first TMEM read of that unit.
+// at 50 + i: the epilogue's first TMEM read of that unit; 63: this CTA's copies of the
+// token rows done (block top-k).
 #ifdef DMOE_TRACE
 __device__ uint64_t g_trace[kMaxPersistentCtas * 64];
 #define DMOE_TRACE_AT(slot) (g_trace[blockIdx.x * 64 + (slot)] = ptx::globaltimer_ns())
@@ -142,7 +143,10 @@ __device__ uint64_t g_trace[kMaxPersistentCtas * 64];
 // blockIdx.x, blockIdx.x + gridDim.x, ... so its gate/up units always precede its down
 // units and a gate/up unit never waits on another unit. A down unit loads its W_down
 // tiles at once and only then waits (bounded) for the gate/up tiles of its token rows to
-// be published (h_ready), so weight streaming of both phases overlaps.
+// be published (h_ready), so weight streaming of both phases overlaps. kSpec: the block
+// top-k form (GemmParams::spec_words), compiled separately so that the other form carries
+// none of its code.
+template <bool kSpec>
 __global__ void __launch_bounds__(kThreads, 1)
 moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -208,7 +212,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     ptx::tmem_alloc(s_tmem, p.tmem_cols);
     ptx::tmem_relinquish();
   }
-  const bool spec = p.spec_words != nullptr;
+  constexpr bool spec = kSpec;
   if (!spec) pdl_wait();  // dispatch output and the gathered rows are complete from here on
 
   // ---------------- groups and unit lists (slot 0 = the shared expert when present)
@@ -719,19 +723,20 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
             p.x + ((size_t)b * p.blk + (size_t)part * prow) * p.d);
         uint4* dst = reinterpret_cast<uint4*>(
             p.xperm + ((size_t)p.blk * (s_bpos[e] + rank) + (size_t)part * prow) * p.d);
-        for (int v0 = et; v0 < n16; v0 += kEpiThreads * 16) {
-          uint4 r[16];
+        for (int v0 = et; v0 < n16; v0 += kEpiThreads * 8) {
+          uint4 r[8];
 #pragma unroll
-          for (int q = 0; q < 16; ++q)
+          for (int q = 0; q < 8; ++q)
             if (v0 + q * kEpiThreads < n16) r[q] = __ldg(src + v0 + q * kEpiThreads);
 #pragma unroll
-          for (int q = 0; q < 16; ++q)
+          for (int q = 0; q < 8; ++q)
             if (v0 + q * kEpiThreads < n16) dst[v0 + q * kEpiThreads] = r[q];
         }
         __threadfence();
         named_bar_sync(4, kEpiThreads);
         if (et == 0) red_release_add(p.x_ready + s_upos[e], prow);
       }
+      if (et == 0) DMOE_TRACE_AT(63);
     }
     if (spec && warp == 2) {
       // the dispatch's outputs: the row of every (token, slot) of this CTA's share of the
@@ -1169,8 +1174,11 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   int dev = 0;
   cudaGetDevice(&dev);
   if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
-    cudaError_t e = cudaFuncSetAttribute(moe_experts_kernel,
+    cudaError_t e = cudaFuncSetAttribute(moe_experts_kernel<false>,
                                          cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(moe_experts_kernel<true>,
+                               cudaFuncAttributeMaxDynamicSharedMemorySize, limit);
     if (e != cudaSuccess) return e;
     if (dev < 31) attr_dev_mask |= 1 << dev;
   }
@@ -1180,8 +1188,10 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   if (spec && a.spec_blocks <= 16 && grid > 4 * a.spec_blocks) grid -= a.spec_blocks;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
-  cudaError_t e = launch_ex(moe_experts_kernel, dim3(grid), dim3(kThreads), smem, s,
-                            !prof_serial(DMOE_KERNEL_EXPERTS), m, gp);
+  cudaError_t e = spec ? launch_ex(moe_experts_kernel<true>, dim3(grid), dim3(kThreads), smem, s,
+                                   !prof_serial(DMOE_KERNEL_EXPERTS), m, gp)
+                        : launch_ex(moe_experts_kernel<false>, dim3(grid), dim3(kThreads), smem,
+                                    s, !prof_serial(DMOE_KERNEL_EXPERTS), m, gp);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
 

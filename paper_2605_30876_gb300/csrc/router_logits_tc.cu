@@ -67,15 +67,20 @@ router_wsplit_kernel(const float* __restrict__ w_r, __nv_bfloat16* __restrict__ 
                      int E) {
   const int e = blockIdx.x * 32 + (threadIdx.x & 31);
   const int k0 = blockIdx.y * 64 + (threadIdx.x >> 5) * 8;
-  // No dependency wait: this launch reads only W_r (an input) and writes only the parts,
-  // which only the logits launch of an earlier call reads. That launch is always followed
-  // by router_softmax_kernel, which releases its dependents only after its own dependency
-  // wait (the logits launch has ended by then); so by the time any later launch, this one
-  // included, can start, the earlier logits launch has ended. The logits launch after
-  // this one waits for it.
+  // The split needs no dependency wait: this launch reads only W_r (an input) and writes
+  // only the parts, which only the logits launch of an earlier call reads. That launch is
+  // always followed by router_softmax_kernel, which releases its dependents only after its
+  // own dependency wait (the logits launch has ended by then); so by the time any later
+  // launch, this one included, can start, the earlier logits launch has ended. The wait at
+  // the end makes this launch end only after the launch before it, so that the logits
+  // launch after this one, which waits for this one, also reads x only after the launch
+  // that may have written it.
   pdl_launch_dependents();
   KLOG(8, 0);
-  if (e >= E) return;
+  if (e >= E) {
+    pdl_wait();
+    return;
+  }
   float w[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) w[j] = w_r[(size_t)(k0 + j) * E + e];
@@ -98,6 +103,7 @@ router_wsplit_kernel(const float* __restrict__ w_r, __nv_bfloat16* __restrict__ 
   *reinterpret_cast<uint4*>(parts + pe + o) = make_uint4(mp[0], mp[1], mp[2], mp[3]);
   *reinterpret_cast<uint4*>(parts + 2 * pe + o) = make_uint4(lp[0], lp[1], lp[2], lp[3]);
   KLOG(8, 1);
+  pdl_wait();
 }
 
 __global__ void __launch_bounds__(kLtThreads, 1)
@@ -314,6 +320,12 @@ int router_tc_splits(int T, int d) {
 
 size_t router_tc_parts_bytes(int d, int E) { return (size_t)3 * E * d * 2; }
 
+cudaError_t launch_router_wsplit(const float* w_r, __nv_bfloat16* parts, int d, int E,
+                                 cudaStream_t s) {
+  return launch_ex(router_wsplit_kernel, dim3((E + 31) / 32, d / 64), dim3(256), 0, s, true, w_r,
+                   parts, d, E);
+}
+
 cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
   if (!router_tc_ok(a.T, a.d, a.E) || a.w_parts == nullptr || a.tc_part == nullptr || splits < 1 ||
       (a.d / kLtKC) % splits != 0 || a.d / splits > kLtMaxDS)
@@ -331,9 +343,11 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
   f.d = a.d;
   f.E = a.E;
   f.ds = a.d / splits;
-  cudaError_t e = launch_ex(router_wsplit_kernel, dim3((a.E + 31) / 32, a.d / 64), dim3(256), 0,
-                            s, true, a.w_r, a.w_parts, a.d, a.E);
-  if (e != cudaSuccess) return e;
+  cudaError_t e = cudaSuccess;
+  if (!a.parts_ready) {   // else dmoe_router_prepare wrote this W_r's parts already
+    e = launch_router_wsplit(a.w_r, a.w_parts, a.d, a.E, s);
+    if (e != cudaSuccess) return e;
+  }
   static int mask = 0;
   int dev = 0;
   cudaGetDevice(&dev);

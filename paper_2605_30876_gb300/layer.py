@@ -6,7 +6,8 @@ from typing import Dict, Optional
 
 import torch
 
-from . import (DMOE_ROUTE_BLOCK, LayerDesc, alloc_workspace, dmoe_layer_forward, make_desc)
+from . import (DMOE_ROUTE_BLOCK, LayerDesc, alloc_workspace, dmoe_layer_forward,
+               dmoe_router_prepare, make_desc)
 
 WEIGHT_KEYS = ("w_r", "bias", "w_gate", "w_up", "w_down", "ws_gate", "ws_up", "ws_down")
 
@@ -31,6 +32,12 @@ class MoELayer:
         self.topk_gate = torch.empty((T, k), dtype=torch.float32, device=self.device)
         self.n_unique = torch.zeros(1, dtype=torch.int32, device=self.device)
         self.unique_ids = torch.empty(E, dtype=torch.int32, device=self.device)
+        # the router weight's tensor-core split, once (the forwards on this workspace then
+        # skip it); prepare() again after changing w_r in place
+        self.prepare()
+
+    def prepare(self, stream=None) -> None:
+        dmoe_router_prepare(self.desc, self.w["w_r"], self.ws, stream=stream)
 
     @classmethod
     def from_shape(cls, shape, weights, device="cuda", workspace=None) -> "MoELayer":

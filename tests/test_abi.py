@@ -103,6 +103,11 @@ def test_null_and_misaligned_pointers_are_rejected_before_launch(dm):
     assert st == 1
     st = lib.dmoe_layer_forward(None, *([P(fake)] * 14), P(fake), n, None)
     assert st == 1
+    # router preparation: misaligned W_r, workspace too small
+    st = lib.dmoe_router_prepare(ctypes.byref(desc), P(fake + 4), P(fake), n, None)
+    assert st == 1
+    st = lib.dmoe_router_prepare(ctypes.byref(desc), P(fake), P(fake), n - 1, None)
+    assert st == 3
 
 
 def test_layer_forward_launch_count(dm):

@@ -106,6 +106,34 @@ def test_moe_forward_on_injected_oracle_routing(name):
     P.check_output(y, ref, label=name)
 
 
+def test_router_prepare_skips_only_a_matching_split():
+    """dmoe_router_prepare (the tensor-core router's split of W_r, once): the prepared
+    forward equals an unprepared one bit for bit; a call with another W_r on the prepared
+    workspace splits that one, and a later call with the first W_r splits it again."""
+    shape = LAYER_B8
+    m = P.dm()
+    dev, _ = P.make(shape, seed=3)
+    from paper_2605_30876_gb300.layer import MoELayer
+    layer = MoELayer.from_shape(shape, dev)   # prepares its workspace
+    y_prep = layer.forward(dev["x"]).clone()
+
+    def fwd(w_r, ws):
+        y = torch.empty_like(y_prep)
+        m.dmoe_layer_forward(layer.desc, dev["x"], w_r, dev["bias"], dev["w_gate"], dev["w_up"],
+                             dev["w_down"], dev["ws_gate"], dev["ws_up"], dev["ws_down"], y,
+                             None, None, None, None, workspace=ws)
+        st, info = m.dmoe_get_device_error(ws)
+        assert st == 0, info
+        return y
+
+    assert torch.equal(fwd(dev["w_r"], m.alloc_workspace(layer.desc)), y_prep)
+    w_r2 = dev["w_r"].flip(1).contiguous()   # the experts' router columns reversed
+    y_b = fwd(w_r2, layer.ws)
+    assert torch.equal(y_b, fwd(w_r2, m.alloc_workspace(layer.desc)))
+    assert not torch.equal(y_b, y_prep)
+    assert torch.equal(layer.forward(dev["x"]), y_prep)
+
+
 def test_stack_shape_layer_sampled():
     """One layer of the 2048-token stack shape (64 blocks of 32): routing parity on all
     tokens, outputs on sampled tokens (the oracle is slow at this size)."""
