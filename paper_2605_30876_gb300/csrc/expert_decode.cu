@@ -200,6 +200,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
   // before it ends; the weight stream starts on them, and only the down epilogue waits for
   // the dispatch. Otherwise (or if the coresets do not come) everything waits for it.
   bool spec = p.spec_words != nullptr;
+  int early = 0;   // stages of the first gate/up unit the producer sent right after the poll
   if (spec) {
     if (warp == 0) {
       // poll every block's words until all are nonzero; a nonzero word is complete (one
@@ -254,6 +255,40 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
           s_spec[u++] = (uint8_t)(lane * 32 + __ffs((int)bits) - 1);
       }
       if (lane == 0) *s_u = bad ? -1 : u_all;
+      __syncwarp();
+      if (lane == 0 && !bad) {
+        // This lane is the producer: the first ring slots of its first gate/up unit are
+        // filled now, before the CTA barrier and the unit bookkeeping below (the same copies
+        // the producer loop would make; fresh ring slots need no wait).
+        const bool h32e = h32_ok && 2 * (ngu64_s + u_all * ngu64_r) <= nb;
+        const int hge = h32e ? 32 : 64, kbge = kTileM / hge;
+        const int slote = h32e ? slot32 : slot64, Se = h32e ? S32 : S64;
+        const int ngse = h32e ? ngu_s32 : ngu64_s, ngre = h32e ? ngu_r32 : ngu64_r;
+        const int kce = h32e ? kc32 : kc64;
+        if (b < ngse + u_all * ngre) {
+          const bool sh = b < ngse;
+          const int m = sh ? b : (b - ngse) % ngre;
+          const int e = sh ? 0 : (int)s_spec[(b - ngse) / ngre];
+          const CUtensorMap* mg = h32e ? (sh ? &tm.sg32 : &tm.wg32) : (sh ? &tm.sg : &tm.wg);
+          const CUtensorMap* mu = h32e ? (sh ? &tm.su32 : &tm.wu32) : (sh ? &tm.su : &tm.wu);
+          const int arow = (sh ? 0 : e * pI) + m * hge;
+          const uint64_t pw = ptx::policy_evict_first(), px = ptx::policy_evict_last();
+          early = Se < kce ? Se : kce;
+          ED_AT(28);
+          for (int c = 0; c < early; ++c) {
+            ptx::mbar_arrive_expect_tx(&full[c], kAStage + kbge * bbox);
+            uint8_t* a_dst = smem + c * slote;
+            uint8_t* b_dst = a_dst + kAStage;
+            for (int kb = 0; kb < kbge; ++kb) {
+              const int kx = (c * kbge + kb) * kTileK;
+              ptx::tma_load_2d(a_dst + kb * 2 * hge * 128, mg, &full[c], kx, arow, pw);
+              ptx::tma_load_2d(a_dst + kb * 2 * hge * 128 + hge * 128, mu, &full[c], kx, arow,
+                               pw);
+              ptx::tma_load_2d(b_dst + kb * bbox, &tm.x, &full[c], kx, 0, px);
+            }
+          }
+        }
+      }
     }
     __syncthreads();
     if (tid == 0) ED_AT(19);
@@ -369,8 +404,9 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
     const uint64_t pol_w = ptx::policy_evict_first();   // weights: streamed once
     const uint64_t pol_x = ptx::policy_evict_last();    // x and H: re-read by many tiles
     ED_AT(31);
-    int stage = 0, issued = 0;
-    uint32_t phase = 0;
+    // the stages sent right after the poll
+    int stage = early == S ? 0 : early, issued = early;
+    uint32_t phase = early == S ? 1u : 0u;
     bool ok = true;
     bool first = true;
     for (int u = b; u < NGU && ok; u += nb) {
@@ -383,7 +419,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
           hg == 32 ? (g.shared ? &tm.su32 : &tm.wu32) : (g.shared ? &tm.su : &tm.wu);
       const int arow = (g.shared ? 0 : g.e * p.I) + m * hg;
       if (first) ED_SET(10, u);
-      for (int c = 0; c < kc; ++c) {
+      for (int c = first ? early : 0; c < kc; ++c) {
         if (!wait(&empty[stage], phase ^ 1u, u)) { ok = false; break; }
         if (first && c == 0) ED_AT(28);
         if (first && c == kc - 1) ED_AT(29);
