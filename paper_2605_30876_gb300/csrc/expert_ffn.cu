@@ -767,6 +767,9 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         if (lane == 0) *p.n_unique_out = U;
         for (int u = lane; u < p.E; u += 32) p.unique_ids_out[u] = u < U ? g_e[u] : -1;
       }
+      // visible before this launch releases the combine (at its end): the combine reads
+      // pos before its dependency wait
+      __threadfence();
     }
     const int q = warp & 3;
     const int cg = (warp - 2) >> 2;                 // column group
@@ -1195,8 +1198,9 @@ cudaError_t launch_experts(const ExpertArgs& a, cudaStream_t s) {
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
 
-  // 3. gate-weighted combine of the bf16 rows
-  return launch_combine(a, s, nullptr, 0, nullptr, 0, false, true);
+  // 3. gate-weighted combine of the bf16 rows (the slot rows and gates were complete before
+  //    this launch released it: the combine may read them before its dependency wait)
+  return launch_combine(a, s, nullptr, 0, nullptr, 0, true, true);
 }
 
 cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero, int n_zero,
