@@ -38,6 +38,12 @@ LAYER_CASES = {
     # the paper's top-p sweep ends beside p = 0.6 (Table 3: p_test 0.4 ... 0.8)
     "layer_block_p04": LAYER.with_(top_p=0.4),
     "layer_block_p08": LAYER.with_(top_p=0.8),
+    # block top-k on the general path (the expert launch plans from the published coresets
+    # and does the dispatch): no shared expert, k not a multiple of three, fewer experts;
+    # 20 blocks of 16 (ragged token tiles), skewed bias, k = 6
+    "spec_b8x16_noshared_k4_E64": LAYER.with_(block_size=16, n_blocks=8, d_ff_shared=0,
+                                              top_k=4, n_experts=64),
+    "spec_b20x16_k6_bias1": LAYER.with_(block_size=16, n_blocks=20, top_k=6, bias_scale=1.0),
     # the block-size x batch x bias grid: its smallest corner, uniform router bias
     "sweep_B4x1_bias0_block": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0),
     "sweep_B4x1_bias0_token": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0,
