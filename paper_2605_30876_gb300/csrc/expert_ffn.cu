@@ -107,6 +107,14 @@ using ptx::red_release_add;
 
 __device__ __forceinline__ float silu_f(float z) { return z / (1.f + __expf(-z)); }
 
+// A bf16 store that asks L2 to keep the line (the slot rows are read back by the combine
+// right after this launch, while the weights stream through L2 with evict-first)
+__device__ __forceinline__ void st_bf16_keep(__nv_bfloat16* p, __nv_bfloat16 v, uint64_t pol) {
+  asm volatile("st.global.L2::cache_hint.b16 [%0], %1, %2;" ::"l"(p),
+               "h"(*reinterpret_cast<const unsigned short*>(&v)), "l"(pol)
+               : "memory");
+}
+
 // AND of `v` over the kEpiThreads epilogue threads (named barrier 1), so that they take the
 // warp-collective TMEM loads, or leave the unit loop, together
 __device__ __forceinline__ bool epi_all_threads(bool v) {
@@ -776,6 +784,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
     const uint32_t lane_off = (uint32_t)(q * 32) << 16;
     float* xg = xchg + cg * (128 * kXchgStride);    // this group's exchange tile
     const int gbar = 2 + cg;                        // this group's named barrier
+    const uint64_t pol_keep = ptx::policy_evict_last();   // the slot rows, for the combine
     int acc = 0, li = 0;
     uint32_t acc_phase = 0;
     for (int u = blockIdx.x; u < units; u += gridDim.x, ++li) {
@@ -857,7 +866,8 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
 #pragma unroll
             for (int c = 0; c < 16; ++c)
               if (c0 + c < nvalid)
-                out[(size_t)(c0 + c) * p.d + drow] = __float2bfloat16_rn(v[c]);
+                st_bf16_keep(out + (size_t)(c0 + c) * p.d + drow, __float2bfloat16_rn(v[c]),
+                             pol_keep);
           }
           ptx::tc_fence_before();
           ptx::mbar_arrive(&acc_empty[slot]);
