@@ -67,10 +67,13 @@ def test_routing_matches_oracle(name):
     g = P.gpu_router(shape, dev)
     orc = P.oracle_routing(shape, host)
     stats = P.check_routing(shape, g, orc)
-    # tokens at an oracle near tie (margin < 1e-5) are checked for validity only; report
-    # how many there were
+    # every token is either compared exactly or sits at an oracle near tie (margin < 1e-5),
+    # where only validity is checked; report how many there were. At a 1e-5 margin and score
+    # gaps of about 1e-3 between neighbouring ranks, about 1 % of the seeded tokens are near
+    # ties: more than 3 % (or 2 tokens) would mean the exact comparison covers too little.
     print(f"{name}: {stats}")
-    assert stats["exact"] >= 0.9 * stats["tokens"], stats
+    assert stats["exact"] + stats["ambiguous"] == stats["tokens"], stats
+    assert stats["ambiguous"] <= max(2, int(0.03 * stats["tokens"])), stats
     if shape.mode == ROUTE_BLOCK and shape.top_p == 0.0:
         for b in range(shape.n_blocks):
             blk = g["idx"][b * shape.block_size:(b + 1) * shape.block_size]
