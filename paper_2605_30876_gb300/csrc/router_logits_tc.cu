@@ -14,11 +14,11 @@
 //
 //   router_wsplit_kernel      the three parts of W_r, each stored K-major ([E, d] bf16: row
 //                             e holds expert e's weights over d), the MMA's B operand
-//   router_logits_tc_kernel   one CTA per (128 tokens, slice of d), all E experts (N = E,
-//                             a multiple of 32, at most 256), no cross-CTA step:
+//   router_logits_tc_kernel   one CTA per (128 tokens, slice of d, group of N experts; N =
+//                             E / nsplit, a multiple of 32, at most 256), no cross-CTA step:
 //     warp 0     TMA, two stages: x chunk (128 tokens x 64 of d, 128-B swizzle, rows past
-//                T read as zero) and the three parts' chunks (E rows x 64)
-//     warp 1     TMEM allocation; lane 0 issues D[128 x E] += x * part^T, 4 K-steps of 16
+//                T read as zero) and the three parts' chunks (N rows x 64)
+//     warp 1     TMEM allocation; lane 0 issues D[128 x N] += x * part^T, 4 K-steps of 16
 //                per chunk and part (hi into one accumulator, mid and lo into the other)
 //     warps 0-3  (after the MMAs; one TMEM lane quadrant each) put hi + (mid + lo) into
 //                shared memory (the stages are free by then) as E / 32 boxes of 32
@@ -53,11 +53,12 @@ constexpr uint64_t kLtTimeoutNs = 1000000000ull;
 
 struct LtArgs {
   CUtensorMap xmap;   // x [T, d] bf16, box 64 columns x 128 rows, 128-B swizzle
-  CUtensorMap pmap;   // parts [3E, d] bf16, box 64 columns x E rows, 128-B swizzle
+  CUtensorMap pmap;   // parts [3E, d] bf16, box 64 columns x N rows, 128-B swizzle
   CUtensorMap omap;   // partials [S, T, E] fp32, box 32 x 128 x 1, 128-B swizzle
   DevErrRecord* err;
   L2Prefetch shared_pf;
   int T, d, E, ds;    // ds: d per slice (blockIdx.y)
+  int N;              // experts per CTA (blockIdx.z: experts N z .. N z + N - 1)
 };
 
 // parts[p][e][i] for the tile of 32 experts x 64 of d: thread (e, 8-wide run of d) reads
@@ -115,13 +116,17 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
   __shared__ int s_abort;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) RTC_AT(0);
-  const int E = f.E;
+  const int E = f.E, N = f.N;
+  const int e_base = blockIdx.z * N;
   const int m0 = blockIdx.x * kLtM;
   const int k_base = blockIdx.y * f.ds;
   const int nch = f.ds / kLtKC;
-  const int pbytes = E * 128;                 // one part's chunk
+  const int pbytes = N * 128;                 // one part's chunk
   const int slot = kLtXBytes + 3 * pbytes;
-  const uint32_t t_ml = 256;                  // the mid/lo accumulator's first column
+  // TMEM: the hi accumulator in columns 0 .. N-1, the mid/lo one from column t_ml
+  uint32_t t_ml = 32;
+  while (t_ml < (uint32_t)N) t_ml <<= 1;
+  const uint32_t t_cols = 2 * t_ml;
   auto x_buf = [&](int s) { return smem + s * slot; };
   auto p_buf = [&](int s, int part) { return smem + s * slot + kLtXBytes + part * pbytes; };
 
@@ -136,11 +141,12 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
     ptx::fence_mbarrier_init();
     s_abort = 0;
     // the shared expert's weights are pulled into L2 for the expert launch
-    issue_shared_prefetch(f.shared_pf, (int)(blockIdx.y * gridDim.x + blockIdx.x),
-                          (int)(gridDim.x * gridDim.y));
+    issue_shared_prefetch(f.shared_pf,
+                          (int)((blockIdx.z * gridDim.y + blockIdx.y) * gridDim.x + blockIdx.x),
+                          (int)(gridDim.x * gridDim.y * gridDim.z));
   }
   if (warp == 1) {
-    ptx::tmem_alloc(&s_tmem, 512);
+    ptx::tmem_alloc(&s_tmem, t_cols);
     ptx::tmem_relinquish();
   }
   pdl_wait();   // the parts of this call are written
@@ -173,14 +179,14 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
         ptx::tma_load_2d(x_buf(s), &f.xmap, &full[s], k0, m0, pol);
 #pragma unroll
         for (int part = 0; part < 3; ++part)
-          ptx::tma_load_2d(p_buf(s, part), &f.pmap, &full[s], k0, part * E, pol);
+          ptx::tma_load_2d(p_buf(s, part), &f.pmap, &full[s], k0, part * E + e_base, pol);
       }
       RTC_AT(2);
     }
   } else if (warp == 1) {
     if (lane == 0) {
       // ================= MMA issuer
-      const uint32_t idesc = ptx::idesc_bf16(kLtM, (uint32_t)E);
+      const uint32_t idesc = ptx::idesc_bf16(kLtM, (uint32_t)N);
       for (int c = 0; c < nch; ++c) {
         const int s = c & 1;
         const uint32_t ph = (uint32_t)((c >> 1) & 1);
@@ -218,7 +224,7 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
     uint8_t* boxes = smem;
     const int r = warp * 32 + lane;
     const uint32_t lanes = (uint32_t)(warp * 32) << 16;
-    for (int c0 = 0; c0 < E; c0 += 32) {
+    for (int c0 = 0; c0 < N; c0 += 32) {
       float h[32], ml[32];
       ptx::tmem_ld32(tmem + lanes + (uint32_t)c0, h);
       ptx::tmem_ld32(tmem + lanes + t_ml + (uint32_t)c0, ml);
@@ -235,8 +241,9 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
     __syncthreads();
     if (tid == 0) {
       if (have_acc)
-        for (int b = 0; b < E / 32; ++b)
-          ptx::tma_store_3d(&f.omap, boxes + b * (kLtM * 128), 32 * b, m0, (int)blockIdx.y);
+        for (int b = 0; b < N / 32; ++b)
+          ptx::tma_store_3d(&f.omap, boxes + b * (kLtM * 128), e_base + 32 * b, m0,
+                            (int)blockIdx.y);
       ptx::bulk_commit_wait_read();   // the shared memory stays until the stores read it
     }
   }
@@ -245,7 +252,7 @@ router_logits_tc_kernel(const __grid_constant__ LtArgs f) {
   if (tid == 0) RTC_AT(6);
   if (warp == 1) {
     ptx::tc_fence_after();
-    ptx::tmem_dealloc(tmem, 512);
+    ptx::tmem_dealloc(tmem, t_cols);
   }
   KLOG(DMOE_KERNEL_ROUTER, 1);
 }
@@ -318,6 +325,16 @@ int router_tc_splits(int T, int d) {
   return best;
 }
 
+// Groups of experts per (token tile, slice): with few token tiles the CTAs are split over
+// the experts too (N = E / nsplit columns each, a multiple of 32), as far as one wave allows.
+int router_tc_nsplit(int T, int E, int splits) {
+  const int ctas = ((T + kLtM - 1) / kLtM) * splits;
+  int best = 1;
+  for (int n = 2; n <= 8; ++n)
+    if ((E / 32) % n == 0 && ctas * n <= 152) best = n;
+  return best;
+}
+
 size_t router_tc_parts_bytes(int d, int E) { return (size_t)3 * E * d * 2; }
 
 cudaError_t launch_router_wsplit(const float* w_r, __nv_bfloat16* parts, int d, int E,
@@ -332,9 +349,11 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
     return cudaErrorInvalidValue;
   EncodeFn enc = encode_fn_lt();
   if (enc == nullptr) return cudaErrorInvalidValue;
+  const int nsplit = router_tc_nsplit(a.T, a.E, splits);
+  const int N = a.E / nsplit;
   LtArgs f{};
   if (!encode_bf16_2d(enc, &f.xmap, a.x, (uint64_t)a.T, (uint64_t)a.d, kLtM) ||
-      !encode_bf16_2d(enc, &f.pmap, a.w_parts, 3 * (uint64_t)a.E, (uint64_t)a.d, (uint32_t)a.E) ||
+      !encode_bf16_2d(enc, &f.pmap, a.w_parts, 3 * (uint64_t)a.E, (uint64_t)a.d, (uint32_t)N) ||
       !encode_part_3d(enc, &f.omap, a.tc_part, splits, a.T, a.E))
     return cudaErrorInvalidValue;
   f.err = a.err;
@@ -343,6 +362,7 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
   f.d = a.d;
   f.E = a.E;
   f.ds = a.d / splits;
+  f.N = N;
   cudaError_t e = cudaSuccess;
   if (!a.parts_ready) {   // else dmoe_router_prepare wrote this W_r's parts already
     e = launch_router_wsplit(a.w_r, a.w_parts, a.d, a.E, s);
@@ -357,8 +377,8 @@ cudaError_t launch_router_tc(const RouterArgs& a, int splits, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     if (dev < 31) mask |= 1 << dev;
   }
-  return launch_ex(router_logits_tc_kernel, dim3((a.T + kLtM - 1) / kLtM, splits),
-                   dim3(kLtThreads), lt_smem_bytes(a.E), s, true, f);
+  return launch_ex(router_logits_tc_kernel, dim3((a.T + kLtM - 1) / kLtM, splits, nsplit),
+                   dim3(kLtThreads), lt_smem_bytes(N), s, true, f);
 }
 
 }  // namespace dmoe
