@@ -273,7 +273,9 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
         arm.step(i)
     torch.cuda.synchronize()
     arm.check()
-    M = n_sets
+    # graphs of up to 64 steps (whole rotations of the weight sets when K allows): a short
+    # timed region is then one or two graph launches, not one per rotation
+    M = min(K, max(n_sets, (64 // n_sets) * n_sets))
     R, tail = divmod(K, M)
     NG = 3
     evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -305,6 +307,9 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
         sampler.start()
         time.sleep(0.2)
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    # the device spins ~0.5 ms before the start event while the host enqueues the first graph
+    # launches, so that the host's launch latency is not inside the device-timed region
+    torch.cuda._sleep(1_000_000)
     start.record()
     for r in range(R):
         graphs[r % NG].replay()
