@@ -126,8 +126,9 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   w.xperm = take(2 * T * k * dm);
   w.h = take(2 * T * k * I);
   w.hs = take(2 * T * Is);
-  // gate/up tile counters, then (block top-k on the general path) the rows copied per group
-  w.h_ready = take(sizeof(int32_t) * (experts_ready_counters((int)T, (int)E, w.n_max) + E + 1));
+  // gate/up tile counters, then (block top-k on the general path) the rows copied per
+  // (group, token tile)
+  w.h_ready = take(sizeof(int32_t) * 2 * experts_ready_counters((int)T, (int)E, w.n_max));
   w.yslot = take(sizeof(float) * T * k * dm);
   w.yshared = take(sizeof(float) * T * dm);
   const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
@@ -478,8 +479,7 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
     spec_w = at<uint32_t>(workspace, plan.spec);
     st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
                     shared_pf, nullptr, spec_w, at<int32_t>(workspace, plan.h_ready),
-                    experts_ready_counters(T, desc->n_experts, plan.n_max) +
-                        desc->n_experts + 1);
+                    2 * experts_ready_counters(T, desc->n_experts, plan.n_max));
     if (st != DMOE_OK) return st;
     return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid,
                        offs, rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w,

@@ -78,8 +78,9 @@ struct GemmParams {
   // routing launch publishes (n_blocks blocks of blk rows). The unique experts are their
   // union, ascending; an expert's token rows are its blocks' rows in block order, which is
   // the dispatch's order. This launch then does the dispatch itself: its CTAs copy every
-  // (block, coreset member) pair's rows of x to their place in xperm (x_ready[g] counts a
-  // group's copied rows; a gate/up unit loads them once they are all there) and write
+  // (block, coreset member) pair's rows of x to their place in xperm (x_ready[g ntiles + n]
+  // counts the copied rows of token tile n of group g; a gate/up unit loads its tile's rows
+  // once they are all there) and write
   // n_unique, unique_ids and pos (the row of every (token, slot), from topk_idx).
   const uint32_t* spec_words;
   int n_blocks, blk;
@@ -87,7 +88,8 @@ struct GemmParams {
   int32_t* pos_out;
   int32_t* n_unique_out;
   int32_t* unique_ids_out;
-  int32_t* x_ready;          // [kMaxGroups], zero at the start (the routing launch clears it)
+  int32_t* x_ready;          // [groups x ntiles], zero at the start (the routing launch
+                             // clears it)
   const __nv_bfloat16* x;
   __nv_bfloat16* xperm;
 };
@@ -495,7 +497,7 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
           int c0 = 0;
           if (spec && !shared) {
             // block top-k: the weight stages first, the token rows once this launch's copies
-            // of the group's rows are all in xperm
+            // of the tile's rows are all in xperm
             const int pre = kc < stages ? kc : stages;
             const int stage0 = stage;
             for (int c = 0; c < pre; ++c) {
@@ -506,10 +508,12 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
               if (++stage == stages) { stage = 0; phase ^= 1u; }
             }
             if (!ok) break;
-            const int32_t* flag = p.x_ready + un.g;
-            if (ld_acquire(flag) < g_cnt[un.g]) {
+            // the rows of this token tile (a pair's rows lie in one tile: n_max % blk == 0)
+            const int32_t* flag = p.x_ready + un.g * p.ntiles + un.n;
+            const int need = min(p.n_max, g_cnt[un.g] - un.n * p.n_max);
+            if (ld_acquire(flag) < need) {
               const uint64_t t0 = ptx::globaltimer_ns();
-              while (ld_acquire(flag) < g_cnt[un.g]) {
+              while (ld_acquire(flag) < need) {
                 if (*s_abort) { ok = false; break; }
                 if (ptx::globaltimer_ns() - t0 > kWaitTimeoutNs) {
                   record_error(p.err, kErrTimeout, kAtGather, u);
@@ -742,7 +746,8 @@ moe_experts_kernel(const __grid_constant__ Maps tm, const GemmParams p) {
         }
         __threadfence();
         named_bar_sync(4, kEpiThreads);
-        if (et == 0) red_release_add(p.x_ready + s_upos[e], prow);
+        if (et == 0)
+          red_release_add(p.x_ready + s_upos[e] * p.ntiles + (p.blk * rank) / p.n_max, prow);
       }
       if (et == 0) DMOE_TRACE_AT(63);
     }
