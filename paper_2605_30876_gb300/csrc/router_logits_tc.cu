@@ -313,6 +313,9 @@ int router_tc_splits(int T, int d) {
   const int tiles = (T + kLtM - 1) / kLtM;
   const int nch = d / kLtKC;
   const int s_min = (d + kLtMaxDS - 1) / kLtMaxDS;
+  // with the experts split over up to 8 CTAs as well, the fewest slices (the fewest partial
+  // rows for the softmax to add) already give a wave of 128 CTAs
+  if (nch % s_min == 0 && tiles * s_min * 8 >= 128) return s_min;
   int best = 0;
   for (int s = s_min; s <= nch && s <= 16; ++s)
     if (nch % s == 0 && (best == 0 || tiles * s <= 152)) best = s;
