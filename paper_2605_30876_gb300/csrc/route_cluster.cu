@@ -447,17 +447,16 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
     int* sCore = reinterpret_cast<int*>(dsm + kOffCore);    // [8 warps][1 + kMaxExperts]
     for (int b = (int)rank; b < a.n_blocks; b += kCl) {
       const int t0 = b * B;
+      // block top-k: the coreset (k experts) is the routing of every token of the block; it
+      // is published for the expert launch as soon as it is known
       const int size = block_coreset_steps(
           E, kc, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
-          a.coreset_size != nullptr ? a.coreset_size + b : nullptr);
+          a.coreset_size != nullptr ? a.coreset_size + b : nullptr,
+          a.spec_words != nullptr && a.top_p <= 0.f && kc == k
+              ? a.spec_words + (size_t)b * spec_words(k)
+              : nullptr);
       CT_AT(25);
-      if (a.spec_words != nullptr) {
-        // block top-k: the coreset (k experts) is the routing of every token of the block;
-        // publish it for the expert launch, three ids and a marker byte per word
-        const int nw = spec_words(k);
-        if (tid < nw) publish_coreset(a.spec_words + (size_t)b * nw, order, k, tid);
-      }
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order
       for (int i = tid; i < B * (size + 1); i += 256) {

@@ -205,7 +205,8 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
 template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
-                                          int32_t* __restrict__ coreset_size) {
+                                          int32_t* __restrict__ coreset_size,
+                                          uint32_t* __restrict__ spec = nullptr) {
   __shared__ __align__(16) float st_s[kMaxExperts];
   __shared__ uint2 nz_kid[kMaxExperts];   // nonzero entries: (order key, id), ids ascending
   __shared__ int wcnt[2][8];
@@ -250,6 +251,20 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
       float my_v;
       warp_topk(v, id, valid, k, my_e, my_v);
       if (lane < k) order[lane] = my_e;
+      if (spec != nullptr) {
+        // block top-k: the coreset (the k best, best first) is every token's routing; it is
+        // published for the expert launch at once, three 8-bit ids and a marker byte per
+        // word, one relaxed store per word (a word reads as zero until it is complete)
+        uint32_t w = 1u << 24;
+#pragma unroll
+        for (int j = 0; j < 3; ++j) {
+          const int src = 3 * lane + j;
+          const int ej = __shfl_sync(0xffffffffu, my_e, src & 31);
+          if (src < k) w |= (uint32_t)ej << (8 * j);
+        }
+        if (lane < spec_words(k))
+          asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(spec + lane), "r"(w) : "memory");
+      }
     }
     __syncthreads();
     if (coreset != nullptr && live) coreset[tid] = (tid < k) ? order[tid] : -1;
@@ -451,26 +466,16 @@ __device__ inline void mask_topk_warps(int k, int B, int size, const int* order,
   }
 }
 
-// Block top-k publication: the block's coreset (its k members, best first), three 8-bit ids
-// and a marker byte per 32-bit word, one relaxed store per word (a word reads as zero until
-// it is complete). Called by threads 0 .. spec_words(k) - 1.
-__device__ inline void publish_coreset(uint32_t* __restrict__ words, const int* order, int k,
-                                       int i) {
-  uint32_t w = 1u << 24;
-  for (int j = 0; j < 3 && 3 * i + j < k; ++j) w |= (uint32_t)order[3 * i + j] << (8 * j);
-  asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(words + i), "r"(w) : "memory");
-}
-
 template <class HatFn, class ProbFn, class OutFn>
 __device__ inline void block_route_steps(int E, int kb, int k, int B, float top_p, HatFn hat,
                                          ProbFn prob, OutFn out, int32_t* __restrict__ coreset,
                                          int32_t* __restrict__ coreset_size,
                                          uint32_t* __restrict__ spec = nullptr) {
   __shared__ int order[kMaxExperts];
-  const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size);
-  // block top-k (the coreset is every token's routing): published for the expert launch
-  if (spec != nullptr && size == k && (int)threadIdx.x < spec_words(k))
-    publish_coreset(spec, order, k, threadIdx.x);
+  // block top-k (p <= 0, the coreset is every token's routing): published for the expert
+  // launch as soon as it is known
+  const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size,
+                                       top_p <= 0.f && kb == k ? spec : nullptr);
   DMOE_STAMP(25);
   mask_topk_warps(k, B, size, order, prob, out);
   __syncthreads();
