@@ -193,9 +193,8 @@ class Arm:
     def unique_counts(self):
         return [int(L.n_unique.item()) for L in self.layers]
 
-    def capture(self, n_steps, first, events=None):
-        """A CUDA graph of n_steps consecutive steps starting at index `first`; events[i] =
-        (begin, end) recorded around step i's gate/up kernel."""
+    def capture(self, n_steps, first):
+        """A CUDA graph of n_steps consecutive steps starting at index `first`."""
         torch = self.torch
         g = torch.cuda.CUDAGraph()
         with torch.cuda.graph(g):
@@ -203,11 +202,7 @@ class Arm:
                 self.capture_host_io(n_steps, first)
             else:
                 for i in range(n_steps):
-                    if events is not None:
-                        self.dm.dmoe_set_profile_events("experts", *events[i])
                     self.step(first + i)
-                if events is not None:
-                    self.dm.dmoe_set_profile_events("experts", None, None)
         return g
 
     def capture_host_io(self, n_steps, first):
@@ -265,9 +260,9 @@ def job_throughput(tokens_per_step: int, steps: int, world: int, secs_max: float
     return tokens_per_step * steps * world / secs_max
 
 
-def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
+def timed_region(arm, K, W, torch, dist, world, sampler=None):
     """W warm-up steps, then exactly K steps from graph replays; returns (seconds over the
-    timed region, max over ranks; mean gate/up launch seconds or None)."""
+    timed region, max over ranks; the clock samples)."""
     n_sets = len(arm.layers)
     for i in range(W):
         arm.step(i)
@@ -278,14 +273,7 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
     M = min(K, max(n_sets, (64 // n_sets) * n_sets))
     R, tail = divmod(K, M)
     NG = 3
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(M)] for _ in range(NG)] if want_kernel else None
-    if want_kernel:           # torch creates the CUDA event on its first record
-        for row in evs:
-            for b, e in row:
-                b.record()
-                e.record()
-    graphs = [arm.capture(M, 0, evs[j] if want_kernel else None) for j in range(NG)]
+    graphs = [arm.capture(M, 0) for _ in range(NG)]
     tail_g = arm.capture(tail, 0) if tail else None
     for g in graphs:       # graph upload
         g.replay()
@@ -293,12 +281,6 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
         tail_g.replay()
     torch.cuda.synchronize()
     arm.check()
-    kernel_ms = []
-
-    def collect(j):
-        for b, e in evs[j]:
-            e.synchronize()
-            kernel_ms.append(b.elapsed_time(e))
 
     if dist is not None:
         dist.barrier()
@@ -313,22 +295,42 @@ def timed_region(arm, K, W, torch, dist, world, want_kernel=True, sampler=None):
     start.record()
     for r in range(R):
         graphs[r % NG].replay()
-        if want_kernel and r >= 2:
-            collect((r - 2) % NG)
     if tail_g is not None:
         tail_g.replay()
     end.record()
     torch.cuda.synchronize()
     clocks = sampler.stop() if sampler is not None else None
-    if want_kernel:
-        for r in range(max(0, R - 2), R):
-            collect(r % NG)
     if dist is not None:
         dist.barrier()
     secs = max_over_ranks(start.elapsed_time(end) / 1e3, dist, world)
     arm.check()
-    kern = (float(np.mean(kernel_ms)) / 1e3) if kernel_ms else None
-    return secs, kern, clocks
+    return secs, clocks
+
+
+def expert_launch_seconds(arm, n_steps, torch, dm):
+    """Mean duration of the expert launch over n_steps steps: CUDA events recorded just
+    before and after it on its stream (the library then makes it without programmatic
+    overlap, so that they bracket its own execution). The steps are launched eagerly: inside
+    a CUDA graph each event-record node adds ~6 us between the kernels it separates."""
+    P = 64                                  # event pairs in flight
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(P)]
+    for b, e in evs:                        # torch creates the CUDA event on its first record
+        b.record()
+        e.record()
+    ms = []
+    for i in range(n_steps + P):
+        b, e = evs[i % P]
+        if i >= P:                          # the pair's previous use has ended
+            e.synchronize()
+            ms.append(b.elapsed_time(e))
+        if i < n_steps:
+            dm.dmoe_set_profile_events("experts", b, e)
+            arm.step(i)
+    dm.dmoe_set_profile_events("experts", None, None)
+    torch.cuda.synchronize()
+    arm.check()
+    return float(np.mean(ms[8:] if len(ms) > 16 else ms)) / 1e3
 
 
 def traffic_from_profile(kernel: str, source: str):
@@ -892,12 +894,12 @@ def main():
     # headline: block routing, p = 0
     arm = Arm(shape, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
     # the headline pass records no events; the expert kernel's launch duration is timed by
-    # CUDA events in a second pass over the same steps (while the events are set, the
-    # library makes that launch without programmatic overlap, so that they bracket its own
-    # execution rather than an early start spent waiting for the routing)
-    secs, _, clocks = timed_region(arm, args.steps, args.warmup, torch, dist, world,
-                                   want_kernel=False, sampler=sampler)
-    _, kern_s, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world)
+    # CUDA events in a second pass over the same steps, launched eagerly (while the events
+    # are set, the library makes that launch without programmatic overlap, so that they
+    # bracket its own execution rather than an early start spent waiting for the routing)
+    secs, clocks = timed_region(arm, args.steps, args.warmup, torch, dist, world,
+                                sampler=sampler)
+    kern_s = expert_launch_seconds(arm, min(args.steps, 4000), torch, dm)
     U = arm.unique_counts()
     U_mean = float(np.mean(U))
     T = shape.T
@@ -909,8 +911,7 @@ def main():
     secs_e2e = None
     if not args.only_headline:
         arm.set_host_io(True)
-        secs_e2e, _, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world,
-                                      want_kernel=False)
+        secs_e2e, _ = timed_region(arm, args.steps, args.warmup, torch, dist, world)
         arm.set_host_io(False)
 
     # side by side: token routing and the paper's p = 0.6
@@ -919,9 +920,8 @@ def main():
                                                ("block_p0.6", workload_shape("block", 0.6)))
     for name, sh in side_cfgs:
         a2 = Arm(sh, args.sets, args.seed + 97 * rank, torch, dm, MoELayer, layer_inputs)
-        s2, _, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world,
-                                want_kernel=False)
-        _, k2, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world)
+        s2, _ = timed_region(a2, args.side_steps, args.warmup, torch, dist, world)
+        k2 = expert_launch_seconds(a2, min(args.side_steps, 2000), torch, dm)
         u2 = float(np.mean(a2.unique_counts()))
         us = s2 / args.side_steps * 1e6
         side[name] = {"us_per_forward": us,
