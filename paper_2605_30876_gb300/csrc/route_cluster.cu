@@ -455,7 +455,8 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr,
           a.spec_words != nullptr && a.top_p <= 0.f && kc == k
               ? a.spec_words + (size_t)b * spec_words(k)
-              : nullptr);
+              : nullptr,
+          sHat + (size_t)t0 * kMaxExperts, kMaxExperts);
       CT_AT(25);
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order

@@ -206,7 +206,8 @@ template <class HatFn>
 __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatFn hat, int* order,
                                           int32_t* __restrict__ coreset,
                                           int32_t* __restrict__ coreset_size,
-                                          uint32_t* __restrict__ spec = nullptr) {
+                                          uint32_t* __restrict__ spec = nullptr,
+                                          const float* rows = nullptr, int row_stride = 0) {
   __shared__ __align__(16) float st_s[kMaxExperts];
   __shared__ uint2 nz_kid[kMaxExperts];   // nonzero entries: (order key, id), ids ascending
   __shared__ int wcnt[2][8];
@@ -215,10 +216,37 @@ __device__ inline int block_coreset_steps(int E, int k, int B, float top_p, HatF
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const bool live = tid < E;
 
-  // S_block = sum over the block's tokens (ascending) of TopKMask(s_i, k); 32 rows are
-  // fetched at a time so that their loads overlap
+  // S_block = sum over the block's tokens of TopKMask(s_i, k). With the rows given as an
+  // array (16-byte aligned, B and E multiples of 4): thread t sums experts 4 (t mod 64) ..
+  // + 3 over the t / 64-th quarter of the tokens (ascending, 16-byte loads), and the four
+  // quarter sums of an expert are added in order; else every thread sums its expert over
+  // all tokens in ascending order, 32 rows fetched at a time so that their loads overlap
   float S = 0.f;
-  if (live) {
+  if (rows != nullptr && B % 4 == 0 && E % 4 == 0 && B >= 8) {
+    __shared__ __align__(16) float qsum[4][kMaxExperts];
+    const int eq = 4 * (tid & 63), rq = tid >> 6, nq = B / 4;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (eq < E) {
+      const float* r0 = rows + (size_t)(rq * nq) * row_stride + eq;
+      for (int i0 = 0; i0 < nq; i0 += 8) {
+        float4 h[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (i0 + u < nq) h[u] = *reinterpret_cast<const float4*>(r0 + (size_t)(i0 + u) * row_stride);
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+          if (i0 + u < nq) {
+            a.x += h[u].x;
+            a.y += h[u].y;
+            a.z += h[u].z;
+            a.w += h[u].w;
+          }
+      }
+    }
+    *reinterpret_cast<float4*>(&qsum[rq][eq]) = a;
+    __syncthreads();
+    if (live) S = ((qsum[0][tid] + qsum[1][tid]) + qsum[2][tid]) + qsum[3][tid];
+  } else if (live) {
     for (int i0 = 0; i0 < B; i0 += 32) {
       float h[32];
 #pragma unroll
@@ -470,12 +498,13 @@ template <class HatFn, class ProbFn, class OutFn>
 __device__ inline void block_route_steps(int E, int kb, int k, int B, float top_p, HatFn hat,
                                          ProbFn prob, OutFn out, int32_t* __restrict__ coreset,
                                          int32_t* __restrict__ coreset_size,
-                                         uint32_t* __restrict__ spec = nullptr) {
+                                         uint32_t* __restrict__ spec = nullptr,
+                                         const float* hat_rows = nullptr) {
   __shared__ int order[kMaxExperts];
   // block top-k (p <= 0, the coreset is every token's routing): published for the expert
   // launch as soon as it is known
   const int size = block_coreset_steps(E, kb, B, top_p, hat, order, coreset, coreset_size,
-                                       top_p <= 0.f && kb == k ? spec : nullptr);
+                                       top_p <= 0.f && kb == k ? spec : nullptr, hat_rows, E);
   DMOE_STAMP(25);
   mask_topk_warps(k, B, size, order, prob, out);
   __syncthreads();
@@ -502,7 +531,7 @@ __device__ inline void block_route_cta(int b, const float* probs, const float* p
       },
       coreset != nullptr ? coreset + (size_t)b * E : nullptr,
       coreset_size != nullptr ? coreset_size + b : nullptr,
-      spec != nullptr ? spec + (size_t)b * spec_words(k) : nullptr);
+      spec != nullptr ? spec + (size_t)b * spec_words(k) : nullptr, probs_hat + r0 * E);
 }
 
 }  // namespace dmoe
