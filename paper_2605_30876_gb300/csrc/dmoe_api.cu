@@ -134,7 +134,10 @@ Workspace plan_workspace(const dmoe_layer_desc& d) {
   const bool dec = experts_decode_ok((int)T, (int)dm, (int)I, (int)Is);
   w.hdense = take(dec ? 2 * (E + 1) * (size_t)((T + 15) / 16 * 16) * (I > Is ? I : Is) : 0);
   w.spec = take(dec || d.mode == DMOE_ROUTE_BLOCK
-                    ? sizeof(uint32_t) * d.n_blocks * spec_words((int)k) : 0);
+                    ? sizeof(uint32_t) * d.n_blocks *
+                          (spec_words((int)k) > kSpecMaskWords ? spec_words((int)k)
+                                                               : kSpecMaskWords)
+                    : 0);
   const size_t nchunks = (T + 31) / 32;
   w.disp_bits = take(sizeof(uint32_t) * nchunks * E);
   w.disp_base = take(sizeof(int32_t) * nchunks * E);
@@ -210,9 +213,11 @@ dmoe_status run_router(const dmoe_layer_desc* desc, const void* x, const float* 
                        int32_t* coreset_size, float* probs, void* ws, const Workspace& plan,
                        cudaStream_t s, const L2Prefetch& shared_pf = L2Prefetch(),
                        const DispatchArgs* dsp = nullptr, uint32_t* spec_words = nullptr,
-                       int32_t* ready_clear = nullptr, int n_ready_clear = 0) {
+                       int32_t* ready_clear = nullptr, int n_ready_clear = 0,
+                       bool spec_mask = false) {
   RouterArgs a{};
   a.spec_words = spec_words;
+  a.spec_mask = spec_mask;
   a.ready_clear = ready_clear;
   a.n_ready_clear = n_ready_clear;
   a.x = static_cast<const __nv_bfloat16*>(x);
@@ -273,8 +278,9 @@ dmoe_status run_experts(const dmoe_layer_desc* desc, const void* x, const void* 
                         bool shared_prefetched = false, uint32_t* spec_words = nullptr,
                         bool gathered = false, int32_t* topk_idx = nullptr,
                         int32_t* pos_out = nullptr, int32_t* n_unique_out = nullptr,
-                        int32_t* unique_ids_out = nullptr) {
+                        int32_t* unique_ids_out = nullptr, bool spec_mask = false) {
   ExpertArgs a{};
+  a.spec_mask = spec_mask;
   a.topk_idx = topk_idx;
   a.pos_out = pos_out;
   a.n_unique_out = n_unique_out;
@@ -465,15 +471,26 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
     dsp.zero = at<int32_t>(workspace, plan.h_ready);
     dsp.n_zero = experts_ready_counters(T_all, desc->n_experts, plan.n_max);
   }
-  // block top-k through the decode-size launches: the expert launch starts streaming on the
-  // early-published coresets, before the routing launch ends (only when every token keeps
-  // the whole coreset, so that the coresets' union is the unique set)
+  // block routing through the decode-size launches: the expert launch starts streaming on
+  // the early-published coresets, before the routing launch ends. With block top-k (every
+  // token keeps the whole coreset) their union is the unique set, published as ids. With
+  // fewer experts per token than the coreset holds, or a small p over blocks of 32 or more
+  // tokens, the union contains the unique set and is seldom larger (most members are kept
+  // by some token of the block): published as masks, and the down epilogue takes each
+  // group's rows from the dispatch once it is complete. Larger p or smaller blocks leave
+  // many members unkept: streaming them cost more than the early start saved.
   const int T = desc->n_blocks * desc->block_size;
   uint32_t* spec_w = nullptr;
-  if (desc->mode == DMOE_ROUTE_BLOCK && desc->top_p <= 0.f && mask_top_k(*desc) == desc->top_k &&
-      route_cluster_ok(T, desc->d_model, desc->n_experts) &&
+  bool spec_mask = false;
+  if (desc->mode == DMOE_ROUTE_BLOCK && route_cluster_ok(T, desc->d_model, desc->n_experts) &&
       experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared)) {
-    spec_w = at<uint32_t>(workspace, plan.spec);
+    const bool ids = desc->top_p <= 0.f && mask_top_k(*desc) == desc->top_k;
+    const bool masks = (desc->top_p <= 0.f && !ids) ||
+                       (desc->top_p > 0.f && desc->top_p <= 0.5f && desc->block_size >= 32);
+    if (ids || masks) {
+      spec_w = at<uint32_t>(workspace, plan.spec);
+      spec_mask = masks;
+    }
   }
   if (spec_general) {
     spec_w = at<uint32_t>(workspace, plan.spec);
@@ -486,11 +503,11 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
                        false, idx, pos, nu, uid);
   }
   st = run_router(desc, x, w_r, bias, idx, gate, nullptr, nullptr, nullptr, workspace, plan, s,
-                  shared_pf, &dsp, spec_w);
+                  shared_pf, &dsp, spec_w, nullptr, 0, spec_mask);
   if (st != DMOE_OK) return st;
   return run_experts(desc, x, w_gate, w_up, w_down, ws_gate, ws_up, ws_down, gate, nu, uid, offs,
                      rows, pos, y, workspace, plan, s, /*shared_prefetched=*/true, spec_w,
-                     gathered);
+                     gathered, nullptr, nullptr, nullptr, nullptr, spec_mask);
 }
 
 dmoe_status dmoe_get_device_error(void* workspace, void* stream, int32_t* info) {

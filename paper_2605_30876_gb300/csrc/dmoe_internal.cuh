@@ -181,6 +181,11 @@ struct RouterArgs {
   // ids and a marker byte each, one 32-bit store per word (a word reads as zero until it is
   // complete; zero between calls); nullptr otherwise
   uint32_t* spec_words;
+  // spec_words hold every block's coreset as a mask instead (block routing with p > 0, or
+  // fewer experts per token than the coreset holds: the coresets' union then contains the
+  // unique experts): kSpecMaskWords words per block, the 256-bit member mask, then a marker
+  // stored with release semantics after it
+  bool spec_mask;
   // with spec_words on the general path: the gate/up tile counters of the expert launch that
   // follows, cleared by the block routing launch before it lets that launch start (the
   // dispatch launches, which clear them otherwise, do not run then)
@@ -262,6 +267,7 @@ struct ExpertArgs {
   // otherwise
   uint32_t* spec_words;
   int spec_blocks;
+  bool spec_mask;         // the words are coreset masks (RouterArgs::spec_mask)
   // general path with spec_words (block top-k): the expert launch writes the dispatch's
   // outputs from the published coresets and the routing's topk_idx
   const int32_t* topk_idx;
@@ -288,6 +294,8 @@ cudaError_t launch_combine(const ExpertArgs& a, cudaStream_t s, int32_t* zero = 
 
 // Words of one block's published coreset (three 8-bit ids and a marker byte per word).
 __host__ __device__ inline int spec_words(int k) { return (k + 2) / 3; }
+// words per block of a published coreset mask: the member mask, then the marker
+constexpr int kSpecMaskWords = kMaxExperts / 32 + 1;
 // Decode-sized forwards (T <= 64): one persistent launch over gate/up and down tiles of
 // every group, all tokens at once (no gather), then the combine.
 bool experts_decode_ok(int T, int d, int I, int Is);

@@ -83,6 +83,8 @@ struct DParams {
   const uint32_t* spec_words;   // block top-k: published coresets (spec_words(k) words per
                                 // block, three ids and a marker byte each), or nullptr
   int spec_blocks;
+  int spec_mask;             // the words are coreset masks (kSpecMaskWords per block): their
+                             // union contains the unique experts, whose rows the dispatch gives
   DevErrRecord* err;
   int T, d, E, k, I, Is;
   int imax;                  // max(I, Is): row length of hdense
@@ -213,6 +215,26 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       const uint64_t t0 = ptx::globaltimer_ns();
       for (;;) {
         bool all = true;
+        if (p.spec_mask) {
+          // masks: a block's words are read once its marker (stored last, with release
+          // semantics) is seen by an acquire load; or-ing a mask twice is harmless
+          for (int b = lane; b < p.spec_blocks; b += 32) {
+            const uint32_t* wb = p.spec_words + (size_t)b * kSpecMaskWords;
+            if (ld_acquire(reinterpret_cast<const int32_t*>(wb + kMaxExperts / 32)) == 0) {
+              all = false;
+              continue;
+            }
+#pragma unroll
+            for (int w = 0; w < kMaxExperts / 32; ++w) {
+              const uint32_t m = ld_relaxed_u32(wb + w);
+              if (m != 0u) {
+                if (32 * w >= p.E || (32 * w + 31 >= p.E && (m >> (p.E - 32 * w)) != 0u))
+                  bad = true;
+                atomicOr(&s_mask[w], m);
+              }
+            }
+          }
+        } else
         for (int i = lane; i < total; i += 32) {
           const uint32_t w = ld_relaxed_u32(p.spec_words + i);
           if (w == 0u) {
@@ -359,7 +381,24 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       g.n = p.T;
       return g;
     }
-    const int u = gi - p.has_shared;
+    int u = gi - p.has_shared;
+    if (spec && p.spec_mask) {
+      // the group is a member of the coresets' union; its rows are those of its place in
+      // the dispatch's unique list (ascending), none if no token kept it
+      const int nd = __ldcg(p.n_unique), e = g.e;
+      int lo = 0, hi = nd;
+      while (lo < hi) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldcg(p.unique_ids + mid) < e) lo = mid + 1;
+        else hi = mid;
+      }
+      if (lo >= nd || __ldcg(p.unique_ids + lo) != e) {
+        g.row0 = 0;
+        g.n = 0;
+        return g;
+      }
+      u = lo;
+    }
     int row0 = __ldcg(p.offsets + u);
     int n = __ldcg(p.offsets + u + 1) - row0;
     if (n < 0 || n > p.T || row0 < 0 || row0 + n > p.T * p.k) {
@@ -684,9 +723,18 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       // the rows of the dispatch from here on; the coresets must have given its unique list
       pdl_wait();
       if (warp == 2) {
-        bool bad = __ldcg(p.n_unique) != U;
-        for (int u = lane; u < U; u += 32)
-          if (__ldcg(p.unique_ids + u) != (int)s_spec[u]) bad = true;
+        // ids: the lists are equal; masks: the dispatch's list is inside the union
+        const int nd = __ldcg(p.n_unique);
+        bool bad = p.spec_mask ? (nd < 0 || nd > U) : nd != U;
+        if (!bad && p.spec_mask) {
+          for (int u = lane; u < nd; u += 32) {
+            const int e = __ldcg(p.unique_ids + u);
+            if (e < 0 || e >= p.E || ((s_mask[e >> 5] >> (e & 31)) & 1u) == 0u) bad = true;
+          }
+        } else if (!bad) {
+          for (int u = lane; u < U; u += 32)
+            if (__ldcg(p.unique_ids + u) != (int)s_spec[u]) bad = true;
+        }
         if (__any_sync(0xffffffffu, bad) && lane == 0)
           record_error(p.err, kErrBadDispatch, kAtDown, -1);
       }
@@ -914,6 +962,7 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   p.h_ready = a.h_ready;
   p.spec_words = a.spec_words;
   p.spec_blocks = a.spec_blocks;
+  p.spec_mask = a.spec_mask ? 1 : 0;
   p.err = a.err;
   p.T = a.T; p.d = a.d; p.E = a.E; p.k = a.k; p.I = a.I; p.Is = a.Is;
   p.imax = imax;
@@ -952,7 +1001,9 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   // the expert launch releases the combine at its end, after its wait for the routing
   // launch (which wrote the slot indices and gates): the combine may read them at once
   return launch_combine(a, s, a.h_ready, a.E + 1, a.spec_words,
-                        a.spec_words != nullptr ? a.spec_blocks * spec_words(a.k) : 0,
+                        a.spec_words != nullptr
+                            ? a.spec_blocks * (a.spec_mask ? kSpecMaskWords : spec_words(a.k))
+                            : 0,
                         /*meta_early=*/true);
 }
 

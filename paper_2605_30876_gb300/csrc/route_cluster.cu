@@ -453,10 +453,12 @@ route_cluster_kernel(const __grid_constant__ ClusterArgs f) {
           E, kc, B, a.top_p, [&](int i, int e) { return sHat[(t0 + i) * kMaxExperts + e]; }, order,
           a.coreset != nullptr ? a.coreset + (size_t)b * E : nullptr,
           a.coreset_size != nullptr ? a.coreset_size + b : nullptr,
-          a.spec_words != nullptr && a.top_p <= 0.f && kc == k
+          a.spec_words != nullptr && !a.spec_mask && a.top_p <= 0.f && kc == k
               ? a.spec_words + (size_t)b * spec_words(k)
               : nullptr,
           sHat + (size_t)t0 * kMaxExperts, kMaxExperts);
+      if (a.spec_words != nullptr && a.spec_mask && warp == 0)
+        publish_coreset_mask(a.spec_words + (size_t)b * kSpecMaskWords, order, size);
       CT_AT(25);
       // the coreset to the scoring warp of every token of the block (token t: CTA t / 8,
       // warp t mod 8): size, then the members in sorted order

@@ -182,6 +182,35 @@ __device__ inline void token_route_warp(const float* lrow, int nsum, size_t pstr
   }
 }
 
+// A block's coreset for the expert launch, by one warp: the 256-bit member mask (relaxed
+// stores), then the marker word with release semantics, so that a reader that acquires a
+// nonzero marker sees the whole mask.
+__device__ inline void publish_coreset_mask(uint32_t* __restrict__ words, const int* order,
+                                            int size) {
+  const int lane = threadIdx.x & 31;
+  uint32_t m[kMaxExperts / 32];
+#pragma unroll
+  for (int w = 0; w < kMaxExperts / 32; ++w) m[w] = 0u;
+  for (int i = lane; i < size; i += 32) {
+    const int e = order[i];
+#pragma unroll
+    for (int w = 0; w < kMaxExperts / 32; ++w)
+      if ((e >> 5) == w) m[w] |= 1u << (e & 31);
+  }
+  uint32_t mine = 0u;
+#pragma unroll
+  for (int w = 0; w < kMaxExperts / 32; ++w) {
+    const uint32_t all = __reduce_or_sync(0xffffffffu, m[w]);
+    if (lane == w) mine = all;
+  }
+  if (lane < kMaxExperts / 32)
+    asm volatile("st.relaxed.gpu.global.u32 [%0], %1;" ::"l"(words + lane), "r"(mine) : "memory");
+  __syncwarp();
+  if (lane == 0)
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(words + kMaxExperts / 32), "r"(1u)
+                 : "memory");
+}
+
 // ---------------------------------------------------------------- Algorithm 1, one block
 // Algorithm 1 for one block of B tokens by a CTA of 256 threads. The block's rows come
 // through accessors, so the same steps serve rows in global memory and rows spread over the
