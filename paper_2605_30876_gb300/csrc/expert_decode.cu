@@ -129,6 +129,9 @@ using ptx::tma_store_2d;
 // silu with the fast divide: H is rounded to bf16 right after
 __device__ __forceinline__ float silu_f(float z) { return __fdividef(z, 1.f + __expf(-z)); }
 
+// kMask: the coresets are published as masks (DParams::spec_mask), compiled separately so
+// that the launch on ids carries none of that code
+template <bool kMask>
 __global__ void __launch_bounds__(kThr, 1)
 moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DParams p) {
   extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -215,7 +218,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       const uint64_t t0 = ptx::globaltimer_ns();
       for (;;) {
         bool all = true;
-        if (p.spec_mask) {
+        if (kMask) {
           // masks: a block's words are read once its marker (stored last, with release
           // semantics) is seen by an acquire load; or-ing a mask twice is harmless
           for (int b = lane; b < p.spec_blocks; b += 32) {
@@ -382,7 +385,7 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       return g;
     }
     int u = gi - p.has_shared;
-    if (spec && p.spec_mask) {
+    if (kMask && spec) {
       // the group is a member of the coresets' union; its rows are those of its place in
       // the dispatch's unique list (ascending), none if no token kept it
       const int nd = __ldcg(p.n_unique), e = g.e;
@@ -725,8 +728,8 @@ moe_decode_kernel(const __grid_constant__ DMaps tm, const __grid_constant__ DPar
       if (warp == 2) {
         // ids: the lists are equal; masks: the dispatch's list is inside the union
         const int nd = __ldcg(p.n_unique);
-        bool bad = p.spec_mask ? (nd < 0 || nd > U) : nd != U;
-        if (!bad && p.spec_mask) {
+        bool bad = kMask ? (nd < 0 || nd > U) : nd != U;
+        if (!bad && kMask) {
           for (int u = lane; u < nd; u += 32) {
             const int e = __ldcg(p.unique_ids + u);
             if (e < 0 || e >= p.E || ((s_mask[e >> 5] >> (e & 31)) & 1u) == 0u) bad = true;
@@ -981,9 +984,12 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   {
     std::lock_guard<std::mutex> lock(mu);
     if (dev >= 31 || !(attr_dev_mask & (1 << dev))) {
-      cudaError_t e = cudaFuncSetAttribute(moe_decode_kernel,
+      cudaError_t e = cudaFuncSetAttribute(moe_decode_kernel<false>,
                                            cudaFuncAttributeMaxDynamicSharedMemorySize,
                                            max_smem_optin());
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(moe_decode_kernel<true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, max_smem_optin());
       if (e != cudaSuccess) return e;
       if (dev < 31) attr_dev_mask |= 1 << dev;
     }
@@ -994,8 +1000,11 @@ cudaError_t launch_experts_decode(const ExpertArgs& a, cudaStream_t s) {
   if (a.spec_words != nullptr && grid > 2 * kRouteClusterCtas) grid -= kRouteClusterCtas;
   if (grid > kMaxPersistentCtas) grid = kMaxPersistentCtas;
   prof_begin(DMOE_KERNEL_EXPERTS, s);
-  cudaError_t e = launch_ex(moe_decode_kernel, dim3(grid), dim3(kThr), smem, s,
-                            !prof_serial(DMOE_KERNEL_EXPERTS), m, p);
+  cudaError_t e =
+      p.spec_mask ? launch_ex(moe_decode_kernel<true>, dim3(grid), dim3(kThr), smem, s,
+                              !prof_serial(DMOE_KERNEL_EXPERTS), m, p)
+                  : launch_ex(moe_decode_kernel<false>, dim3(grid), dim3(kThr), smem, s,
+                              !prof_serial(DMOE_KERNEL_EXPERTS), m, p);
   prof_end(DMOE_KERNEL_EXPERTS, s);
   if (e != cudaSuccess) return e;
   // the expert launch releases the combine at its end, after its wait for the routing
