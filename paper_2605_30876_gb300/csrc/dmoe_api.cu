@@ -474,7 +474,7 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
   // block routing through the decode-size launches: the expert launch starts streaming on
   // the early-published coresets, before the routing launch ends. With block top-k (every
   // token keeps the whole coreset) their union is the unique set, published as ids. With
-  // fewer experts per token than the coreset holds, or a small p over blocks of 32 or more
+  // fewer experts per token than the coreset holds, or p <= 0.6 over blocks of 32 or more
   // tokens, the union contains the unique set and is seldom larger (most members are kept
   // by some token of the block): published as masks, and the down epilogue takes each
   // group's rows from the dispatch once it is complete. Larger p or smaller blocks leave
@@ -486,7 +486,7 @@ dmoe_status dmoe_layer_forward(const dmoe_layer_desc* desc, const void* x, const
       experts_decode_ok(T, desc->d_model, desc->d_ff, desc->d_ff_shared)) {
     const bool ids = desc->top_p <= 0.f && mask_top_k(*desc) == desc->top_k;
     const bool masks = (desc->top_p <= 0.f && !ids) ||
-                       (desc->top_p > 0.f && desc->top_p <= 0.5f && desc->block_size >= 32);
+                       (desc->top_p > 0.f && desc->top_p <= 0.6f && desc->block_size >= 32);
     if (ids || masks) {
       spec_w = at<uint32_t>(workspace, plan.spec);
       spec_mask = masks;
