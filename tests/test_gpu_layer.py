@@ -44,6 +44,11 @@ LAYER_CASES = {
     "spec_b8x16_noshared_k4_E64": LAYER.with_(block_size=16, n_blocks=8, d_ff_shared=0,
                                               top_k=4, n_experts=64),
     "spec_b20x16_k6_bias1": LAYER.with_(block_size=16, n_blocks=20, top_k=6, bias_scale=1.0),
+    # decode size, the coresets published as masks (the expert launch streams their union):
+    # two blocks at p = 0.4, and k = 1 of 8 over blocks of 4 tokens (at most 4 of a block's
+    # 8 coreset members are kept: the others take no rows from the dispatch)
+    "decode_masks_b2_p04": LAYER.with_(n_blocks=2, top_p=0.4),
+    "decode_masks_k1_of8": LAYER.with_(block_size=4, n_blocks=2, top_k=1, block_top_k=8),
     # the block-size x batch x bias grid: its smallest corner, uniform router bias
     "sweep_B4x1_bias0_block": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0),
     "sweep_B4x1_bias0_token": LAYER.with_(block_size=4, n_blocks=1, bias_scale=0.0,
@@ -273,3 +278,16 @@ def test_stack20_end_to_end():
     # reported figure: once a near-tie flips a block's coreset the two streams carry different
     # experts' outputs from there on; the bound only rules out a systematic drift
     assert err < 0.25
+
+
+def test_decode_masks_case_has_unkept_coreset_members():
+    """The k = 1 of 8 case above streams coreset members that no token keeps (their groups
+    take no rows from the dispatch): the oracle's coresets' union is larger than its set of
+    routed experts, so the output parity case exercises that path."""
+    shape = LAYER_CASES["decode_masks_k1_of8"]
+    dev, host = P.make(shape, seed=3)
+    orc = P.oracle_routing(shape, host)
+    union = set(np.concatenate([np.asarray(c) for c in orc.coresets]).tolist())
+    routed = set(np.unique(orc.idx).tolist())
+    assert routed <= union and len(union) > len(routed), (len(union), len(routed))
+
